@@ -1,0 +1,227 @@
+"""Seeded synthetic inputs for PCTree drafting rounds.
+
+This module is shared by the tests, the benchmark and the smoke check. It holds
+no part of the drafting method's arithmetic (no Markov head, no softmax, no
+selection): it only draws the inputs a drafting round consumes, with the shapes
+and value distributions of Qwen3-shaped DSpark drafters (Sec. 5.1, Table 6;
+Appendix A).  Both the oracle and the CUDA path read the arrays made here.
+
+Draw order, per workload and seed (numpy PCG64 via ``SeedSequence(seed)``):
+
+* ``SeedSequence(seed).spawn(1 + batch)``: child 0 draws the Markov-head
+  weights, child ``1 + r`` draws everything that belongs to request ``r``.
+* head (child 0): ``E_in`` then ``W_out``, each ``[V][H]`` drawn in row chunks
+  of ``_CHUNK_ROWS`` rows as float32 standard normals times the head scale;
+  bf16 workloads round each value to bf16 (round to nearest even).
+* request ``r``: base-logit noise ``[B][V]`` float32 normals; then the
+  per-depth structure (planted tokens, or Zipf rank permutations); then the
+  per-depth temperature coins (mixed-temperature workloads only); then the
+  root token; then, per depth, the target coin and the target's fallback token.
+
+The target's greedy token ``g[r][d]`` (the token the target model wants at
+draft depth ``d+1``) is a stand-in for the target model's forward, which is
+outside the drafting round: with probability ``target_p`` it is the
+generator's own "likely" token for that depth (the planted token, or the
+argmax of the base logits ``L_d``), otherwise a uniform token.  A node ``i``
+of a drafted tree at depth ``t`` then receives ``target[i] = g[r][t]``.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import Dict, Optional
+
+import numpy as np
+
+_CHUNK_ROWS = 8192
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    """One drafting-round workload: shapes, hyper-parameters and input recipe."""
+
+    name: str
+    V: int              # vocabulary size |V|
+    H: int              # Markov-head rank (hidden size of E_in / W_out)
+    B: int              # block size = number of sequential Markov stages
+    k: int              # local branching factor (per-parent top-k, frontier width)
+    N: int              # verification node budget, root included
+    batch: int          # independent requests drafted together
+    weight_dtype: str   # "bf16" or "f32"
+    logits: str         # "planted", "zipf" or "zipf_mixed_temp"
+    head_scale_e: float  # std of E_in entries
+    head_scale_w: float  # std of W_out entries
+    target_p: float     # probability that the target's token is the likely one
+    seed: int
+    pos_offset: int = 0  # verified-prefix length added to tree depths
+
+    def with_(self, **kw) -> "Workload":
+        return dataclasses.replace(self, **kw)
+
+    @property
+    def pool_size(self) -> int:
+        """Candidate pool size, root included: 1 + k + (B-1) k^2 (Sec. 4.1)."""
+        return 1 + self.k + (self.B - 1) * self.k * self.k
+
+    def describe(self) -> Dict[str, object]:
+        return {
+            "workload": self.name, "V": self.V, "H": self.H, "B": self.B,
+            "k": self.k, "N": self.N, "batch": self.batch,
+            "weights": self.weight_dtype, "logits": self.logits,
+        }
+
+
+def _tiny() -> Workload:
+    H = 64
+    return Workload("tiny_V1024_H64_B4_k4_N8", V=1024, H=H, B=4, k=4, N=8,
+                    batch=1, weight_dtype="f32", logits="planted",
+                    head_scale_e=1.0, head_scale_w=2.0 / np.sqrt(H),
+                    target_p=0.8, seed=0)
+
+
+WORKLOADS: Dict[str, Workload] = {
+    # small case the oracle finishes in milliseconds
+    "tiny": _tiny(),
+    # Qwen3-4B-shaped drafting rounds (V of the Qwen3 tokenizer, H=2560)
+    "4b_b7": Workload("qwen3_4b_V151936_H2560_B7_k8_N32_bs1", V=151936,
+                      H=2560, B=7, k=8, N=32, batch=1, weight_dtype="bf16",
+                      logits="zipf", head_scale_e=0.02, head_scale_w=0.02,
+                      target_p=0.85, seed=1),
+    "4b_b16": Workload("qwen3_4b_V151936_H2560_B16_k8_N64_bs1", V=151936,
+                       H=2560, B=16, k=8, N=64, batch=1, weight_dtype="bf16",
+                       logits="zipf", head_scale_e=0.02, head_scale_w=0.02,
+                       target_p=0.85, seed=2),
+    # DSpark-chain control on the same inputs as 4b_b16 (k=1)
+    "4b_b16_chain": Workload("qwen3_4b_V151936_H2560_B16_k1_N16_bs1_chain",
+                             V=151936, H=2560, B=16, k=1, N=16, batch=1,
+                             weight_dtype="bf16", logits="zipf",
+                             head_scale_e=0.02, head_scale_w=0.02,
+                             target_p=0.85, seed=2),
+    # Qwen3-8B-shaped batched serving round
+    "8b_b7_bs16": Workload("qwen3_8b_V151936_H4096_B7_k8_N64_bs16", V=151936,
+                           H=4096, B=7, k=8, N=64, batch=16,
+                           weight_dtype="bf16", logits="zipf",
+                           head_scale_e=0.02, head_scale_w=0.02,
+                           target_p=0.85, seed=3),
+    # Qwen3-14B-shaped stress round (flat and peaked rows mixed per depth)
+    "14b_b16_bs32": Workload("qwen3_14b_V151936_H5120_B16_k16_N128_bs32",
+                             V=151936, H=5120, B=16, k=16, N=128, batch=32,
+                             weight_dtype="bf16", logits="zipf_mixed_temp",
+                             head_scale_e=0.02, head_scale_w=0.02,
+                             target_p=0.85, seed=4),
+}
+
+
+def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round float32 values to bf16 (nearest, ties to even); return the bits."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
+    rounded = (u + np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1)))
+    return (rounded >> np.uint32(16)).astype(np.uint16)
+
+
+def bf16_bits_to_f32(bits: np.ndarray) -> np.ndarray:
+    """Widen bf16 bit patterns to float32 (exact)."""
+    return (bits.astype(np.uint32) << np.uint32(16)).view(np.float32)
+
+
+def _draw_matrix(rng: np.random.Generator, V: int, H: int, scale: float,
+                 dtype: str) -> np.ndarray:
+    out = np.empty((V, H), dtype=np.uint16 if dtype == "bf16" else np.float32)
+    for r0 in range(0, V, _CHUNK_ROWS):
+        r1 = min(V, r0 + _CHUNK_ROWS)
+        blk = rng.standard_normal((r1 - r0, H), dtype=np.float32)
+        blk *= np.float32(scale)
+        out[r0:r1] = f32_to_bf16_bits(blk) if dtype == "bf16" else blk
+    return out
+
+
+@dataclasses.dataclass
+class RoundInputs:
+    """Host arrays for one drafting round (all requests)."""
+
+    wl: Workload
+    L: np.ndarray          # [batch][B][V] float32 base logits
+    E_in: np.ndarray       # [V][H] uint16 (bf16 bits) or float32
+    W_out: np.ndarray      # [V][H] uint16 (bf16 bits) or float32
+    root: np.ndarray       # [batch] int32
+    greedy: np.ndarray     # [batch][B+1] int32: target's token after depth t
+    likely: np.ndarray     # [batch][B] int32: generator's likely token per depth
+
+
+def draw_head(wl: Workload, seed: Optional[int] = None):
+    """Markov-head weights ``(E_in, W_out)`` for a workload."""
+    ss = np.random.SeedSequence(wl.seed if seed is None else seed)
+    rng = np.random.default_rng(ss.spawn(1 + wl.batch)[0])
+    E_in = _draw_matrix(rng, wl.V, wl.H, wl.head_scale_e, wl.weight_dtype)
+    W_out = _draw_matrix(rng, wl.V, wl.H, wl.head_scale_w, wl.weight_dtype)
+    return E_in, W_out
+
+
+def draw_request(wl: Workload, r: int, seed: Optional[int] = None):
+    """Base logits, root token and target tokens of request ``r``.
+
+    Returns ``(L [B][V] f32, root, greedy [B+1], likely [B])``; ``greedy[t]``
+    is the target's token after a node at depth ``t`` (``t = 0`` is the root).
+    """
+    ss = np.random.SeedSequence(wl.seed if seed is None else seed)
+    rng = np.random.default_rng(ss.spawn(1 + wl.batch)[1 + r])
+    B, V = wl.B, wl.V
+    noise = rng.standard_normal((B, V), dtype=np.float32)
+    if wl.logits == "planted":
+        # 3 N(0,1) with a +6 spike at one uniformly drawn token per depth
+        L = noise * np.float32(3.0)
+        likely = rng.integers(0, V, size=B)
+        L[np.arange(B), likely] += np.float32(6.0)
+    elif wl.logits in ("zipf", "zipf_mixed_temp"):
+        # 4 N(0,1) plus a Zipf(s=1.1) log-rank boost, ranks a random
+        # permutation per depth: boost(v) = -1.1 ln rank_d(v)
+        L = noise * np.float32(4.0)
+        for d in range(B):
+            rank = rng.permutation(V).astype(np.float32) + np.float32(1.0)
+            L[d] -= np.float32(1.1) * np.log(rank)
+        if wl.logits == "zipf_mixed_temp":
+            # per depth: flat rows (temperature 2.0) or peaked (0.3), 50/50
+            flat = rng.random(B) < 0.5
+            temp = np.where(flat, np.float32(2.0), np.float32(0.3))
+            L = L / temp[:, None].astype(np.float32)
+        likely = np.argmax(L, axis=1)
+    else:
+        raise ValueError(f"unknown logits recipe {wl.logits!r}")
+    root = int(rng.integers(0, V))
+    coin = rng.random(B) < wl.target_p
+    fallback = rng.integers(0, V, size=B + 1)
+    # entry B is the token after a fully drafted block (bonus position)
+    greedy = np.concatenate([np.where(coin, likely, fallback[:B]),
+                             fallback[B:]])
+    return (np.ascontiguousarray(L, dtype=np.float32), root,
+            greedy.astype(np.int32), likely.astype(np.int32))
+
+
+def draw_round(wl: Workload, seed: Optional[int] = None,
+               requests: Optional[range] = None) -> RoundInputs:
+    """All inputs of one drafting round.  ``requests`` limits the requests
+    drawn (the head is always drawn in full)."""
+    E_in, W_out = draw_head(wl, seed)
+    reqs = range(wl.batch) if requests is None else requests
+    Ls, roots, greedy, likely = [], [], [], []
+    for r in reqs:
+        L, root, g, lk = draw_request(wl, r, seed)
+        Ls.append(L)
+        roots.append(root)
+        greedy.append(g)
+        likely.append(lk)
+    return RoundInputs(wl, np.stack(Ls), E_in, W_out,
+                       np.asarray(roots, dtype=np.int32),
+                       np.stack(greedy), np.stack(likely))
+
+
+def target_for_tree(greedy: np.ndarray, depth: np.ndarray) -> np.ndarray:
+    """Per-node target tokens of a drafted tree: ``target[i] = g[depth[i]]``.
+
+    ``greedy`` is ``[batch][B+1]``, ``depth`` is ``[batch][N]`` (-1 for
+    unused rows, which receive -1).
+    """
+    out = np.full(depth.shape, -1, dtype=np.int32)
+    for r in range(depth.shape[0]):
+        valid = (depth[r] >= 0) & (depth[r] < greedy.shape[1])
+        out[r, valid] = greedy[r, depth[r, valid]]
+    return out
