@@ -1,0 +1,390 @@
+#!/usr/bin/env python
+"""Benchmark: PCTree drafting rounds on one GB300 per process.
+
+One step = one whole drafting round of the Qwen3-4B-shaped workload
+(V=151936, H=2560 bf16 head, B=16 stages, k=8, N=64, one request): B Markov
+projections + log-softmax/top-k + merges, the global top-N and packing, then
+the greedy accept walk against a synthetic target.  Inputs are resident in HBM
+when the timed region starts; W_out (778 MB) is streamed once per stage, far
+larger than L2, and the base logits rotate over 16 seeded request sets.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Under torchrun each rank drafts its own requests (independent replicas, no
+collective on the data path); rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from workloads import WORKLOADS, draw_head, draw_request  # noqa: E402
+
+METRIC = ("tree-draft rounds/sec & µs/round (V=151936, B=16, N=64); "
+          "% of HBM roofline")
+N_SETS = 16          # rotating request inputs
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="4b_b16", choices=sorted(WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            return json.load(f), "measured"
+    return {"hbm_gbs": FALLBACK_HBM_GBS}, "fallback"
+
+
+def stage_bytes(wl, d):
+    """Algorithmic HBM bytes of stage d's Markov projection: W_out once, the
+    base logits of every request at depth d, the gathered parent rows."""
+    rows = wl.batch * (1 if d == 0 else wl.k)
+    return wl.V * wl.H * 2 + wl.batch * wl.V * 4 + rows * wl.H * 2
+
+
+def round_bytes(wl):
+    return sum(stage_bytes(wl, d) for d in range(wl.B))
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,"
+              "clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id):
+        self.proc = None
+        self.path = None
+        self.gpu_id = gpu_id
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200",
+                 "-i", str(self.gpu_id)], stdout=self.out,
+                stderr=subprocess.DEVNULL)
+        except (OSError, ValueError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.out.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                 "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4)
+                          if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+# ---------------------------------------------------------------------------
+# the oracle on the host cores (CPU baseline and reference arm)
+# ---------------------------------------------------------------------------
+
+def oracle_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads", 0) for i in threadpool_info()
+             if i.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    return os.cpu_count() or 1
+
+
+class OracleRunner:
+    """Runs the oracle's drafting round on prefixes of the workload's rounds:
+    a sample of `stages` of the B stages, scaled to whole rounds."""
+
+    def __init__(self, wl, E_in, W_out_bits, sets):
+        from oracle import pctree_oracle as O
+        self.O, self.wl, self.E_in, self.sets = O, wl, E_in, sets
+        self.W = O.as_f64(W_out_bits, wl.weight_dtype)   # weights load once
+
+    def run(self, i, stages):
+        L, root = self.sets[i % len(self.sets)]
+        self.O.draft(L[:stages], self.E_in, self.W, root, stages, self.wl.k,
+                     self.wl.N)
+
+
+def cpu_baseline(runner, wl, budget_s=12.0):
+    stages = min(wl.B, 4)
+    t0 = time.perf_counter()
+    n = 0
+    while True:
+        runner.run(n, stages)
+        n += 1
+        if time.perf_counter() - t0 >= budget_s:
+            break
+    dt = time.perf_counter() - t0
+    rounds = n * stages / wl.B
+    return {"value": rounds / dt, "unit": "rounds/s", "cores": oracle_threads(),
+            "kind": "oracle",
+            "sample": f"{n} oracle runs of the first {stages} of {wl.B} stages "
+                      f"of {wl.name} request rounds ({dt:.1f} s), scaled to "
+                      f"whole rounds by {wl.B}/{stages}"}
+
+
+def run_reference(args, wl, rank, world):
+    if rank != 0:
+        return
+    E_in, W_out = draw_head(wl)
+    sets = []
+    for r in range(4):
+        L, root, _, _ = draw_request(wl.with_(batch=N_SETS), r)
+        sets.append((L, root))
+    runner = OracleRunner(wl, E_in, W_out, sets)
+    stages = 1
+    for i in range(args.warmup):
+        runner.run(i, stages)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        runner.run(i, stages)
+    dt = time.perf_counter() - t0
+    value = args.steps * stages / wl.B / dt
+    line = {
+        "metric": METRIC, "value": value, "unit": "rounds/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": dt * 1e3 / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "impl": "reference",
+        "config": {"workload": wl.name, "V": wl.V, "H": wl.H, "B": wl.B,
+                   "k": wl.k, "N": wl.N, "batch": wl.batch,
+                   "step": f"one oracle stage ({stages} of {wl.B}) of a round"},
+        "cpu_baseline": {"value": value, "unit": "rounds/s",
+                         "cores": oracle_threads(), "kind": "oracle",
+                         "sample": f"{args.steps} single-stage oracle runs"},
+        "e2e": {"value": value, "unit": "rounds/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# the CUDA path
+# ---------------------------------------------------------------------------
+
+def run_ours(args, wl, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_02123_gb300 import pctree as P
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    E_bits, W_bits = draw_head(wl)
+    E = torch.from_numpy(E_bits.view(np.int16)).to(dev).view(torch.bfloat16)
+    W = torch.from_numpy(W_bits.view(np.int16)).to(dev).view(torch.bfloat16)
+    sets = []
+    for i in range(N_SETS):
+        r = rank * N_SETS + i
+        L, root, greedy, _ = draw_request(wl.with_(batch=N_SETS * world), r)
+        sets.append((L, root, greedy))
+    L_dev = [torch.from_numpy(L[None]).to(dev) for L, _, _ in sets]
+    root_dev = [torch.tensor([root], dtype=torch.int32, device=dev)
+                for _, root, _ in sets]
+    greedy_dev = [torch.from_numpy(g[None].astype(np.int64)).to(dev)
+                  for _, _, g in sets]
+    cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, wl.batch)
+    dr = P.Drafter(cfg, dev)
+    stream = torch.cuda.current_stream()
+
+    def target_of(i):
+        # synthetic target model: node i at depth t wants g[t] as its child
+        depth = dr.tree.depth.long().clamp_min(0)
+        return torch.gather(greedy_dev[i % N_SETS], 1, depth).to(torch.int32)
+
+    def step(i):
+        dr.draft(L_dev[i % N_SETS], E, W, root_dev[i % N_SETS], stream)
+        dr.accept(target_of(i), stream)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    dr.check_status()
+    if world > 1:
+        dist.barrier()
+
+    gpu_index = os.environ.get("CUDA_VISIBLE_DEVICES", str(local_rank))
+    gpu_index = gpu_index.split(",")[local_rank] if "," in gpu_index else gpu_index
+    clocks = ClockSampler(gpu_index)
+    clocks.start()
+    time.sleep(0.3)  # first sample lands inside the timed work below
+    P.pctree_profile_enable(True)
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    start.record(stream)
+    for i in range(args.steps):
+        step(i)
+    end.record(stream)
+    torch.cuda.synchronize()
+    launches, proj_ms = P.pctree_profile_collect()
+    P.pctree_profile_enable(False)
+    dr.check_status()
+    ms = start.elapsed_time(end)
+
+    # end to end through the public API: pinned host inputs in, tree out
+    L_host = [torch.from_numpy(L[None]).pin_memory() for L, _, _ in sets]
+    root_host = [torch.tensor([root], dtype=torch.int32).pin_memory()
+                 for _, root, _ in sets]
+    out_names = ("n_nodes", "tokens", "parent", "depth", "logp",
+                 "position_ids", "mask", "retrieve", "n_leaves", "status")
+    out_host = {n: torch.empty_like(getattr(dr.tree, n), device="cpu").pin_memory()
+                for n in out_names}
+    acc_host = [torch.empty_like(t, device="cpu").pin_memory()
+                for t in (dr.accepted_idx, dr.accepted_len, dr.bonus)]
+    h2d = L_host[0].numel() * 4 + root_host[0].numel() * 4
+    d2h = sum(t.numel() * t.element_size() for t in out_host.values()) + \
+        sum(t.numel() * t.element_size() for t in acc_host)
+    L_stage = torch.empty_like(L_dev[0])
+    root_stage = torch.empty_like(root_dev[0])
+
+    def e2e_step(i):
+        L_stage.copy_(L_host[i % N_SETS], non_blocking=True)
+        root_stage.copy_(root_host[i % N_SETS], non_blocking=True)
+        dr.draft(L_stage, E, W, root_stage, stream)
+        dr.accept(target_of(i), stream)
+        for n in out_names:
+            out_host[n].copy_(getattr(dr.tree, n), non_blocking=True)
+        for h, t in zip(acc_host, (dr.accepted_idx, dr.accepted_len, dr.bonus)):
+            h.copy_(t, non_blocking=True)
+        stream.synchronize()   # the caller reads the tree before the next round
+
+    for i in range(3):
+        e2e_step(i)
+    e_start = torch.cuda.Event(enable_timing=True)
+    e_end = torch.cuda.Event(enable_timing=True)
+    e_start.record(stream)
+    for i in range(args.steps):
+        e2e_step(i)
+    e_end.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e_start.elapsed_time(e_end)
+    clk = clocks.stop()
+
+    if world > 1:
+        t = torch.tensor([ms, e2e_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms, e2e_ms = float(t[0]), float(t[1])
+    if rank != 0:
+        return
+
+    rounds = args.steps * world * wl.batch
+    value = rounds / (ms / 1e3)
+    peaks, peak_kind = measured_peaks()
+    peak = float(peaks["hbm_gbs"])
+    bytes_round = round_bytes(wl)
+    proj_bytes = args.steps * bytes_round          # timed launches' bytes
+    achieved = proj_bytes / (proj_ms / 1e3) / 1e9 if proj_ms > 0 else None
+    us_round = ms * 1e3 / args.steps
+    passes = lambda rows: (rows + 255) // 256  # noqa: E731
+    kernels_per_step = 1 + sum(
+        passes(wl.batch * (1 if d == 0 else wl.k)) + 2 for d in range(wl.B)) + 1 + 1
+    line = {
+        "metric": METRIC, "value": value, "unit": "rounds/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded Qwen3-4B-shaped logits, random-init head)",
+        "config": {"workload": wl.name, "V": wl.V, "H": wl.H, "B": wl.B,
+                   "k": wl.k, "N": wl.N, "batch": wl.batch,
+                   "parallelism": f"replicas x{world}",
+                   "l2": "inputs larger than L2: W_out (778 MB) streamed per "
+                         "stage; base logits rotate over 16 request sets"},
+        "us_per_round": us_round,
+        "round_hbm_fraction": (bytes_round / (us_round * 1e-6) / 1e9) / peak,
+        "roofline": {"bound": "hbm", "kernel": "markov_tc_kernel",
+                     "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak if achieved else None,
+                     "peak_source": peak_kind,
+                     "launches": launches,
+                     "avg_launch_us": proj_ms * 1e3 / launches if launches else None,
+                     "traffic": None},
+        "e2e": {"value": rounds / (e2e_ms / 1e3), "unit": "rounds/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": kernels_per_step * args.steps,
+        "clocks": clk,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        E_bits_host, W_bits_host = E_bits, W_bits
+        runner = OracleRunner(wl, E_bits_host, W_bits_host,
+                              [(L, root) for L, root, _ in sets[:4]])
+        line["cpu_baseline"] = cpu_baseline(runner, wl)
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    wl = WORKLOADS[args.workload]
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, wl, rank, world)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    try:
+        run_ours(args, wl, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

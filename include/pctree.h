@@ -1,0 +1,215 @@
+/*
+ * pctree.h -- C ABI of the PCTree drafting-round library for NVIDIA GB300
+ * (sm_103a).
+ *
+ * One call, pctree_draft, runs a whole PCTree drafting round (Algorithm 1) for
+ * a batch of independent requests on one GPU: B sequential stages, each a
+ * batched parent-conditioned Markov-head evaluation over every frontier
+ * parent (Eq. 3), a vocabulary-wide log-softmax (Eq. 2), per-parent top-k
+ * children scored by their joint path log-probability (Eq. 4) and a
+ * layer-wise frontier prune (Sec. 4.1); then the global top-N selection under
+ * the node budget and the tree tensors (Sec. 4.2; Appendix A "Tensor
+ * implementation").  pctree_accept runs the greedy tree acceptance against
+ * the target model's tokens (Sec. 4.2; Appendix A).
+ *
+ * Conventions for every entry point:
+ *  - Pointers to tensors are DEVICE pointers owned by the caller; the library
+ *    never allocates device memory and keeps no pointer after returning.
+ *  - Work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *    stream) and runs asynchronously: outputs are valid once the stream has
+ *    reached this point.  The host returns without synchronising.
+ *  - A negative return value is an error found on the host before any work
+ *    was enqueued (argument checks) or a failed launch (PCTREE_ERR_CUDA).
+ *    Conditions found on the device (non-finite values, a bounded wait that
+ *    ran out, a root token out of range) are written to `out->status` on the
+ *    device; read it after the stream has synchronised.
+ *  - Tensors are dense and row-major ("C order") with the shapes stated.
+ *  - Thread-safety: calls on different streams may run concurrently if they
+ *    use different workspaces; the profiling switch is process-wide.
+ */
+#ifndef PCTREE_H_
+#define PCTREE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+/* Symbols of this header are the library's only exported names. */
+#if defined(__GNUC__)
+#define PCTREE_API __attribute__((visibility("default")))
+#else
+#define PCTREE_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  PCTREE_OK = 0,
+  PCTREE_ERR_INVALID_ARG = -1, /* a size, pointer, alignment or token is bad */
+  PCTREE_ERR_WORKSPACE = -2,   /* workspace NULL, misaligned or too small    */
+  PCTREE_ERR_CUDA = -3,        /* a CUDA call or launch failed               */
+  PCTREE_ERR_TIMEOUT = -4,     /* a bounded device-side wait ran out         */
+  PCTREE_ERR_NONFINITE = -5,   /* NaN/+inf input, or a depth with no finite
+                                  logit (probabilities undefined)            */
+  PCTREE_ERR_UNSUPPORTED = -6  /* shape outside the compiled limits          */
+} pctree_status;
+
+typedef enum { PCTREE_F32 = 0, PCTREE_BF16 = 1 } pctree_dtype;
+
+/* Compiled limits. */
+#define PCTREE_MAX_K 32        /* per-parent top-k and frontier width        */
+#define PCTREE_MAX_N 1024      /* node budget, root included                 */
+#define PCTREE_MAX_POOL 16384  /* 1 + k + (B-1) k^2 candidate nodes          */
+#define PCTREE_MAX_ROWS 4096   /* batch * k Markov rows per stage            */
+
+/*
+ * Round configuration.
+ *   V            vocabulary size |V|; 1 <= k <= V.
+ *   H            Markov-head rank.  BF16 weights need H % 8 == 0 (16-byte
+ *                rows for TMA); F32 weights take any H >= 1.
+ *   B            block size: number of sequential Markov stages and the
+ *                deepest drafted level (Sec. 4.1), 1 <= B.
+ *   k            local branching factor: children kept per parent and width
+ *                of the frontier (Sec. 4.1), 1 <= k <= PCTREE_MAX_K.
+ *   N            verification node budget including the root (Sec. 4.1),
+ *                1 <= N <= PCTREE_MAX_N.
+ *   batch        independent requests drafted together, 1 <= batch and
+ *                batch * k <= PCTREE_MAX_ROWS.
+ *   pos_offset   verified prefix length: position id = depth + pos_offset
+ *                (Appendix A).
+ *   weight_dtype storage type of both head matrices (pctree_dtype).
+ * The candidate pool holds 1 + k + (B-1) k^2 nodes (Sec. 4.1); it must not
+ * exceed PCTREE_MAX_POOL.
+ */
+typedef struct {
+  int32_t V, H, B, k, N, batch, pos_offset, weight_dtype;
+} pctree_config;
+
+/*
+ * Output tree tensors, one block per request.  Nodes are listed breadth
+ * first: by depth, then by the parent's index, then by token id; the root is
+ * node 0 and every node's parent has a smaller index.  Rows beyond
+ * n_nodes[r] hold -1 (logp: -inf; mask: 0).
+ *   n_nodes      [batch]          min(N, pool size)
+ *   tokens       [batch][N]       draft token of each node (root: root token)
+ *   parent       [batch][N]       index of the parent node; root -1
+ *   depth        [batch][N]       0 for the root, 1..B for drafted nodes
+ *   logp         [batch][N]       joint path log-probability s (Eq. 4); root 0
+ *   position_ids [batch][N]       depth + pos_offset; siblings share one
+ *   mask         [batch][N][N]    1 iff column j is row i or an ancestor of i
+ *                                 (the ancestor-only tree attention mask; the
+ *                                 verified prefix is always visible and not
+ *                                 part of this tensor)
+ *   retrieve     [batch][N][B+1]  one row per leaf, in leaf-index order: the
+ *                                 node indices from the root to the leaf,
+ *                                 -1 padded; rows >= n_leaves[r] are all -1
+ *   n_leaves     [batch]
+ *   status       [1]              device status word, set to PCTREE_OK at the
+ *                                 start of pctree_draft and to the first
+ *                                 device-detected error code; required
+ *   pool_token   [batch][P]       optional (NULL: not written).  The
+ *   pool_parent  [batch][P]       candidate pool in creation order
+ *   pool_logp    [batch][P]       (P = pctree_pool_capacity): token, parent's
+ *                                 pool id (-1 for the root) and joint score.
+ *                                 Node ids: root 0, then layer by layer; in
+ *                                 a layer, the parent's frontier slot major
+ *                                 and the child's rank minor.
+ */
+typedef struct {
+  int32_t* n_nodes;
+  int32_t* tokens;
+  int32_t* parent;
+  int32_t* depth;
+  float* logp;
+  int32_t* position_ids;
+  uint8_t* mask;
+  int32_t* retrieve;
+  int32_t* n_leaves;
+  int32_t* status;
+  int32_t* pool_token;
+  int32_t* pool_parent;
+  float* pool_logp;
+} pctree_tree;
+
+/* Checks a configuration against the rules above; no GPU work. */
+PCTREE_API pctree_status pctree_check_config(const pctree_config* cfg);
+
+/* Candidate pool size 1 + k + (B-1) k^2 (Sec. 4.1); 0 for a bad config. */
+PCTREE_API int32_t pctree_pool_capacity(const pctree_config* cfg);
+
+/* Device workspace bytes pctree_draft needs for `cfg` (256-byte aligned
+ * start required); 0 for a bad config.  The workspace holds the per-stage
+ * Markov rows, the stage logits, the per-chunk softmax/top-k partials, the
+ * candidate pool and the frontier; its contents are scratch between calls. */
+PCTREE_API size_t pctree_workspace_bytes(const pctree_config* cfg);
+
+/*
+ * One PCTree drafting round (Algorithm 1; Eqs. 2-4; Sec. 4.2; Appendix A).
+ *   base_logits  [batch][B][V] float32: the backbone's shared logits L_d per
+ *                request (Sec. 3.2 "Parallel backbone"); -inf allowed.
+ *   head_emb     [V][H] E_in  (weight_dtype), 16-byte aligned: Markov-head
+ *                input rows, one per parent token.
+ *   head_out     [V][H] W_out (weight_dtype), 16-byte aligned: Markov-head
+ *                output projection.  The head's bias for parent p is
+ *                Markov(p)[v] = sum_h W_out[v][h] * E_in[p][h] (Sec. 3.2,
+ *                "low-rank Markov head"), accumulated in float32.
+ *   root_token   [batch] int32: the last verified token x_t of each request;
+ *                out of range -> status PCTREE_ERR_INVALID_ARG.
+ *   out          output tensors (see pctree_tree); all non-optional pointers
+ *                required.
+ *   workspace    device scratch of at least pctree_workspace_bytes(cfg)
+ *                bytes, 256-byte aligned, not used concurrently by another
+ *                call.
+ * Ranking rules: children of a parent by (log pi desc, token asc); the
+ * frontier by (score desc, id asc); the global budget by (score desc, depth
+ * asc, id asc), all on float32 scores accumulated along paths in float64.
+ * Errors: PCTREE_ERR_INVALID_ARG / _WORKSPACE / _UNSUPPORTED before any work;
+ * PCTREE_ERR_CUDA if a launch fails.
+ */
+PCTREE_API pctree_status pctree_draft(const pctree_config* cfg, const float* base_logits,
+                           const void* head_emb, const void* head_out,
+                           const int32_t* root_token, const pctree_tree* out,
+                           void* workspace, size_t workspace_bytes,
+                           void* stream);
+
+/*
+ * Greedy tree acceptance (Sec. 4.2 "standard greedy tree rule"; Appendix A).
+ * Starting at the root, repeatedly accept the child whose token equals the
+ * target model's token at the current node, until no child matches.
+ *   tree           the tokens, parent and n_nodes of a drafted tree (other
+ *                  fields unused)
+ *   target_tokens  [batch][N] int32: the target's greedy token at each node's
+ *                  position, i.e. the token it wants as that node's child
+ *   accepted_idx   [batch][B+1] out: node indices of the accepted path from
+ *                  the root, -1 padded
+ *   accepted_len   [batch] out: accepted draft tokens (tau = len + 1 with the
+ *                  bonus token, Sec. 5.1)
+ *   bonus_token    [batch] out: the target's token at the last accepted node
+ */
+PCTREE_API pctree_status pctree_accept(const pctree_config* cfg, const pctree_tree* tree,
+                            const int32_t* target_tokens,
+                            int32_t* accepted_idx, int32_t* accepted_len,
+                            int32_t* bonus_token, void* stream);
+
+/* Human-readable name of a status code. */
+PCTREE_API const char* pctree_status_string(int32_t status);
+
+/*
+ * Kernel timing for roofline reports.  While enabled, pctree_draft records a
+ * CUDA event before and after every Markov-projection launch on the call's
+ * stream (at most 8192 launches are recorded).  pctree_profile_collect
+ * waits for the recorded events, returns the number of launches and their
+ * summed duration in milliseconds, and clears the record.  Not thread-safe.
+ */
+PCTREE_API pctree_status pctree_profile_enable(int32_t on);
+PCTREE_API pctree_status pctree_profile_collect(int64_t* launches, double* total_ms);
+
+/* ABI version (major * 100 + minor). */
+PCTREE_API int32_t pctree_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PCTREE_H_ */

@@ -32,8 +32,10 @@ Readings of the paper taken here (each also listed in the design notes):
   tokens).  ``tau = accepted_len + 1`` counts the bonus token (Sec. 5.1).
 * Unused output rows (fewer than N pool nodes): token / parent / depth /
   position id -1, logp -inf, mask 0, retrieve -1.
-* Non-finite inputs: NaN or +inf anywhere, or a depth whose logits are all
-  -inf, raise ``NonFiniteInput``; -inf logits are legal (probability 0).
+* Non-finite inputs: NaN or +inf base logits, a depth whose logits are all
+  -inf, or head weights that make a stage logit NaN or infinite where the
+  base logit is finite, raise ``NonFiniteInput``; -inf base logits are legal
+  (probability 0).
 
 Replay of near-tie decisions.  The CUDA path computes in float32 and so can
 order two candidates differently from this float64 oracle when their values
@@ -57,8 +59,10 @@ constructed targets.  No function here is "parity unpinned".
 """
 from __future__ import annotations
 
+import concurrent.futures
 import dataclasses
 import math
+import os
 from typing import Dict, List, Optional, Sequence, Set, Tuple
 
 import numpy as np
@@ -83,9 +87,26 @@ class ParityViolation(AssertionError):
 
 def decode_bf16(bits: np.ndarray) -> np.ndarray:
     """bf16 bit patterns (uint16) -> float64.  bf16 is the top half of an
-    IEEE binary32, so shifting the pattern left by 16 bits is exact."""
-    b = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)
-    return b.view(np.float32).astype(np.float64)
+    IEEE binary32, so shifting the pattern left by 16 bits is exact.  Large
+    arrays are decoded in independent slices on several threads."""
+    src = np.ascontiguousarray(bits, dtype=np.uint16)
+    out = np.empty(src.shape, dtype=np.float64)
+    fin, fout = src.reshape(-1), out.reshape(-1)
+    step = 1 << 22
+
+    def part(i: int) -> None:
+        sl = slice(i, min(i + step, fin.size))
+        wide = fin[sl].astype(np.uint32) << np.uint32(16)
+        fout[sl] = wide.view(np.float32)
+
+    starts = range(0, fin.size, step)
+    if len(starts) <= 1:
+        for i in starts:
+            part(i)
+    else:
+        with concurrent.futures.ThreadPoolExecutor(os.cpu_count() or 1) as ex:
+            list(ex.map(part, starts))
+    return out
 
 
 def as_f64(w: np.ndarray, dtype: str) -> np.ndarray:
@@ -97,6 +118,13 @@ def as_f64(w: np.ndarray, dtype: str) -> np.ndarray:
     raise ValueError(dtype)
 
 
+def _values(a: np.ndarray) -> np.ndarray:
+    """float64 values of an array stored as bf16 bits (uint16) or floats."""
+    if a.dtype == np.uint16:
+        return decode_bf16(a)
+    return np.asarray(a, dtype=np.float64)
+
+
 # ----------------------------------------------------------------------------
 # Eq. 3: one batched Markov call; Eq. 2: log-softmax
 # ----------------------------------------------------------------------------
@@ -104,9 +132,10 @@ def as_f64(w: np.ndarray, dtype: str) -> np.ndarray:
 def markov_bias(E_in: np.ndarray, W_out: np.ndarray,
                 parents: Sequence[int]) -> np.ndarray:
     """Markov(P) for the stacked parent tokens P (Eq. 3): one row per parent,
-    ``Markov(p)[v] = sum_h W_out[v, h] * E_in[p, h]``."""
-    X = E_in[np.asarray(parents, dtype=np.int64)]       # [b][H]
-    return X @ W_out.T                                   # [b][V]
+    ``Markov(p)[v] = sum_h W_out[v, h] * E_in[p, h]``.  Weights may be given
+    as bf16 bits (uint16) or floats; the product is taken in float64."""
+    X = _values(E_in[np.asarray(parents, dtype=np.int64)])   # [b][H]
+    return X @ _values(W_out).T                               # [b][V]
 
 
 def stage_logits(L_d: np.ndarray, E_in: np.ndarray, W_out: np.ndarray,
@@ -265,14 +294,19 @@ class Round:
     markov_calls: List[int]   # batch size b_d of each Markov call
 
 
-def _check_finite(L: np.ndarray, E_in: np.ndarray, W_out: np.ndarray) -> None:
-    for name, a in (("base logits", L), ("E_in", E_in), ("W_out", W_out)):
-        if np.isnan(a).any() or np.isposinf(a).any():
-            raise NonFiniteInput(f"{name} holds NaN or +inf")
-    if np.isneginf(E_in).any() or np.isneginf(W_out).any():
-        raise NonFiniteInput("head weights hold -inf")
+def _check_logits(L: np.ndarray) -> None:
+    if np.isnan(L).any() or np.isposinf(L).any():
+        raise NonFiniteInput("base logits hold NaN or +inf")
     if not np.isfinite(L).any(axis=1).all():
         raise NonFiniteInput("a depth has no finite base logit")
+
+
+def _check_stage(Z: np.ndarray, L_d: np.ndarray) -> None:
+    """A non-finite head weight shows up as a NaN / infinite stage logit where
+    the base logit is finite."""
+    bad = np.isnan(Z) | (np.isinf(Z) & np.isfinite(L_d)[None, :]) | np.isposinf(Z)
+    if bad.any():
+        raise NonFiniteInput("non-finite Markov bias")
 
 
 def draft(L: np.ndarray, E_in: np.ndarray, W_out: np.ndarray, root: int,
@@ -280,13 +314,15 @@ def draft(L: np.ndarray, E_in: np.ndarray, W_out: np.ndarray, root: int,
           hint: Optional[Choices] = None, delta: float = DELTA) -> Round:
     """One PCTree drafting round for one request.
 
-    ``L`` is ``[B][V]`` (float32 or float64), ``E_in``/``W_out`` are float64
-    ``[V][H]``.  Returns the candidate pool, the selection and the packed tree.
+    ``L`` is ``[B][V]`` (float32 or float64); ``E_in``/``W_out`` are ``[V][H]``
+    as floats or bf16 bits (uint16; pass ``W_out`` pre-decoded with
+    ``as_f64`` to decode it once for many rounds).  Returns the candidate
+    pool, the selection and the packed tree.
     """
     V = L.shape[1]
     if not (1 <= k <= V and N >= 1 and B >= 1 and 0 <= root < V):
         raise ValueError("invalid round parameters")
-    _check_finite(np.asarray(L, dtype=np.float64), E_in, W_out)
+    _check_logits(np.asarray(L, dtype=np.float64))
     pool = Pool([root], [-1], [0], [0.0], [()])       # root: score 0, id 0
     frontier = [0]
     margins = {"children": math.inf, "frontier": math.inf, "global": math.inf}
@@ -296,6 +332,7 @@ def draft(L: np.ndarray, E_in: np.ndarray, W_out: np.ndarray, root: int,
         parents = [pool.token[i] for i in frontier]
         calls.append(len(parents))
         Z = stage_logits(L[d], E_in, W_out, parents)  # one batched call, Eq. 3
+        _check_stage(Z, L[d])
         layer: List[int] = []
         for slot, pid in enumerate(frontier):
             z = Z[slot]

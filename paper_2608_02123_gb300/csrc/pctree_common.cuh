@@ -1,0 +1,177 @@
+// Shared declarations of the PCTree CUDA library: workspace layout, ranking
+// keys, warp-level top-k lists and the launchers each translation unit
+// provides to the host API.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "pctree.h"
+
+namespace pct {
+
+constexpr unsigned kFull = 0xffffffffu;
+constexpr int kChunk = 2048;          // vocabulary entries per partials CTA
+constexpr int kChunkThreads = 256;
+
+// ---------------------------------------------------------------------------
+// workspace layout (host and device agree through this struct)
+// ---------------------------------------------------------------------------
+
+struct Layout {
+  int rows_max;   // batch * k: Markov rows of a full stage
+  int rows_pad;   // rows of the X buffer (multiple of 16)
+  int bn;         // MMA N tile (rows per projection pass)
+  int ldz;        // row stride of the stage logits Z, in floats
+  int n_chunks;   // vocabulary chunks per row in the partials pass
+  int P;          // candidate pool capacity per request
+  int x_elem;     // bytes per X element
+  size_t off_x, off_z, off_pm, off_ps, off_pz, off_pt;
+  size_t off_pool_tok, off_pool_par, off_pool_s, off_front;
+  size_t total;
+};
+
+// Pool id of the first node of level t (t >= 1).  Level 1 has k nodes, every
+// deeper level k * k (Sec. 4.1: b_0 = 1, b_d = k afterwards).
+__host__ __device__ inline int level_base(int t, int k) {
+  return t <= 1 ? t : 1 + k + (t - 2) * k * k;
+}
+
+__host__ __device__ inline int level_of(int id, int k) {
+  if (id == 0) return 0;
+  if (id <= k) return 1;
+  return 2 + (id - 1 - k) / (k * k);
+}
+
+// ---------------------------------------------------------------------------
+// ranking keys
+// ---------------------------------------------------------------------------
+
+// Maps a float to a uint32 whose unsigned order is the DEScending order of
+// the float (-0 and +0 equal).  NaN never reaches here (rejected earlier).
+__device__ __forceinline__ uint32_t desc_key(float x) {
+  x = x + 0.0f;  // -0 -> +0
+  uint32_t u = __float_as_uint(x);
+  uint32_t asc = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+  return ~asc;
+}
+
+// Candidate order inside one parent: larger logit first, then lower token.
+__device__ __forceinline__ bool cand_better(float a, int ta, float b, int tb) {
+  return a > b || (a == b && ta < tb);
+}
+
+// ---------------------------------------------------------------------------
+// warp-resident sorted top-k list: lane i < k holds entry i (best first);
+// other lanes hold the sentinel (-inf, INT_MAX), worse than every entry
+// ---------------------------------------------------------------------------
+
+struct WarpList {
+  float v;
+  int t;
+  __device__ __forceinline__ void reset() {
+    v = -__int_as_float(0x7f800000);
+    t = 0x7fffffff;
+  }
+  // Inserts the warp-uniform candidate (cv, ct), dropping the k-th entry.
+  __device__ __forceinline__ void insert(float cv, int ct, int k) {
+    const int lane = threadIdx.x & 31;
+    const bool ahead = lane < k && cand_better(v, t, cv, ct);
+    const int pos = __popc(__ballot_sync(kFull, ahead));
+    const float uv = __shfl_up_sync(kFull, v, 1);
+    const int ut = __shfl_up_sync(kFull, t, 1);
+    if (pos < k) {
+      if (lane == pos) {
+        v = cv;
+        t = ct;
+      } else if (lane > pos && lane < k) {
+        v = uv;
+        t = ut;
+      }
+    }
+  }
+  // Offers one candidate per lane (lanes with nothing pass the sentinel).
+  __device__ __forceinline__ void offer(float cv, int ct, int k) {
+    float tv = __shfl_sync(kFull, v, k - 1);
+    int tt = __shfl_sync(kFull, t, k - 1);
+    unsigned m = __ballot_sync(kFull, cand_better(cv, ct, tv, tt));
+    while (m) {
+      const int src = __ffs(m) - 1;
+      const float sv = __shfl_sync(kFull, cv, src);
+      const int st = __shfl_sync(kFull, ct, src);
+      insert(sv, st, k);
+      tv = __shfl_sync(kFull, v, k - 1);
+      tt = __shfl_sync(kFull, t, k - 1);
+      m &= ~(1u << src);
+      m &= __ballot_sync(kFull, cand_better(cv, ct, tv, tt));
+    }
+  }
+};
+
+// Online (max, sum exp) pair; m = -inf means "no finite value yet".
+__device__ __forceinline__ void lse_push(float& m, float& s, float z) {
+  if (z > m) {
+    s = s * expf(m - z) + 1.0f;
+    m = z;
+  } else if (z > -__int_as_float(0x7f800000)) {
+    s += expf(z - m);
+  }
+}
+
+__device__ __forceinline__ void lse_merge(float& m, float& s, float m2,
+                                          float s2) {
+  const float M = fmaxf(m, m2);
+  if (M == -__int_as_float(0x7f800000)) return;
+  s = s * expf(m - M) + s2 * expf(m2 - M);
+  m = M;
+}
+
+__device__ __forceinline__ void set_status(int32_t* status, int code) {
+  atomicCAS(status, 0, code);
+}
+
+// ---------------------------------------------------------------------------
+// launchers (return cudaGetLastError() of the launch)
+// ---------------------------------------------------------------------------
+
+// Z[row][v] = L[req(row)][v] + sum_h W_out[v][h] X[row][h] for rows
+// [0, rows), req(row) = row / rows_per_req.  `L` points at depth d of
+// request 0; requests are `l_req_stride` floats apart.
+cudaError_t launch_markov_bf16(const CUtensorMap* tmap_w,
+                               const CUtensorMap* tmap_x, const float* L,
+                               long long l_req_stride, float* Z, int ldz,
+                               int V, int H, int rows, int rows_per_req,
+                               int bn, int num_sms, int32_t* status,
+                               cudaStream_t stream);
+
+cudaError_t launch_markov_f32(const float* W_out, const float* X,
+                              const float* L, long long l_req_stride, float* Z,
+                              int ldz, int V, int H, int rows,
+                              int rows_per_req, int32_t* status,
+                              cudaStream_t stream);
+
+cudaError_t launch_init(const pctree_config& c, const Layout& lay,
+                        const int32_t* root, const void* E_in,
+                        unsigned char* ws, int32_t* status,
+                        cudaStream_t stream);
+
+cudaError_t launch_partials(const Layout& lay, int k, int V, int rows,
+                            unsigned char* ws, int32_t* status,
+                            cudaStream_t stream);
+
+cudaError_t launch_merge(const pctree_config& c, const Layout& lay, int d,
+                         const void* E_in, unsigned char* ws,
+                         int32_t* status, cudaStream_t stream);
+
+cudaError_t launch_pack(const pctree_config& c, const Layout& lay,
+                        unsigned char* ws, const pctree_tree& out,
+                        cudaStream_t stream);
+
+cudaError_t launch_accept(const pctree_config& c, const pctree_tree& tree,
+                          const int32_t* target, int32_t* accepted_idx,
+                          int32_t* accepted_len, int32_t* bonus,
+                          cudaStream_t stream);
+
+}  // namespace pct

@@ -1,0 +1,585 @@
+// Selection side of a PCTree drafting round on GB300:
+//   init      the root of every request (Algorithm 1, initial frontier/pool)
+//   partials  per vocabulary chunk of a stage-logit row: online max / sum-exp
+//             (Eq. 2) and the chunk's top-k tokens
+//   merge     per request: log-softmax normaliser and top-k children of each
+//             parent, joint scores (Eq. 4), pool push, layer-wise frontier
+//             (Sec. 4.1) and the parents' Markov input rows for the next stage
+//   pack      per request: global top-N by radix select (Sec. 4.2), breadth-
+//             first packing, ancestor mask, position ids and retrieve rows
+//             (Appendix A "Tensor implementation")
+//   accept    per request: greedy tree walk (Sec. 4.2; Appendix A)
+#include <cuda_bf16.h>
+
+#include "pctree_common.cuh"
+
+namespace pct {
+
+namespace {
+
+constexpr float kNegInf = -INFINITY;
+
+__device__ __forceinline__ bool is_nonfinite_logit(float z) {
+  return isnan(z) || z == __int_as_float(0x7f800000);
+}
+
+// Copies one Markov input row E_in[token] into X[row] (bf16: 16-byte words).
+__device__ void copy_row(const void* E_in, void* X, int token, int row, int H,
+                         int x_elem, int tid, int nthreads) {
+  if (x_elem == 2) {
+    const uint4* src = reinterpret_cast<const uint4*>(
+        static_cast<const __nv_bfloat16*>(E_in) + static_cast<size_t>(token) * H);
+    uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(X) +
+                                          static_cast<size_t>(row) * H);
+    for (int i = tid; i < H / 8; i += nthreads) dst[i] = src[i];
+  } else {
+    const float* src = static_cast<const float*>(E_in) + static_cast<size_t>(token) * H;
+    float* dst = static_cast<float*>(X) + static_cast<size_t>(row) * H;
+    for (int i = tid; i < H; i += nthreads) dst[i] = src[i];
+  }
+}
+
+// ---------------------------------------------------------------------------
+// init: pool = {root}, frontier = [root], X[r] = E_in[root_r]
+// ---------------------------------------------------------------------------
+
+__global__ void init_kernel(const int32_t* __restrict__ root, const void* E_in,
+                            void* X, int32_t* pool_tok, int32_t* pool_par,
+                            double* pool_s, int32_t* front, int V, int H,
+                            int P, int k, int x_elem, int32_t* status) {
+  const int r = blockIdx.x;
+  int tok = root[r];
+  if (tok < 0 || tok >= V) {
+    if (threadIdx.x == 0) set_status(status, PCTREE_ERR_INVALID_ARG);
+    tok = 0;  // keep every later access in bounds
+  }
+  if (threadIdx.x == 0) {
+    pool_tok[static_cast<size_t>(r) * P] = tok;
+    pool_par[static_cast<size_t>(r) * P] = -1;
+    pool_s[static_cast<size_t>(r) * P] = 0.0;  // s(root) = 0 (Sec. 4.2)
+    front[static_cast<size_t>(r) * k] = 0;
+  }
+  copy_row(E_in, X, tok, r, H, x_elem, threadIdx.x, blockDim.x);
+}
+
+// ---------------------------------------------------------------------------
+// partials: one CTA per (chunk of kChunk logits, row)
+// ---------------------------------------------------------------------------
+
+__global__ void __launch_bounds__(kChunkThreads)
+partials_kernel(const float* __restrict__ Z, int ldz, int V, int k,
+                int n_chunks, float* __restrict__ part_m,
+                float* __restrict__ part_s, float* __restrict__ part_z,
+                int32_t* __restrict__ part_t, int32_t* status) {
+  const int chunk = blockIdx.x;
+  const int row = blockIdx.y;
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  constexpr int kWarps = kChunkThreads / 32;
+  __shared__ float sm_m[kWarps], sm_s[kWarps];
+  __shared__ float sm_v[kWarps][32];
+  __shared__ int sm_t[kWarps][32];
+
+  const float* z_row = Z + static_cast<size_t>(row) * ldz;
+  const int v0 = chunk * kChunk;
+  float m = kNegInf, s = 0.0f;
+  WarpList lst;
+  lst.reset();
+  bool bad = false;
+#pragma unroll 2
+  for (int i = 0; i < kChunk / kChunkThreads; ++i) {
+    const int v = v0 + i * kChunkThreads + threadIdx.x;
+    float z = kNegInf;
+    int t = 0x7fffffff;
+    if (v < V) {
+      z = z_row[v];
+      t = v;
+      bad |= is_nonfinite_logit(z);
+      lse_push(m, s, z);
+    }
+    lst.offer(z, t, k);
+  }
+  if (bad) set_status(status, PCTREE_ERR_NONFINITE);
+  // warp reduction of (m, s)
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(kFull, m, o);
+    const float s2 = __shfl_xor_sync(kFull, s, o);
+    lse_merge(m, s, m2, s2);
+  }
+  if (lane == 0) {
+    sm_m[warp] = m;
+    sm_s[warp] = s;
+  }
+  sm_v[warp][lane] = lst.v;
+  sm_t[warp][lane] = lst.t;
+  __syncthreads();
+  if (warp == 0) {
+    float mm = lane < kWarps ? sm_m[lane] : kNegInf;
+    float ss = lane < kWarps ? sm_s[lane] : 0.0f;
+    for (int o = 16; o > 0; o >>= 1) {
+      const float m2 = __shfl_xor_sync(kFull, mm, o);
+      const float s2 = __shfl_xor_sync(kFull, ss, o);
+      lse_merge(mm, ss, m2, s2);
+    }
+    // lane 0 keeps its own list; merge the other warps' lists into it
+    for (int w = 1; w < kWarps; ++w) {
+      const float cv = lane < k ? sm_v[w][lane] : kNegInf;
+      const int ct = lane < k ? sm_t[w][lane] : 0x7fffffff;
+      lst.offer(cv, ct, k);
+    }
+    const size_t p = static_cast<size_t>(row) * n_chunks + chunk;
+    if (lane == 0) {
+      part_m[p] = mm;
+      part_s[p] = ss;
+    }
+    if (lane < k) {
+      part_z[p * k + lane] = lst.v;
+      part_t[p * k + lane] = lst.t;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// merge: one CTA per request
+// ---------------------------------------------------------------------------
+
+constexpr int kMergeThreads = 256;
+
+__global__ void __launch_bounds__(kMergeThreads)
+merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
+             int x_elem, const float* __restrict__ part_m,
+             const float* __restrict__ part_s,
+             const float* __restrict__ part_z,
+             const int32_t* __restrict__ part_t, int32_t* pool_tok,
+             int32_t* pool_par, double* pool_s, int32_t* front,
+             const void* E_in, void* X, int32_t* status) {
+  const int r = blockIdx.x;
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  constexpr int kWarps = kMergeThreads / 32;
+  extern __shared__ unsigned long long sm_keys[];  // b_d * k layer keys
+  __shared__ int sm_front[PCTREE_MAX_K];
+
+  int32_t* tok = pool_tok + static_cast<size_t>(r) * P;
+  int32_t* par = pool_par + static_cast<size_t>(r) * P;
+  double* sc = pool_s + static_cast<size_t>(r) * P;
+  int32_t* fr = front + static_cast<size_t>(r) * k;
+  const int base = level_base(d + 1, k);
+
+  // children of each parent slot j: one warp per slot
+  for (int j = warp; j < b_d; j += kWarps) {
+    const int row = r * b_d + j;
+    const size_t p0 = static_cast<size_t>(row) * n_chunks;
+    // log-softmax normaliser from the chunk partials, in float64
+    double M = -INFINITY;
+    for (int c = lane; c < n_chunks; c += 32) M = fmax(M, (double)part_m[p0 + c]);
+    for (int o = 16; o > 0; o >>= 1) M = fmax(M, __shfl_xor_sync(kFull, M, o));
+    double S = 0.0;
+    if (M > -INFINITY) {
+      for (int c = lane; c < n_chunks; c += 32) {
+        const float mc = part_m[p0 + c];
+        if (mc > kNegInf) S += (double)part_s[p0 + c] * exp((double)mc - M);
+      }
+    }
+    for (int o = 16; o > 0; o >>= 1) S += __shfl_xor_sync(kFull, S, o);
+    if (!(M > -INFINITY)) {
+      if (lane == 0) set_status(status, PCTREE_ERR_NONFINITE);
+    }
+    const double lse = M + log(S);
+    // top-k children of this parent over all chunk lists
+    WarpList lst;
+    lst.reset();
+    const int n_cand = n_chunks * k;
+    for (int c0 = 0; c0 < n_cand; c0 += 32) {
+      const int c = c0 + lane;
+      float cv = kNegInf;
+      int ct = 0x7fffffff;
+      if (c < n_cand) {
+        cv = part_z[p0 * k + c];
+        ct = part_t[p0 * k + c];
+      }
+      lst.offer(cv, ct, k);
+    }
+    const int pid = fr[j];
+    if (lane < k) {
+      const int id = base + j * k + lane;
+      int t = lst.t;
+      double logpi = (double)lst.v - lse;
+      if (t < 0 || t >= V) {  // only when V < k (rejected on the host)
+        t = 0;
+        logpi = -INFINITY;
+      }
+      tok[id] = t;
+      par[id] = pid;
+      sc[id] = sc[pid] + logpi;  // Eq. 4: s(child) = s(p) + log pi(child|p)
+    }
+  }
+  if (d == B - 1) return;
+  __syncthreads();
+  // frontier: the k best nodes of this layer by (score desc, id asc)
+  const int n_layer = b_d * k;
+  for (int i = threadIdx.x; i < n_layer; i += blockDim.x) {
+    const int id = base + i;
+    sm_keys[i] = (static_cast<unsigned long long>(desc_key((float)sc[id])) << 32) |
+                 static_cast<unsigned int>(id);
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < n_layer; i += blockDim.x) {
+    const unsigned long long key = sm_keys[i];
+    int rank = 0;
+    for (int j = 0; j < n_layer; ++j) rank += sm_keys[j] < key;
+    if (rank < k) {
+      sm_front[rank] = base + i;
+      fr[rank] = base + i;
+    }
+  }
+  __syncthreads();
+  // Markov input rows of the next stage: X[r * k + slot] = E_in[token]
+  for (int slot = 0; slot < k; ++slot) {
+    copy_row(E_in, X, tok[sm_front[slot]], r * k + slot, H, x_elem,
+             threadIdx.x, blockDim.x);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// pack: one CTA of 1024 threads per request
+// ---------------------------------------------------------------------------
+
+constexpr int kPackThreads = 1024;
+
+__device__ __forceinline__ int block_excl_scan(int x, int* sm_warp, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int incl = x;
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(kFull, incl, o);
+    if (lane >= o) incl += y;
+  }
+  if (lane == 31) sm_warp[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    const int nw = blockDim.x >> 5;
+    int w = lane < nw ? sm_warp[lane] : 0;
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(kFull, w, o);
+      if (lane >= o) w += y;
+    }
+    if (lane < nw) sm_warp[lane] = w;  // inclusive per warp
+  }
+  __syncthreads();
+  const int before = (warp == 0 ? 0 : sm_warp[warp - 1]) + incl - x;
+  if (total) *total = sm_warp[(blockDim.x >> 5) - 1];
+  __syncthreads();
+  return before;
+}
+
+__global__ void __launch_bounds__(kPackThreads)
+pack_kernel(int B, int k, int N, int P, int pos_offset,
+            const int32_t* __restrict__ pool_tok,
+            const int32_t* __restrict__ pool_par,
+            const double* __restrict__ pool_s, pctree_tree out) {
+  const int r = blockIdx.x;
+  const int tid = threadIdx.x;
+  extern __shared__ unsigned long long sm_key[];  // P keys; later reused
+  __shared__ unsigned int sm_hist[256];
+  __shared__ int sm_warp[32];
+  __shared__ int sm_sel[PCTREE_MAX_N];    // packed index -> pool id
+  __shared__ int sm_par[PCTREE_MAX_N];    // packed index -> packed parent
+  __shared__ unsigned char sm_haschild[PCTREE_MAX_N];
+  __shared__ unsigned long long sm_prefix;
+  __shared__ int sm_remaining, sm_count;
+
+  const int32_t* tok = pool_tok + static_cast<size_t>(r) * P;
+  const int32_t* par = pool_par + static_cast<size_t>(r) * P;
+  const double* sc = pool_s + static_cast<size_t>(r) * P;
+  const int n = min(N, P);
+
+  // 46-bit keys: descending fp32 score in bits 45..14, pool id in 13..0.
+  // Ids grow with depth, so (score desc, id asc) is (score desc, depth asc,
+  // id asc) of Sec. 4.2.
+  for (int i = tid; i < P; i += blockDim.x) {
+    sm_key[i] = (static_cast<unsigned long long>(desc_key((float)sc[i])) << 14) |
+                static_cast<unsigned long long>(i);
+  }
+  if (tid == 0) {
+    sm_prefix = 0ull;
+    sm_remaining = n;
+  }
+  __syncthreads();
+  // radix select of the n-th smallest key, 8 bits per pass from bit 40
+  unsigned long long mask = 0ull;
+  for (int shift = 40; shift >= 0; shift -= 8) {
+    for (int i = tid; i < 256; i += blockDim.x) sm_hist[i] = 0u;
+    __syncthreads();
+    const unsigned long long prefix = sm_prefix;
+    for (int i = tid; i < P; i += blockDim.x) {
+      const unsigned long long key = sm_key[i];
+      if ((key & mask) == prefix) atomicAdd(&sm_hist[(key >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (tid < 32) {
+      // lane L owns bins 8L .. 8L+7
+      int cnt = 0;
+      for (int b = 0; b < 8; ++b) cnt += sm_hist[tid * 8 + b];
+      int incl = cnt;
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(kFull, incl, o);
+        if (tid >= o) incl += y;
+      }
+      const int need = sm_remaining;
+      const int excl = incl - cnt;
+      const bool here = excl < need && incl >= need;
+      if (here) {
+        int acc = excl;
+        for (int b = 0; b < 8; ++b) {
+          const int hb = sm_hist[tid * 8 + b];
+          if (acc + hb >= need) {
+            sm_prefix = prefix | (static_cast<unsigned long long>(tid * 8 + b) << shift);
+            sm_remaining = need - acc;
+            break;
+          }
+          acc += hb;
+        }
+      }
+    }
+    mask |= 255ull << shift;
+    __syncthreads();
+  }
+  const unsigned long long kth = sm_prefix;  // n-th smallest key, exactly
+  // gather the selected pool ids (unordered) into sm_sel
+  if (tid == 0) sm_count = 0;
+  __syncthreads();
+  for (int i = tid; i < P; i += blockDim.x) {
+    if (sm_key[i] <= kth) sm_sel[atomicAdd(&sm_count, 1)] = i;
+  }
+  __syncthreads();
+  // breadth-first packing: level by level, (parent's index, token) order
+  int* pidx = reinterpret_cast<int*>(sm_key);  // pool id -> packed index
+  for (int i = tid; i < P; i += blockDim.x) pidx[i] = -1;
+  __syncthreads();
+  int my_id = tid < n ? sm_sel[tid] : -1;
+  const int my_lvl = my_id >= 0 ? level_of(my_id, k) : -1;
+  __syncthreads();
+  int placed = 0;
+  for (int t = 0; t <= B; ++t) {
+    const bool at = my_lvl == t;
+    unsigned long long key2 = 0ull;
+    if (at) {
+      const int pp = t == 0 ? -1 : pidx[par[my_id]];
+      key2 = (static_cast<unsigned long long>(static_cast<unsigned int>(pp + 1)) << 32) |
+             static_cast<unsigned int>(tok[my_id]);
+    }
+    int n_t;
+    block_excl_scan(at ? 1 : 0, sm_warp, &n_t);
+    if (n_t == 0) break;
+    // rank among the nodes of this level (<= n of them)
+    __shared__ unsigned long long sm_k2[PCTREE_MAX_N];
+    __shared__ int sm_lvl_slot;
+    if (tid == 0) sm_lvl_slot = 0;
+    __syncthreads();
+    int slot = -1;
+    if (at) {
+      slot = atomicAdd(&sm_lvl_slot, 1);
+      sm_k2[slot] = key2;
+    }
+    __syncthreads();
+    if (at) {
+      int rank = 0;
+      for (int j = 0; j < n_t; ++j) rank += sm_k2[j] < key2;
+      const int a = placed + rank;
+      pidx[my_id] = a;
+      sm_sel[a] = my_id;  // safe: slots of this level are read via my_id only
+    }
+    placed += n_t;
+    __syncthreads();
+  }
+  // per packed node: parent index, child flags
+  for (int a = tid; a < n; a += blockDim.x) {
+    const int id = sm_sel[a];
+    sm_par[a] = a == 0 ? -1 : pidx[par[id]];
+    sm_haschild[a] = 0;
+  }
+  __syncthreads();
+  for (int a = tid; a < n; a += blockDim.x)
+    if (a > 0) sm_haschild[sm_par[a]] = 1;
+  __syncthreads();
+  int32_t* o_tok = out.tokens + static_cast<size_t>(r) * N;
+  int32_t* o_par = out.parent + static_cast<size_t>(r) * N;
+  int32_t* o_dep = out.depth + static_cast<size_t>(r) * N;
+  float* o_lp = out.logp + static_cast<size_t>(r) * N;
+  int32_t* o_pos = out.position_ids + static_cast<size_t>(r) * N;
+  uint8_t* o_mask = out.mask + static_cast<size_t>(r) * N * N;
+  int32_t* o_ret = out.retrieve + static_cast<size_t>(r) * N * (B + 1);
+  for (int a = tid; a < N; a += blockDim.x) {
+    if (a < n) {
+      const int id = sm_sel[a];
+      const int lvl = level_of(id, k);
+      o_tok[a] = tok[id];
+      o_par[a] = sm_par[a];
+      o_dep[a] = lvl;
+      o_lp[a] = (float)sc[id];
+      o_pos[a] = lvl + pos_offset;  // siblings share a position (Appendix A)
+    } else {
+      o_tok[a] = -1;
+      o_par[a] = -1;
+      o_dep[a] = -1;
+      o_lp[a] = kNegInf;
+      o_pos[a] = -1;
+    }
+  }
+  // leaves in packed order
+  const int is_leaf = (tid < n && !sm_haschild[tid]) ? 1 : 0;
+  int n_leaves;
+  const int leaf_rank = block_excl_scan(is_leaf, sm_warp, &n_leaves);
+  // clear mask and retrieve, then scatter the ancestor chains
+  const size_t mask_bytes = static_cast<size_t>(N) * N;
+  for (size_t i = tid; i < mask_bytes; i += blockDim.x) o_mask[i] = 0;
+  const int ret_len = N * (B + 1);
+  for (int i = tid; i < ret_len; i += blockDim.x) o_ret[i] = -1;
+  __syncthreads();
+  if (tid < n) {
+    // ancestor-or-self mask row (the prefix is visible to every node)
+    for (int b = tid; b >= 0; b = sm_par[b]) o_mask[static_cast<size_t>(tid) * N + b] = 1;
+    if (is_leaf) {
+      int32_t* row = o_ret + static_cast<size_t>(leaf_rank) * (B + 1);
+      int dpt = level_of(sm_sel[tid], k);
+      for (int b = tid; b >= 0; b = sm_par[b]) row[dpt--] = b;
+    }
+  }
+  if (tid == 0) {
+    out.n_nodes[r] = n;
+    out.n_leaves[r] = n_leaves;
+  }
+  if (out.pool_token != nullptr) {
+    for (int i = tid; i < P; i += blockDim.x) {
+      out.pool_token[static_cast<size_t>(r) * P + i] = tok[i];
+      out.pool_parent[static_cast<size_t>(r) * P + i] = par[i];
+      out.pool_logp[static_cast<size_t>(r) * P + i] = (float)sc[i];
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// accept: one warp per request
+// ---------------------------------------------------------------------------
+
+__global__ void accept_kernel(int B, int N, const int32_t* __restrict__ n_nodes,
+                              const int32_t* __restrict__ tokens,
+                              const int32_t* __restrict__ parent,
+                              const int32_t* __restrict__ target,
+                              int32_t* accepted_idx, int32_t* accepted_len,
+                              int32_t* bonus, int batch) {
+  const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (r >= batch) return;
+  const int lane = threadIdx.x & 31;
+  const int n = n_nodes[r];
+  const int32_t* tk = tokens + static_cast<size_t>(r) * N;
+  const int32_t* pa = parent + static_cast<size_t>(r) * N;
+  const int32_t* tg = target + static_cast<size_t>(r) * N;
+  int32_t* acc = accepted_idx + static_cast<size_t>(r) * (B + 1);
+  for (int i = lane; i <= B; i += 32) acc[i] = -1;
+  __syncwarp();
+  int cur = 0, len = 0;
+  if (lane == 0) acc[0] = 0;
+  while (len < B) {
+    const int want = tg[cur];
+    int next = -1;
+    // children of `cur` have indices > cur; siblings carry distinct tokens
+    for (int c0 = cur + 1; c0 < n && next < 0; c0 += 32) {
+      const int c = c0 + lane;
+      const bool hit = c < n && pa[c] == cur && tk[c] == want;
+      const unsigned m = __ballot_sync(kFull, hit);
+      if (m) next = c0 + __ffs(m) - 1;
+    }
+    if (next < 0) break;
+    cur = next;
+    ++len;
+    if (lane == 0) acc[len] = cur;
+  }
+  if (lane == 0) {
+    accepted_len[r] = len;
+    bonus[r] = tg[cur];
+  }
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// launchers
+// ---------------------------------------------------------------------------
+
+cudaError_t launch_init(const pctree_config& c, const Layout& lay,
+                        const int32_t* root, const void* E_in,
+                        unsigned char* ws, int32_t* status,
+                        cudaStream_t stream) {
+  init_kernel<<<c.batch, 256, 0, stream>>>(
+      root, E_in, ws + lay.off_x, reinterpret_cast<int32_t*>(ws + lay.off_pool_tok),
+      reinterpret_cast<int32_t*>(ws + lay.off_pool_par),
+      reinterpret_cast<double*>(ws + lay.off_pool_s),
+      reinterpret_cast<int32_t*>(ws + lay.off_front), c.V, c.H, lay.P, c.k,
+      lay.x_elem, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_partials(const Layout& lay, int k, int V, int rows,
+                            unsigned char* ws, int32_t* status,
+                            cudaStream_t stream) {
+  dim3 grid(lay.n_chunks, rows);
+  partials_kernel<<<grid, kChunkThreads, 0, stream>>>(
+      reinterpret_cast<const float*>(ws + lay.off_z), lay.ldz, V, k,
+      lay.n_chunks, reinterpret_cast<float*>(ws + lay.off_pm),
+      reinterpret_cast<float*>(ws + lay.off_ps),
+      reinterpret_cast<float*>(ws + lay.off_pz),
+      reinterpret_cast<int32_t*>(ws + lay.off_pt), status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_merge(const pctree_config& c, const Layout& lay, int d,
+                         const void* E_in, unsigned char* ws,
+                         int32_t* status, cudaStream_t stream) {
+  const int b_d = d == 0 ? 1 : c.k;
+  const size_t smem = static_cast<size_t>(b_d) * c.k * sizeof(unsigned long long);
+  merge_kernel<<<c.batch, kMergeThreads, smem, stream>>>(
+      d, c.B, c.k, b_d, c.V, c.H, lay.P, lay.n_chunks, lay.x_elem,
+      reinterpret_cast<const float*>(ws + lay.off_pm),
+      reinterpret_cast<const float*>(ws + lay.off_ps),
+      reinterpret_cast<const float*>(ws + lay.off_pz),
+      reinterpret_cast<const int32_t*>(ws + lay.off_pt),
+      reinterpret_cast<int32_t*>(ws + lay.off_pool_tok),
+      reinterpret_cast<int32_t*>(ws + lay.off_pool_par),
+      reinterpret_cast<double*>(ws + lay.off_pool_s),
+      reinterpret_cast<int32_t*>(ws + lay.off_front), E_in, ws + lay.off_x,
+      status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pack(const pctree_config& c, const Layout& lay,
+                        unsigned char* ws, const pctree_tree& out,
+                        cudaStream_t stream) {
+  const size_t smem = static_cast<size_t>(lay.P) * sizeof(unsigned long long);
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaFuncSetAttribute(pack_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         PCTREE_MAX_POOL * static_cast<int>(sizeof(unsigned long long)));
+    attr_set = true;
+  }
+  pack_kernel<<<c.batch, kPackThreads, smem, stream>>>(
+      c.B, c.k, c.N, lay.P, c.pos_offset,
+      reinterpret_cast<const int32_t*>(ws + lay.off_pool_tok),
+      reinterpret_cast<const int32_t*>(ws + lay.off_pool_par),
+      reinterpret_cast<const double*>(ws + lay.off_pool_s), out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_accept(const pctree_config& c, const pctree_tree& tree,
+                          const int32_t* target, int32_t* accepted_idx,
+                          int32_t* accepted_len, int32_t* bonus,
+                          cudaStream_t stream) {
+  const int warps = 4;
+  const int blocks = (c.batch + warps - 1) / warps;
+  accept_kernel<<<blocks, warps * 32, 0, stream>>>(
+      c.B, c.N, tree.n_nodes, tree.tokens, tree.parent, target, accepted_idx,
+      accepted_len, bonus, c.batch);
+  return cudaGetLastError();
+}
+
+}  // namespace pct

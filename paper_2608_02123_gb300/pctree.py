@@ -1,0 +1,270 @@
+"""Python binding of the PCTree C ABI (include/pctree.h).
+
+Argument marshalling only: every step of a drafting round runs in the CUDA
+library ``_build/libpctree_gb300.so``.  PyTorch supplies device memory and
+streams; tensors are passed to the library as raw device pointers.  If the
+library is missing, importing this module raises -- there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+from typing import Dict, Optional
+
+import torch
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_build",
+                         "libpctree_gb300.so")
+
+PCTREE_OK = 0
+PCTREE_F32 = 0
+PCTREE_BF16 = 1
+MAX_K, MAX_N, MAX_POOL, MAX_ROWS = 32, 1024, 16384, 4096
+
+STATUS_NAMES = {0: "ok", -1: "invalid argument", -2: "workspace",
+                -3: "CUDA error", -4: "timeout", -5: "non-finite input",
+                -6: "unsupported shape"}
+
+
+class PctreeError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        super().__init__(f"{where}: {STATUS_NAMES.get(code, code)} ({code})")
+        self.code = code
+
+
+class Config(ctypes.Structure):
+    _fields_ = [("V", ctypes.c_int32), ("H", ctypes.c_int32),
+                ("B", ctypes.c_int32), ("k", ctypes.c_int32),
+                ("N", ctypes.c_int32), ("batch", ctypes.c_int32),
+                ("pos_offset", ctypes.c_int32),
+                ("weight_dtype", ctypes.c_int32)]
+
+
+class _Tree(ctypes.Structure):
+    _fields_ = [(name, ctypes.c_void_p) for name in (
+        "n_nodes", "tokens", "parent", "depth", "logp", "position_ids",
+        "mask", "retrieve", "n_leaves", "status", "pool_token",
+        "pool_parent", "pool_logp")]
+
+
+def _load() -> ctypes.CDLL:
+    if not os.path.exists(_LIB_PATH):
+        raise ImportError(
+            f"PCTree CUDA library not built ({_LIB_PATH}); run "
+            "`python -m paper_2608_02123_gb300.build`")
+    lib = ctypes.CDLL(_LIB_PATH)
+    vp, cfgp = ctypes.c_void_p, ctypes.POINTER(Config)
+    lib.pctree_check_config.argtypes = [cfgp]
+    lib.pctree_check_config.restype = ctypes.c_int
+    lib.pctree_pool_capacity.argtypes = [cfgp]
+    lib.pctree_pool_capacity.restype = ctypes.c_int32
+    lib.pctree_workspace_bytes.argtypes = [cfgp]
+    lib.pctree_workspace_bytes.restype = ctypes.c_size_t
+    lib.pctree_draft.argtypes = [cfgp, vp, vp, vp, vp, ctypes.POINTER(_Tree),
+                                 vp, ctypes.c_size_t, vp]
+    lib.pctree_draft.restype = ctypes.c_int
+    lib.pctree_accept.argtypes = [cfgp, ctypes.POINTER(_Tree), vp, vp, vp, vp,
+                                  vp]
+    lib.pctree_accept.restype = ctypes.c_int
+    lib.pctree_status_string.argtypes = [ctypes.c_int32]
+    lib.pctree_status_string.restype = ctypes.c_char_p
+    lib.pctree_profile_enable.argtypes = [ctypes.c_int32]
+    lib.pctree_profile_enable.restype = ctypes.c_int
+    lib.pctree_profile_collect.argtypes = [ctypes.POINTER(ctypes.c_int64),
+                                           ctypes.POINTER(ctypes.c_double)]
+    lib.pctree_profile_collect.restype = ctypes.c_int
+    lib.pctree_version.argtypes = []
+    lib.pctree_version.restype = ctypes.c_int32
+    return lib
+
+
+LIB = _load()
+LIB_PATH = _LIB_PATH
+
+
+def make_config(V: int, H: int, B: int, k: int, N: int, batch: int = 1,
+                pos_offset: int = 0, weight_dtype: str = "bf16") -> Config:
+    return Config(V, H, B, k, N, batch, pos_offset,
+                  PCTREE_BF16 if weight_dtype == "bf16" else PCTREE_F32)
+
+
+def pctree_check_config(cfg: Config) -> int:
+    return LIB.pctree_check_config(ctypes.byref(cfg))
+
+
+def pctree_pool_capacity(cfg: Config) -> int:
+    return LIB.pctree_pool_capacity(ctypes.byref(cfg))
+
+
+def pctree_workspace_bytes(cfg: Config) -> int:
+    return LIB.pctree_workspace_bytes(ctypes.byref(cfg))
+
+
+def pctree_status_string(code: int) -> str:
+    return LIB.pctree_status_string(code).decode()
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+@dataclasses.dataclass
+class Tree:
+    """Device tensors of drafted trees (see pctree_tree in include/pctree.h)."""
+
+    n_nodes: torch.Tensor
+    tokens: torch.Tensor
+    parent: torch.Tensor
+    depth: torch.Tensor
+    logp: torch.Tensor
+    position_ids: torch.Tensor
+    mask: torch.Tensor
+    retrieve: torch.Tensor
+    n_leaves: torch.Tensor
+    status: torch.Tensor
+    pool_token: Optional[torch.Tensor] = None
+    pool_parent: Optional[torch.Tensor] = None
+    pool_logp: Optional[torch.Tensor] = None
+
+    def c_struct(self) -> _Tree:
+        return _Tree(*[_ptr(getattr(self, f.name))
+                       for f in dataclasses.fields(self)])
+
+    def to_host(self) -> Dict[str, "object"]:
+        return {f.name: (None if getattr(self, f.name) is None
+                         else getattr(self, f.name).cpu().numpy())
+                for f in dataclasses.fields(self)}
+
+
+def alloc_tree(cfg: Config, device, with_pool: bool = False) -> Tree:
+    R, N, B = cfg.batch, cfg.N, cfg.B
+    i32 = dict(dtype=torch.int32, device=device)
+    P = pctree_pool_capacity(cfg)
+    return Tree(
+        n_nodes=torch.empty(R, **i32), tokens=torch.empty(R, N, **i32),
+        parent=torch.empty(R, N, **i32), depth=torch.empty(R, N, **i32),
+        logp=torch.empty(R, N, dtype=torch.float32, device=device),
+        position_ids=torch.empty(R, N, **i32),
+        mask=torch.empty(R, N, N, dtype=torch.uint8, device=device),
+        retrieve=torch.empty(R, N, B + 1, **i32),
+        n_leaves=torch.empty(R, **i32), status=torch.empty(1, **i32),
+        pool_token=torch.empty(R, P, **i32) if with_pool else None,
+        pool_parent=torch.empty(R, P, **i32) if with_pool else None,
+        pool_logp=(torch.empty(R, P, dtype=torch.float32, device=device)
+                   if with_pool else None))
+
+
+def alloc_workspace(cfg: Config, device) -> torch.Tensor:
+    nbytes = pctree_workspace_bytes(cfg)
+    if nbytes == 0:
+        raise PctreeError(pctree_check_config(cfg), "pctree_workspace_bytes")
+    # torch's caching allocator returns 512-byte aligned blocks
+    return torch.empty(nbytes, dtype=torch.uint8, device=device)
+
+
+def _stream_ptr(stream: Optional[torch.cuda.Stream]) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+def pctree_draft(cfg: Config, base_logits: torch.Tensor, head_emb: torch.Tensor,
+                 head_out: torch.Tensor, root_token: torch.Tensor, tree: Tree,
+                 workspace: torch.Tensor,
+                 stream: Optional[torch.cuda.Stream] = None) -> None:
+    """Enqueue one drafting round (see pctree_draft in include/pctree.h)."""
+    for name, t in (("base_logits", base_logits), ("head_emb", head_emb),
+                    ("head_out", head_out), ("root_token", root_token)):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous CUDA tensor")
+    ts = tree.c_struct()
+    rc = LIB.pctree_draft(ctypes.byref(cfg), base_logits.data_ptr(),
+                          head_emb.data_ptr(), head_out.data_ptr(),
+                          root_token.data_ptr(), ctypes.byref(ts),
+                          workspace.data_ptr(), workspace.numel(),
+                          _stream_ptr(stream))
+    if rc != PCTREE_OK:
+        raise PctreeError(rc, "pctree_draft")
+
+
+def pctree_accept(cfg: Config, tree: Tree, target_tokens: torch.Tensor,
+                  accepted_idx: torch.Tensor, accepted_len: torch.Tensor,
+                  bonus_token: torch.Tensor,
+                  stream: Optional[torch.cuda.Stream] = None) -> None:
+    """Enqueue the greedy tree acceptance (see pctree_accept)."""
+    ts = tree.c_struct()
+    rc = LIB.pctree_accept(ctypes.byref(cfg), ctypes.byref(ts),
+                           target_tokens.data_ptr(), accepted_idx.data_ptr(),
+                           accepted_len.data_ptr(), bonus_token.data_ptr(),
+                           _stream_ptr(stream))
+    if rc != PCTREE_OK:
+        raise PctreeError(rc, "pctree_accept")
+
+
+def pctree_profile_enable(on: bool) -> None:
+    rc = LIB.pctree_profile_enable(1 if on else 0)
+    if rc != PCTREE_OK:
+        raise PctreeError(rc, "pctree_profile_enable")
+
+
+def pctree_profile_collect():
+    """Returns (launches, total milliseconds) of timed Markov projections."""
+    n = ctypes.c_int64(0)
+    ms = ctypes.c_double(0.0)
+    rc = LIB.pctree_profile_collect(ctypes.byref(n), ctypes.byref(ms))
+    if rc != PCTREE_OK:
+        raise PctreeError(rc, "pctree_profile_collect")
+    return int(n.value), float(ms.value)
+
+
+def pctree_version() -> int:
+    return LIB.pctree_version()
+
+
+class Drafter:
+    """Owns the device workspace and output tensors for one configuration."""
+
+    def __init__(self, cfg: Config, device="cuda", with_pool: bool = False):
+        rc = pctree_check_config(cfg)
+        if rc != PCTREE_OK:
+            raise PctreeError(rc, "pctree_check_config")
+        self.cfg = cfg
+        self.device = torch.device(device)
+        self.workspace = alloc_workspace(cfg, self.device)
+        self.tree = alloc_tree(cfg, self.device, with_pool)
+        i32 = dict(dtype=torch.int32, device=self.device)
+        self.accepted_idx = torch.empty(cfg.batch, cfg.B + 1, **i32)
+        self.accepted_len = torch.empty(cfg.batch, **i32)
+        self.bonus = torch.empty(cfg.batch, **i32)
+
+    def draft(self, base_logits, head_emb, head_out, root_token, stream=None):
+        pctree_draft(self.cfg, base_logits, head_emb, head_out, root_token,
+                     self.tree, self.workspace, stream)
+        return self.tree
+
+    def accept(self, target_tokens, stream=None):
+        pctree_accept(self.cfg, self.tree, target_tokens, self.accepted_idx,
+                      self.accepted_len, self.bonus, stream)
+        return self.accepted_idx, self.accepted_len, self.bonus
+
+    def check_status(self) -> None:
+        code = int(self.tree.status.item())
+        if code != PCTREE_OK:
+            raise PctreeError(code, "device status")
+
+    def draft_from_host(self, base_logits_host: torch.Tensor,
+                        root_host: torch.Tensor, head_emb, head_out,
+                        stream=None):
+        """End-to-end call a serving loop makes: pinned host inputs in, packed
+        tree back on the host.  Returns the host tree arrays."""
+        s = stream if stream is not None else torch.cuda.current_stream()
+        with torch.cuda.stream(s):
+            L = base_logits_host.to(self.device, non_blocking=True)
+            root = root_host.to(self.device, non_blocking=True)
+            self.draft(L, head_emb, head_out, root, s)
+            host = {name: getattr(self.tree, name).to("cpu", non_blocking=True)
+                    for name in ("n_nodes", "tokens", "parent", "depth",
+                                 "logp", "position_ids", "mask", "retrieve",
+                                 "n_leaves", "status")}
+        s.synchronize()
+        return host

@@ -1,0 +1,95 @@
+"""The C ABI library loads and exports every declared symbol, and its host
+side rejects bad arguments before touching a GPU (no GPU needed)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "pctree.h")
+
+
+@pytest.fixture(scope="module")
+def P():
+    from paper_2608_02123_gb300 import build
+    if not os.path.exists(build.LIB):
+        build.build()
+    from paper_2608_02123_gb300 import pctree
+    return pctree
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"PCTREE_API\s+[\w\s\*]+?\b(pctree_\w+)\(", text)))
+
+
+def test_header_declares_the_api():
+    names = declared_symbols()
+    for n in ("pctree_draft", "pctree_accept", "pctree_workspace_bytes",
+              "pctree_pool_capacity", "pctree_check_config"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(P):
+    lib = ctypes.CDLL(P.LIB_PATH)
+    for name in declared_symbols():
+        assert hasattr(lib, name), name
+
+
+def test_config_checks(P):
+    mk = P.make_config
+    assert P.pctree_check_config(mk(151936, 2560, 16, 8, 64, 1)) == 0
+    assert P.pctree_check_config(mk(1024, 64, 4, 4, 8, 1, 0, "f32")) == 0
+    assert P.pctree_check_config(mk(10, 8, 2, 11, 4, 1)) == -1      # k > V
+    assert P.pctree_check_config(mk(100, 12, 2, 2, 4, 1)) == -1     # H % 8
+    assert P.pctree_check_config(mk(100, 12, 2, 2, 4, 1, 0, "f32")) == 0
+    assert P.pctree_check_config(mk(100, 8, 2, 33, 4, 1)) == -6     # k limit
+    assert P.pctree_check_config(mk(100, 8, 2, 2, 1025, 1)) == -6   # N limit
+    assert P.pctree_check_config(mk(100, 8, 2, 8, 4, 513)) == -6    # rows
+    assert P.pctree_check_config(mk(100, 8, 300, 8, 4, 1)) == -6    # pool
+    assert P.pctree_check_config(mk(100, 8, 0, 2, 4, 1)) == -1
+    assert P.pctree_check_config(mk(100, 8, 2, 2, 0, 1)) == -1
+
+
+def test_sizes(P):
+    c = P.make_config(151936, 2560, 16, 8, 64, 1)
+    assert P.pctree_pool_capacity(c) == 1 + 8 + 15 * 64
+    ws = P.pctree_workspace_bytes(c)
+    assert ws % 256 == 0 and ws > 8 * 151936 * 4
+    assert P.pctree_workspace_bytes(P.make_config(10, 8, 2, 11, 4, 1)) == 0
+
+
+def test_draft_rejects_bad_arguments_on_the_host(P):
+    c = P.make_config(1000, 64, 3, 4, 8, 1)
+    tree = P._Tree(*([256] * 10 + [None] * 3))
+    fake = 4096
+    lib = P.LIB
+    # missing output pointer
+    t2 = P._Tree(*([256] * 9 + [None] * 4))
+    assert lib.pctree_draft(ctypes.byref(c), fake, fake, fake, fake,
+                            ctypes.byref(t2), fake, 1 << 30, None) == -1
+    # misaligned weights
+    assert lib.pctree_draft(ctypes.byref(c), fake, fake + 2, fake, fake,
+                            ctypes.byref(tree), fake, 1 << 30, None) == -1
+    # workspace too small or misaligned
+    assert lib.pctree_draft(ctypes.byref(c), fake, fake, fake, fake,
+                            ctypes.byref(tree), fake, 16, None) == -2
+    assert lib.pctree_draft(ctypes.byref(c), fake, fake, fake, fake,
+                            ctypes.byref(tree), fake + 8, 1 << 30, None) == -2
+    # only some of the optional pool outputs
+    t3 = P._Tree(*([256] * 11 + [None] * 2))
+    assert lib.pctree_draft(ctypes.byref(c), fake, fake, fake, fake,
+                            ctypes.byref(t3), fake, 1 << 30, None) == -1
+    # bad config
+    bad = P.make_config(10, 8, 2, 11, 4, 1)
+    assert lib.pctree_draft(ctypes.byref(bad), fake, fake, fake, fake,
+                            ctypes.byref(tree), fake, 1 << 30, None) == -1
+    assert lib.pctree_accept(ctypes.byref(c), ctypes.byref(t2), None, fake,
+                             fake, fake, None) == -1
+
+
+def test_status_strings(P):
+    assert P.pctree_status_string(0) == "ok"
+    assert "timed out" in P.pctree_status_string(-4)
+    assert P.pctree_version() >= 100

@@ -10,9 +10,12 @@ Draw order, per workload and seed (numpy PCG64 via ``SeedSequence(seed)``):
 
 * ``SeedSequence(seed).spawn(1 + batch)``: child 0 draws the Markov-head
   weights, child ``1 + r`` draws everything that belongs to request ``r``.
-* head (child 0): ``E_in`` then ``W_out``, each ``[V][H]`` drawn in row chunks
-  of ``_CHUNK_ROWS`` rows as float32 standard normals times the head scale;
-  bf16 workloads round each value to bf16 (round to nearest even).
+* head (child 0): ``child0.spawn(2)`` gives one sequence for ``E_in`` and one
+  for ``W_out``; each ``[V][H]`` matrix is cut into row chunks of
+  ``_CHUNK_ROWS`` rows and chunk ``i`` is drawn from ``seq.spawn(n_chunks)[i]``
+  as float32 standard normals times the head scale (chunks are independent,
+  so they are drawn in parallel threads); bf16 workloads round each value to
+  bf16 (round to nearest even).
 * request ``r``: base-logit noise ``[B][V]`` float32 normals; then the
   per-depth structure (planted tokens, or Zipf rank permutations); then the
   per-depth temperature coins (mixed-temperature workloads only); then the
@@ -27,7 +30,9 @@ of a drafted tree at depth ``t`` then receives ``target[i] = g[r][t]``.
 """
 from __future__ import annotations
 
+import concurrent.futures
 import dataclasses
+import os
 from typing import Dict, Optional
 
 import numpy as np
@@ -113,9 +118,12 @@ WORKLOADS: Dict[str, Workload] = {
 
 def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
     """Round float32 values to bf16 (nearest, ties to even); return the bits."""
-    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
-    rounded = (u + np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1)))
-    return (rounded >> np.uint32(16)).astype(np.uint16)
+    u = np.array(x, dtype=np.float32, copy=True).view(np.uint32)
+    lsb = (u >> np.uint32(16)) & np.uint32(1)
+    u += np.uint32(0x7FFF)
+    u += lsb
+    u >>= np.uint32(16)
+    return u.astype(np.uint16)
 
 
 def bf16_bits_to_f32(bits: np.ndarray) -> np.ndarray:
@@ -123,14 +131,22 @@ def bf16_bits_to_f32(bits: np.ndarray) -> np.ndarray:
     return (bits.astype(np.uint32) << np.uint32(16)).view(np.float32)
 
 
-def _draw_matrix(rng: np.random.Generator, V: int, H: int, scale: float,
+def _draw_matrix(seq: np.random.SeedSequence, V: int, H: int, scale: float,
                  dtype: str) -> np.ndarray:
     out = np.empty((V, H), dtype=np.uint16 if dtype == "bf16" else np.float32)
-    for r0 in range(0, V, _CHUNK_ROWS):
-        r1 = min(V, r0 + _CHUNK_ROWS)
-        blk = rng.standard_normal((r1 - r0, H), dtype=np.float32)
+    n_chunks = (V + _CHUNK_ROWS - 1) // _CHUNK_ROWS
+    seeds = seq.spawn(n_chunks)
+
+    def fill(i: int) -> None:
+        r0, r1 = i * _CHUNK_ROWS, min(V, (i + 1) * _CHUNK_ROWS)
+        blk = np.random.default_rng(seeds[i]).standard_normal(
+            (r1 - r0, H), dtype=np.float32)
         blk *= np.float32(scale)
         out[r0:r1] = f32_to_bf16_bits(blk) if dtype == "bf16" else blk
+
+    workers = max(1, min(n_chunks, os.cpu_count() or 1))
+    with concurrent.futures.ThreadPoolExecutor(workers) as ex:
+        list(ex.map(fill, range(n_chunks)))
     return out
 
 
@@ -150,9 +166,9 @@ class RoundInputs:
 def draw_head(wl: Workload, seed: Optional[int] = None):
     """Markov-head weights ``(E_in, W_out)`` for a workload."""
     ss = np.random.SeedSequence(wl.seed if seed is None else seed)
-    rng = np.random.default_rng(ss.spawn(1 + wl.batch)[0])
-    E_in = _draw_matrix(rng, wl.V, wl.H, wl.head_scale_e, wl.weight_dtype)
-    W_out = _draw_matrix(rng, wl.V, wl.H, wl.head_scale_w, wl.weight_dtype)
+    seq_e, seq_w = ss.spawn(1 + wl.batch)[0].spawn(2)
+    E_in = _draw_matrix(seq_e, wl.V, wl.H, wl.head_scale_e, wl.weight_dtype)
+    W_out = _draw_matrix(seq_w, wl.V, wl.H, wl.head_scale_w, wl.weight_dtype)
     return E_in, W_out
 
 
