@@ -13,7 +13,7 @@
 namespace pct {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kChunk = 2048;          // vocabulary entries per partials CTA
+constexpr int kChunk = 8192;          // vocabulary entries per partials CTA
 constexpr int kChunkThreads = 256;
 
 // ---------------------------------------------------------------------------
@@ -91,6 +91,29 @@ struct WarpList {
         t = ut;
       }
     }
+  }
+  // Starts the list from one candidate per lane (the list must be empty):
+  // a warp bitonic sort puts the best first, lanes >= k take the sentinel.
+  __device__ __forceinline__ void seed(float cv, int ct, int k) {
+    const int lane = threadIdx.x & 31;
+    v = cv;
+    t = ct;
+#pragma unroll
+    for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+      for (int j = size >> 1; j > 0; j >>= 1) {
+        const float ov = __shfl_xor_sync(kFull, v, j);
+        const int ot = __shfl_xor_sync(kFull, t, j);
+        const bool take_best = ((lane & j) == 0) == ((lane & size) == 0);
+        const bool swap = take_best ? cand_better(ov, ot, v, t)
+                                    : cand_better(v, t, ov, ot);
+        if (swap) {
+          v = ov;
+          t = ot;
+        }
+      }
+    }
+    if (lane >= k) reset();
   }
   // Offers one candidate per lane (lanes with nothing pass the sentinel).
   __device__ __forceinline__ void offer(float cv, int ct, int k) {

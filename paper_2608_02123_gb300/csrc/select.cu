@@ -82,22 +82,32 @@ partials_kernel(const float* __restrict__ Z, int ldz, int V, int k,
 
   const float* z_row = Z + static_cast<size_t>(row) * ldz;
   const int v0 = chunk * kChunk;
+  constexpr int kPer = kChunk / kChunkThreads;
+  float zs[kPer];
+  // every load of the chunk in flight at once; selection work afterwards
+#pragma unroll
+  for (int i = 0; i < kPer; ++i) {
+    const int v = v0 + i * kChunkThreads + threadIdx.x;
+    zs[i] = v < V ? z_row[v] : kNegInf;
+  }
   float m = kNegInf, s = 0.0f;
   WarpList lst;
-  lst.reset();
   bool bad = false;
-#pragma unroll 2
-  for (int i = 0; i < kChunk / kChunkThreads; ++i) {
+#pragma unroll
+  for (int i = 0; i < kPer; ++i) {
     const int v = v0 + i * kChunkThreads + threadIdx.x;
-    float z = kNegInf;
-    int t = 0x7fffffff;
-    if (v < V) {
-      z = z_row[v];
-      t = v;
+    const bool in = v < V;
+    const float z = zs[i];
+    const int t = in ? v : 0x7fffffff;
+    if (in) {
       bad |= is_nonfinite_logit(z);
       lse_push(m, s, z);
     }
-    lst.offer(z, t, k);
+    if (i == 0) {
+      lst.seed(z, t, k);
+    } else {
+      lst.offer(z, t, k);
+    }
   }
   if (bad) set_status(status, PCTREE_ERR_NONFINITE);
   // warp reduction of (m, s)
@@ -140,12 +150,53 @@ partials_kernel(const float* __restrict__ Z, int ldz, int V, int k,
 }
 
 // ---------------------------------------------------------------------------
-// merge: one CTA per request
+// merge: one CTA per request, one warp per parent slot
 // ---------------------------------------------------------------------------
 
-constexpr int kMergeThreads = 256;
+constexpr int kUnroll = 8;
 
-__global__ void __launch_bounds__(kMergeThreads)
+// Copies the Markov input rows of the next stage, X[first_row + slot] =
+// E_in[tok[slot]] for slot < n_rows, with all loads of a batch in flight.
+__device__ void gather_rows(const void* E_in, void* X, const int* tok,
+                            int n_rows, int first_row, int H, int x_elem) {
+  const int tid = threadIdx.x, nt = blockDim.x;
+  if (x_elem == 2) {
+    const int per_row = H / 8;
+    const int total = n_rows * per_row;
+    const uint4* src = static_cast<const uint4*>(E_in);
+    uint4* dst = static_cast<uint4*>(X);
+    for (int i0 = tid; i0 < total; i0 += nt * 4) {
+      uint4 tmp[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + u * nt;
+        if (i < total) {
+          const int slot = i / per_row, off = i - slot * per_row;
+          tmp[u] = src[static_cast<size_t>(tok[slot]) * per_row + off];
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + u * nt;
+        if (i < total) {
+          const int slot = i / per_row, off = i - slot * per_row;
+          dst[static_cast<size_t>(first_row + slot) * per_row + off] = tmp[u];
+        }
+      }
+    }
+  } else {
+    const int total = n_rows * H;
+    const float* src = static_cast<const float*>(E_in);
+    float* dst = static_cast<float*>(X);
+    for (int i = tid; i < total; i += nt) {
+      const int slot = i / H, off = i - slot * H;
+      dst[static_cast<size_t>(first_row + slot) * H + off] =
+          src[static_cast<size_t>(tok[slot]) * H + off];
+    }
+  }
+}
+
+__global__ void __launch_bounds__(1024)
 merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
              int x_elem, const float* __restrict__ part_m,
              const float* __restrict__ part_s,
@@ -156,9 +207,8 @@ merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
   const int r = blockIdx.x;
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
-  constexpr int kWarps = kMergeThreads / 32;
   extern __shared__ unsigned long long sm_keys[];  // b_d * k layer keys
-  __shared__ int sm_front[PCTREE_MAX_K];
+  __shared__ int sm_tok[PCTREE_MAX_K];
 
   int32_t* tok = pool_tok + static_cast<size_t>(r) * P;
   int32_t* par = pool_par + static_cast<size_t>(r) * P;
@@ -166,39 +216,65 @@ merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
   int32_t* fr = front + static_cast<size_t>(r) * k;
   const int base = level_base(d + 1, k);
 
-  // children of each parent slot j: one warp per slot
-  for (int j = warp; j < b_d; j += kWarps) {
+  if (warp < b_d) {
+    const int j = warp;
     const int row = r * b_d + j;
     const size_t p0 = static_cast<size_t>(row) * n_chunks;
-    // log-softmax normaliser from the chunk partials, in float64
-    double M = -INFINITY;
-    for (int c = lane; c < n_chunks; c += 32) M = fmax(M, (double)part_m[p0 + c]);
-    for (int o = 16; o > 0; o >>= 1) M = fmax(M, __shfl_xor_sync(kFull, M, o));
-    double S = 0.0;
-    if (M > -INFINITY) {
-      for (int c = lane; c < n_chunks; c += 32) {
-        const float mc = part_m[p0 + c];
-        if (mc > kNegInf) S += (double)part_s[p0 + c] * exp((double)mc - M);
+    // log-softmax normaliser from the chunk partials (Eq. 2), in float64
+    float Mf = kNegInf;
+    for (int c0 = 0; c0 < n_chunks; c0 += 32 * kUnroll) {
+      float mv[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int c = c0 + u * 32 + lane;
+        mv[u] = c < n_chunks ? part_m[p0 + c] : kNegInf;
       }
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) Mf = fmaxf(Mf, mv[u]);
+    }
+    for (int o = 16; o > 0; o >>= 1) Mf = fmaxf(Mf, __shfl_xor_sync(kFull, Mf, o));
+    double S = 0.0;
+    if (Mf > kNegInf) {
+      for (int c0 = 0; c0 < n_chunks; c0 += 32 * kUnroll) {
+        float mv[kUnroll], sv[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+          const int c = c0 + u * 32 + lane;
+          mv[u] = c < n_chunks ? part_m[p0 + c] : kNegInf;
+          sv[u] = c < n_chunks ? part_s[p0 + c] : 0.0f;
+        }
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u)
+          if (mv[u] > kNegInf) S += (double)sv[u] * exp((double)mv[u] - (double)Mf);
+      }
+    } else if (lane == 0) {
+      set_status(status, PCTREE_ERR_NONFINITE);
     }
     for (int o = 16; o > 0; o >>= 1) S += __shfl_xor_sync(kFull, S, o);
-    if (!(M > -INFINITY)) {
-      if (lane == 0) set_status(status, PCTREE_ERR_NONFINITE);
-    }
-    const double lse = M + log(S);
-    // top-k children of this parent over all chunk lists
+    const double lse = (double)Mf + log(S);
+    // top-k children of this parent over every chunk's list
     WarpList lst;
     lst.reset();
     const int n_cand = n_chunks * k;
-    for (int c0 = 0; c0 < n_cand; c0 += 32) {
-      const int c = c0 + lane;
-      float cv = kNegInf;
-      int ct = 0x7fffffff;
-      if (c < n_cand) {
-        cv = part_z[p0 * k + c];
-        ct = part_t[p0 * k + c];
+    const float* cz = part_z + p0 * k;
+    const int32_t* ct = part_t + p0 * k;
+    for (int c0 = 0; c0 < n_cand; c0 += 32 * kUnroll) {
+      float cv[kUnroll];
+      int ci[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int c = c0 + u * 32 + lane;
+        cv[u] = c < n_cand ? cz[c] : kNegInf;
+        ci[u] = c < n_cand ? ct[c] : 0x7fffffff;
       }
-      lst.offer(cv, ct, k);
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        if (c0 == 0 && u == 0) {
+          lst.seed(cv[u], ci[u], k);
+        } else {
+          lst.offer(cv[u], ci[u], k);
+        }
+      }
     }
     const int pid = fr[j];
     if (lane < k) {
@@ -229,16 +305,13 @@ merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
     int rank = 0;
     for (int j = 0; j < n_layer; ++j) rank += sm_keys[j] < key;
     if (rank < k) {
-      sm_front[rank] = base + i;
       fr[rank] = base + i;
+      sm_tok[rank] = tok[base + i];
     }
   }
   __syncthreads();
   // Markov input rows of the next stage: X[r * k + slot] = E_in[token]
-  for (int slot = 0; slot < k; ++slot) {
-    copy_row(E_in, X, tok[sm_front[slot]], r * k + slot, H, x_elem,
-             threadIdx.x, blockDim.x);
-  }
+  gather_rows(E_in, X, sm_tok, k, r * k, H, x_elem);
 }
 
 // ---------------------------------------------------------------------------
@@ -538,7 +611,8 @@ cudaError_t launch_merge(const pctree_config& c, const Layout& lay, int d,
                          int32_t* status, cudaStream_t stream) {
   const int b_d = d == 0 ? 1 : c.k;
   const size_t smem = static_cast<size_t>(b_d) * c.k * sizeof(unsigned long long);
-  merge_kernel<<<c.batch, kMergeThreads, smem, stream>>>(
+  const int threads = b_d * 32 > 256 ? b_d * 32 : 256;
+  merge_kernel<<<c.batch, threads, smem, stream>>>(
       d, c.B, c.k, b_d, c.V, c.H, lay.P, lay.n_chunks, lay.x_elem,
       reinterpret_cast<const float*>(ws + lay.off_pm),
       reinterpret_cast<const float*>(ws + lay.off_ps),
