@@ -328,9 +328,7 @@ def run_ours(args, wl, rank, world, local_rank):
     proj_bytes = args.steps * bytes_round          # timed launches' bytes
     achieved = proj_bytes / (proj_ms / 1e3) / 1e9 if proj_ms > 0 else None
     us_round = ms * 1e3 / args.steps
-    passes = lambda rows: (rows + 255) // 256  # noqa: E731
-    kernels_per_step = 1 + sum(
-        passes(wl.batch * (1 if d == 0 else wl.k)) + 2 for d in range(wl.B)) + 1 + 1
+    kernels_per_step = P.kernels_per_round(cfg) + 1    # + accept
     line = {
         "metric": METRIC, "value": value, "unit": "rounds/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
@@ -344,7 +342,9 @@ def run_ours(args, wl, rank, world, local_rank):
                          "stage; base logits rotate over 16 request sets"},
         "us_per_round": us_round,
         "round_hbm_fraction": (bytes_round / (us_round * 1e-6) / 1e9) / peak,
-        "roofline": {"bound": "hbm", "kernel": "markov_tc_kernel",
+        "roofline": {"bound": "hbm",
+                     "kernel": ("round_fused_kernel" if P.uses_fused_round(cfg)
+                                else "markov_tc_kernel"),
                      "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak if achieved else None,
                      "peak_source": peak_kind,

@@ -205,6 +205,19 @@ PCTREE_API const char* pctree_status_string(int32_t status);
 PCTREE_API pctree_status pctree_profile_enable(int32_t on);
 PCTREE_API pctree_status pctree_profile_collect(int64_t* launches, double* total_ms);
 
+/*
+ * Kernel path.  PCTREE_PATH_AUTO (default) runs rounds with bf16 heads and
+ * batch * k <= 16, k <= 16 as one persistent cooperative launch (all B stages
+ * fused: projection, log-softmax, top-k, merge and frontier); other rounds
+ * run three kernels per stage.  PCTREE_PATH_STAGEWISE forces the per-stage
+ * kernels for every round (same results; used to compare the two).
+ * Process-wide; not thread-safe.  Returns PCTREE_ERR_INVALID_ARG for an
+ * unknown value.
+ */
+#define PCTREE_PATH_AUTO 0
+#define PCTREE_PATH_STAGEWISE 1
+PCTREE_API pctree_status pctree_set_path(int32_t path);
+
 /* ABI version (major * 100 + minor). */
 PCTREE_API int32_t pctree_version(void);
 

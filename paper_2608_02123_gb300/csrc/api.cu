@@ -65,8 +65,16 @@ Layout make_layout(const pctree_config& c) {
   l.off_pt = take(rows * l.n_chunks * c.k * sizeof(int32_t));
   l.off_pool_tok = take(static_cast<size_t>(c.batch) * l.P * sizeof(int32_t));
   l.off_pool_par = take(static_cast<size_t>(c.batch) * l.P * sizeof(int32_t));
-  l.off_pool_s = take(static_cast<size_t>(c.batch) * l.P * sizeof(double));
+  l.off_pool_s = take(static_cast<size_t>(c.batch) * l.P * sizeof(float2));
   l.off_front = take(static_cast<size_t>(c.batch) * c.k * sizeof(int32_t));
+  l.sync_bytes = 2 * static_cast<size_t>(c.B) * sizeof(int);
+  l.off_sync = take(l.sync_bytes);
+  const size_t fparts = static_cast<size_t>(kFusedRows) * kFusedMaxGrid;
+  l.off_fpm = take(fparts * sizeof(float));
+  l.off_fps = take(fparts * sizeof(float));
+  l.off_fcz = take(fparts * c.k * sizeof(float));
+  l.off_fct = take(fparts * c.k * sizeof(int32_t));
+  l.off_xtok = take(static_cast<size_t>(c.batch) * c.k * sizeof(int32_t));
   l.total = off;
   return l;
 }
@@ -152,6 +160,66 @@ pctree_status cuda_status(cudaError_t e) {
   return e == cudaSuccess ? PCTREE_OK : PCTREE_ERR_CUDA;
 }
 
+// The fused round kernel covers bf16 heads with at most 16 Markov rows per
+// stage; larger parent batches take the per-stage kernels.
+int g_path = PCTREE_PATH_AUTO;
+
+bool fused_path(const pctree_config& c) {
+  return g_path == PCTREE_PATH_AUTO && c.weight_dtype == PCTREE_BF16 &&
+         c.batch * c.k <= kFusedRows && c.k <= kFusedMaxK;
+}
+
+pctree_status draft_fused(const pctree_config& c, const Layout& lay,
+                          const float* base_logits, const void* head_emb,
+                          const void* head_out, const int32_t* root_token,
+                          const pctree_tree& out, unsigned char* ws,
+                          int num_sms, cudaStream_t stream) {
+  CUtensorMap tmap_w, tmap_x;
+  pctree_status st = encode_bf16_map(&tmap_w, head_out, c.V, c.H, 128);
+  if (st != PCTREE_OK) return st;
+  st = encode_bf16_map(&tmap_x, ws + lay.off_x, kFusedRows, c.H, kFusedRows);
+  if (st != PCTREE_OK) return st;
+  const int n_tiles = (c.V + 127) / 128;
+  int grid = num_sms < n_tiles ? num_sms : n_tiles;
+  if (grid > kFusedMaxGrid) grid = kFusedMaxGrid;
+  FusedArgs a{};
+  a.L = base_logits;
+  a.V = c.V;
+  a.H = c.H;
+  a.B = c.B;
+  a.k = c.k;
+  a.batch = c.batch;
+  a.P = lay.P;
+  a.n_k = (c.H + 63) / 64;
+  a.n_tiles = n_tiles;
+  a.pool_tok = reinterpret_cast<int32_t*>(ws + lay.off_pool_tok);
+  a.pool_par = reinterpret_cast<int32_t*>(ws + lay.off_pool_par);
+  a.pool_s = reinterpret_cast<float2*>(ws + lay.off_pool_s);
+  a.front = reinterpret_cast<int32_t*>(ws + lay.off_front);
+  a.xtok = reinterpret_cast<int32_t*>(ws + lay.off_xtok);
+  a.E_in = head_emb;
+  a.X = ws + lay.off_x;
+  int* sync = reinterpret_cast<int*>(ws + lay.off_sync);
+  a.stage_cnt = sync;
+  a.ready = sync + c.B;
+  a.part_m = reinterpret_cast<float*>(ws + lay.off_fpm);
+  a.part_s = reinterpret_cast<float*>(ws + lay.off_fps);
+  a.cand_z = reinterpret_cast<float*>(ws + lay.off_fcz);
+  a.cand_t = reinterpret_cast<int32_t*>(ws + lay.off_fct);
+  a.status = out.status;
+  if (cudaMemsetAsync(out.status, 0, sizeof(int32_t), stream) != cudaSuccess ||
+      cudaMemsetAsync(sync, 0, lay.sync_bytes, stream) != cudaSuccess)
+    return PCTREE_ERR_CUDA;
+  st = cuda_status(launch_init(c, lay, root_token, head_emb, ws, out.status,
+                               stream));
+  if (st != PCTREE_OK) return st;
+  prof_record(0, stream);
+  const cudaError_t e = launch_round_fused(&tmap_w, &tmap_x, a, grid, stream);
+  prof_record(1, stream);
+  if (e != cudaSuccess) return PCTREE_ERR_CUDA;
+  return cuda_status(launch_pack(c, lay, ws, out, stream));
+}
+
 }  // namespace
 }  // namespace pct
 
@@ -222,6 +290,8 @@ pctree_status pctree_draft(const pctree_config* cfg, const float* base_logits,
 
   cudaStream_t stream = static_cast<cudaStream_t>(stream_ptr);
   unsigned char* ws = static_cast<unsigned char*>(workspace);
+  if (fused_path(c)) return draft_fused(c, lay, base_logits, head_emb, head_out,
+                                        root_token, *out, ws, num_sms, stream);
   CUtensorMap tmap_w, tmap_x;
   if (c.weight_dtype == PCTREE_BF16) {
     st = encode_bf16_map(&tmap_w, head_out, c.V, c.H, 128);
@@ -277,6 +347,13 @@ pctree_status pctree_accept(const pctree_config* cfg, const pctree_tree* tree,
   return cuda_status(launch_accept(*cfg, *tree, target_tokens, accepted_idx,
                                    accepted_len, bonus_token,
                                    static_cast<cudaStream_t>(stream_ptr)));
+}
+
+pctree_status pctree_set_path(int32_t path) {
+  if (path != PCTREE_PATH_AUTO && path != PCTREE_PATH_STAGEWISE)
+    return PCTREE_ERR_INVALID_ARG;
+  g_path = path;
+  return PCTREE_OK;
 }
 
 pctree_status pctree_profile_enable(int32_t on) {

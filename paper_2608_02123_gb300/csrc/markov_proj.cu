@@ -100,6 +100,7 @@ markov_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
+      const uint64_t stream_policy = l2_policy_evict_first();
       int stage = 0;
       uint32_t phase = 0;
       int armed[8];
@@ -114,7 +115,8 @@ markov_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
           unsigned char* a_dst = ring + stage * C::kStageBytes;
           unsigned char* b_dst = a_dst + C::kABytes;
           mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
-          tma_load_2d(a_dst, &tmap_w, &full[stage], kc * kBK, tile * kBM);
+          tma_load_2d_hint(a_dst, &tmap_w, &full[stage], kc * kBK, tile * kBM,
+                           stream_policy);
           tma_load_2d(b_dst, &tmap_x, &full[stage], kc * kBK, col0);
           armed[stage] = static_cast<int>(phase);
           if (++stage == C::kStages) {

@@ -30,7 +30,34 @@ struct Layout {
   int x_elem;     // bytes per X element
   size_t off_x, off_z, off_pm, off_ps, off_pz, off_pt;
   size_t off_pool_tok, off_pool_par, off_pool_s, off_front;
+  // fused-round path: cross-CTA flags, per-CTA partials, parent tokens
+  size_t off_sync, sync_bytes, off_fpm, off_fps, off_fcz, off_fct, off_xtok;
   size_t total;
+};
+
+// Fused round path limits: at most kFusedRows Markov rows per stage
+// (batch * k), k <= kFusedMaxK, at most kFusedMaxGrid CTAs.
+constexpr int kFusedRows = 16;
+constexpr int kFusedMaxK = 16;
+constexpr int kFusedMaxGrid = 256;
+
+struct FusedArgs {
+  const float* L;        // [batch][B][V] base logits
+  int V, H, B, k, batch, P, n_k, n_tiles;
+  int32_t* pool_tok;     // [batch][P]
+  int32_t* pool_par;     // [batch][P]
+  float2* pool_s;        // [batch][P] joint score as (hi, lo)
+  int32_t* front;        // [batch][k] frontier pool ids
+  int32_t* xtok;         // [batch * k] parent tokens of the next stage
+  const void* E_in;      // [V][H] bf16 Markov input rows
+  void* X;               // [kFusedRows][H] bf16 parent rows of the stage
+  int* stage_cnt;        // [B] CTAs done with stage d
+  int* ready;            // [B] parent tokens of stage d published
+  float* part_m;         // [kFusedRows][grid] per-CTA max
+  float* part_s;         // [kFusedRows][grid] per-CTA sum of exp
+  float* cand_z;         // [kFusedRows][grid][k] per-CTA top-k logits
+  int32_t* cand_t;       // [kFusedRows][grid][k] per-CTA top-k tokens
+  int32_t* status;
 };
 
 // Pool id of the first node of level t (t >= 1).  Level 1 has k nodes, every
@@ -151,6 +178,56 @@ __device__ __forceinline__ void lse_merge(float& m, float& s, float m2,
   m = M;
 }
 
+// Log-sum-exp normaliser of one row (Eq. 2) from n per-chunk (max, sum-exp)
+// partials, in float32: a warp max, then each lane rescales and sums its
+// partials, then a warp sum.  Returns -inf when no partial is finite.  Kept
+// compact: it runs once per stage from a cold instruction cache.
+template <int U>
+__device__ __forceinline__ float warp_lse_from_partials(const float* pm,
+                                                        const float* ps,
+                                                        int n) {
+  const int lane = threadIdx.x & 31;
+  float M = -INFINITY, S = 0.0f;
+  for (int c0 = 0; c0 < n; c0 += 32 * U) {
+    float mv[U], sv[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int c = c0 + u * 32 + lane;
+      mv[u] = c < n ? pm[c] : -INFINITY;
+      sv[u] = c < n ? ps[c] : 0.0f;
+    }
+    float Mc = -INFINITY;
+#pragma unroll
+    for (int u = 0; u < U; ++u) Mc = fmaxf(Mc, mv[u]);
+    float Sc = 0.0f;
+    if (Mc > -INFINITY) {
+#pragma unroll
+      for (int u = 0; u < U; ++u) Sc += sv[u] * expf(mv[u] - Mc);
+    }
+    lse_merge(M, S, Mc, Sc);
+  }
+  float Mw = M;
+#pragma unroll 1
+  for (int o = 16; o > 0; o >>= 1) Mw = fmaxf(Mw, __shfl_xor_sync(kFull, Mw, o));
+  float Sw = M > -INFINITY ? S * expf(M - Mw) : 0.0f;
+#pragma unroll 1
+  for (int o = 16; o > 0; o >>= 1) Sw += __shfl_xor_sync(kFull, Sw, o);
+  return Mw == -INFINITY ? -INFINITY : Mw + logf(Sw);
+}
+
+// Joint scores are accumulated along a path as an unevaluated float pair
+// (hi, lo) with hi + lo exact: each step adds a float log-probability with
+// an error-free transformation (Knuth's TwoSum), so the only rounding left is
+// in the log-probabilities themselves.  hi is the score rounded to float.
+__device__ __forceinline__ float2 ff_add(float2 a, float b) {
+  const float s = a.x + b;
+  if (!isfinite(s)) return make_float2(s, 0.0f);
+  const float bb = s - a.x;
+  const float e = (a.x - (s - bb)) + (b - bb) + a.y;
+  const float hi = s + e;
+  return make_float2(hi, e - (hi - s));
+}
+
 __device__ __forceinline__ void set_status(int32_t* status, int code) {
   atomicCAS(status, 0, code);
 }
@@ -174,6 +251,12 @@ cudaError_t launch_markov_f32(const float* W_out, const float* X,
                               int ldz, int V, int H, int rows,
                               int rows_per_req, int32_t* status,
                               cudaStream_t stream);
+
+// One drafting round's B stages in one cooperative launch (fused path).
+cudaError_t launch_round_fused(const CUtensorMap* tmap_w,
+                               const CUtensorMap* tmap_x, const FusedArgs& args,
+                               int grid, cudaStream_t stream);
+size_t round_fused_smem_bytes();
 
 cudaError_t launch_init(const pctree_config& c, const Layout& lay,
                         const int32_t* root, const void* E_in,

@@ -1,0 +1,559 @@
+// One whole PCTree drafting round (Algorithm 1, stages d = 0..B-1) in a single
+// persistent, cooperative launch, for rounds with at most 16 Markov rows per
+// stage (batch * k <= 16, k <= 16) -- the batch-1 drafting of Sec. 5.
+//
+// Per stage d, every CTA (one per SM) streams its share of W_out tiles with
+// TMA and multiplies them on the tensor cores (tcgen05, bf16 -> f32 in TMEM)
+// against the stage's parent rows X = E_in[parent tokens] (Eq. 3), a 16-row
+// buffer in global memory loaded with one TMA box per ring slot.  The epilogue adds the shared base
+// logits L_d and keeps, per parent, a running log-sum-exp (Eq. 2) and a
+// warp-resident top-k list -- the stage logits never reach HBM.  When a CTA
+// has finished its tiles it publishes per-CTA partials; the last CTA to
+// arrive (atomic ticket, no waiting) merges them: per-parent normaliser and
+// top-k children, joint scores s(child) = s(p) + log pi (Eq. 4), the pool
+// push, the layer-wise frontier (Sec. 4.1) and the next stage's parent rows,
+// then releases a flag.  Producers keep prefetching the next stage's
+// W_out tiles while that merge runs and only hold back the parent-row loads
+// until the flag is set.
+//
+// Warp roles: warp 0 TMA producer, warp 1 TMEM allocator + MMA issuer,
+// warps 2..5 epilogue (TMEM lane quadrant = warp % 4) and merge.
+#include <cuda_runtime.h>
+
+#include "pctree_common.cuh"
+#include "sm103_ptx.cuh"
+
+namespace pct {
+namespace {
+
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+constexpr int kUmmaK = 16;
+constexpr int kBN = kFusedRows;                  // Markov rows per stage (max)
+constexpr int kMaxKF = kFusedMaxK;               // k limit of this path
+constexpr int kThreads = 192;
+constexpr int kEpiWarps = 4;
+constexpr int kABytes = kBM * kBK * 2;           // 16 KB of W_out per slot
+constexpr int kBBytes = kBN * kBK * 2;           // 2 KB of parent rows
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kStages = 8;
+constexpr int kTmemCols = 32;                    // two 16-column accumulators
+constexpr uint64_t kLimitNs = 1000000000ull;     // 1 s per bounded wait
+constexpr float kNegInf = -INFINITY;
+
+struct FusedSmem {
+  uint64_t full[kStages], empty[kStages], acc_full[2], acc_empty[2], drain;
+  uint32_t tmem_slot;
+  int abort;
+  int ticket;
+  float lv[kEpiWarps][kBN][kMaxKF];        // per-warp top-k lists per row
+  int lt[kEpiWarps][kBN][kMaxKF];
+  union {
+    struct {                               // per-thread (max, sum-exp)
+      float m[kBN][kEpiWarps * 32];
+      float s[kBN][kEpiWarps * 32];
+    } part;
+    struct {                               // merge: 32 CTAs' lists per warp
+      float z[kEpiWarps][kMaxKF][32];
+      int t[kEpiWarps][kMaxKF][32];
+    } stage;
+  } u;
+  unsigned long long keys[kBN * kMaxKF];   // new layer: (score, id) keys
+  int ktok[kBN * kMaxKF];                  // new layer: tokens
+  int ftok[kBN];                           // next stage's parent tokens
+};
+
+constexpr size_t kSmemBytes =
+    1024 + static_cast<size_t>(kStages) * kStageBytes + sizeof(FusedSmem);
+
+__device__ __forceinline__ void epi_barrier() { named_barrier(1, kEpiWarps * 32); }
+
+// --------------------------------------------------------------------------
+// producer: W_out tiles (A) and parent rows (B) into the shared-memory ring
+// --------------------------------------------------------------------------
+
+__device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
+                        const FusedArgs& a, unsigned char* ring, FusedSmem* S,
+                        volatile int* abort_v) {
+  const int grid = gridDim.x;
+  const uint64_t stream_policy = l2_policy_evict_first();
+  int stage = 0;
+  uint32_t phase = 0;
+  int armed[kStages];
+#pragma unroll
+  for (int s = 0; s < kStages; ++s) armed[s] = -1;
+  int pend_stage[kStages], pend_kc[kStages];
+  bool ok = true;
+
+  for (int d = 0; d < a.B && ok; ++d) {
+    constexpr uint32_t tx = kABytes + kBBytes;
+    bool have = d == 0;   // stage 0 rows were written before the launch
+    int n_pend = 0;
+    auto acquire_rows = [&]() {
+      fence_proxy_async_global();   // rows written by another CTA's merge
+    };
+    auto issue_rows = [&](int st, int kc) {
+      tma_load_2d(ring + st * kStageBytes + kABytes, tmap_x, &S->full[st],
+                  kc * kBK, 0);
+    };
+    for (int tile = blockIdx.x; tile < a.n_tiles && ok; tile += grid) {
+      for (int kc = 0; kc < a.n_k; ++kc) {
+        if (!have) {
+          bool rdy = poll_flag(&a.ready[d]);
+          if (!rdy && n_pend == kStages) {
+            if (!wait_flag_bounded(&a.ready[d], abort_v, kLimitNs)) {
+              ok = false;
+              break;
+            }
+            rdy = true;
+          }
+          if (rdy) {
+            acquire_rows();
+            have = true;
+            for (int p = 0; p < n_pend; ++p) issue_rows(pend_stage[p], pend_kc[p]);
+            n_pend = 0;
+          }
+        }
+        if (!mbar_wait_bounded(&S->empty[stage], phase ^ 1u, abort_v, kLimitNs)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(&S->full[stage], tx);
+        tma_load_2d_hint(ring + stage * kStageBytes, tmap_w, &S->full[stage],
+                         kc * kBK, tile * kBM, stream_policy);
+        if (have) {
+          issue_rows(stage, kc);
+        } else {
+          pend_stage[n_pend] = stage;
+          pend_kc[n_pend] = kc;
+          ++n_pend;
+        }
+        armed[stage] = static_cast<int>(phase);
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+    if (ok && !have) {
+      if (!wait_flag_bounded(&a.ready[d], abort_v, kLimitNs)) {
+        ok = false;
+      } else {
+        acquire_rows();
+        for (int p = 0; p < n_pend; ++p) issue_rows(pend_stage[p], pend_kc[p]);
+      }
+    }
+  }
+  if (!ok) {
+    *abort_v = 1;
+    set_status(a.status, PCTREE_ERR_TIMEOUT);
+  }
+  // every copy issued here must land before the CTA may exit
+  volatile int never = 0;
+  for (int s = 0; s < kStages; ++s)
+    if (armed[s] >= 0)
+      mbar_wait_bounded(&S->full[s], static_cast<uint32_t>(armed[s]), &never,
+                        kLimitNs);
+}
+
+// --------------------------------------------------------------------------
+// MMA issuer
+// --------------------------------------------------------------------------
+
+__device__ void mma(const FusedArgs& a, unsigned char* ring, FusedSmem* S,
+                    uint32_t tmem_base, volatile int* abort_v) {
+  constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN);
+  const int grid = gridDim.x;
+  int stage = 0;
+  uint32_t phase = 0;
+  int acc = 0;
+  uint32_t acc_phase = 0;
+  bool ok = true;
+  for (int d = 0; d < a.B && ok; ++d) {
+    for (int tile = blockIdx.x; tile < a.n_tiles && ok; tile += grid) {
+      if (!mbar_wait_bounded(&S->acc_empty[acc], acc_phase ^ 1u, abort_v, kLimitNs)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after_sync();
+      const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * kBN);
+      for (int kc = 0; kc < a.n_k; ++kc) {
+        if (!mbar_wait_bounded(&S->full[stage], phase, abort_v, kLimitNs)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after_sync();
+        const uint32_t a_addr = smem_u32(ring + stage * kStageBytes);
+        const uint32_t b_addr = a_addr + kABytes;
+#pragma unroll
+        for (int kk = 0; kk < kBK / kUmmaK; ++kk) {
+          tc_mma_bf16(d_tmem, desc_kmajor_sw128(a_addr + kk * kUmmaK * 2),
+                      desc_kmajor_sw128(b_addr + kk * kUmmaK * 2), idesc,
+                      (kc | kk) != 0 ? 1u : 0u);
+        }
+        tc_commit(&S->empty[stage]);
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      if (!ok) break;
+      tc_commit(&S->acc_full[acc]);
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1u;
+    }
+  }
+  if (!ok) {
+    *abort_v = 1;
+    set_status(a.status, PCTREE_ERR_TIMEOUT);
+  }
+  tc_commit(&S->drain);
+  volatile int never = 0;
+  mbar_wait_bounded(&S->drain, 0, &never, kLimitNs);
+}
+
+// --------------------------------------------------------------------------
+// merge of stage d by the last CTA (the four epilogue warps)
+// --------------------------------------------------------------------------
+
+__device__ void merge_stage(const FusedArgs& a, FusedSmem* S, int d) {
+  const int ew = (threadIdx.x >> 5) - 2;   // 0..3
+  const int lane = threadIdx.x & 31;
+  const int tid = ew * 32 + lane;          // 0..127
+  const int grid = gridDim.x;
+  const int b_d = d == 0 ? 1 : a.k;
+  const int rows = a.batch * b_d;
+  const int k = a.k;
+  const int n_layer = b_d * k;
+  const int base = level_base(d + 1, k);
+  if (d > 0) (void)ld_acquire_gpu(&a.ready[d]);   // pool of earlier stages
+  for (int c = ew; c < rows; c += kEpiWarps) {
+    // log-softmax normaliser of parent row c over all CTAs' partials (Eq. 2)
+    const float lse = warp_lse_from_partials<8>(
+        a.part_m + static_cast<size_t>(c) * grid,
+        a.part_s + static_cast<size_t>(c) * grid, grid);
+    if (lse == kNegInf && lane == 0) set_status(a.status, PCTREE_ERR_NONFINITE);
+    // Every CTA list is sorted best first.  Pass 1: the top-k of the CTAs'
+    // first entries; its k-th value T is a lower bound of the row's k-th
+    // value (k distinct CTAs hold an entry >= T).  Pass 2: only CTAs whose
+    // first entry is >= T can hold further children; their lower ranks are
+    // offered.  Loops stay rolled: this code runs once per stage.
+    const float* cz = a.cand_z + static_cast<size_t>(c) * grid * k;
+    const int32_t* ct = a.cand_t + static_cast<size_t>(c) * grid * k;
+    constexpr int kG = kFusedMaxGrid / 32;
+    float(*sz)[32] = S->u.stage.z[ew];
+    int(*st)[32] = S->u.stage.t[ew];
+#pragma unroll
+    for (int u = 0; u < kG; ++u) {
+      const int g = u * 32 + lane;
+      const float v = g < grid ? cz[static_cast<size_t>(g) * k] : kNegInf;
+      const int t = g < grid ? ct[static_cast<size_t>(g) * k] : 0x7fffffff;
+      sz[u][lane] = v;
+      st[u][lane] = t;
+    }
+    __syncwarp();
+    WarpList lst;
+    lst.seed(sz[0][lane], st[0][lane], k);
+#pragma unroll 1
+    for (int u = 1; u < kG; ++u) lst.offer(sz[u][lane], st[u][lane], k);
+    const float T = __shfl_sync(kFull, lst.v, k - 1);
+#pragma unroll 1
+    for (int u = 0; u < kG; ++u) {
+      unsigned q = __ballot_sync(kFull, u * 32 + lane < grid && sz[u][lane] >= T &&
+                                            st[u][lane] != 0x7fffffff);
+      // ranks 1..k-1 of up to 32/(k-1) qualifying CTAs per warp-wide load
+      while (q) {
+        const int per = 32 / (k - 1 > 0 ? k - 1 : 1);
+        int g_lane = -1, r_lane = 0;
+        unsigned take = q;
+        for (int n = 0; n < per && take; ++n) {
+          const int src = __ffs(take) - 1;
+          take &= take - 1;
+          if (k > 1 && lane >= n * (k - 1) && lane < (n + 1) * (k - 1)) {
+            g_lane = u * 32 + src;
+            r_lane = 1 + lane - n * (k - 1);
+          }
+        }
+        q = take;
+        float v = kNegInf;
+        int t = 0x7fffffff;
+        if (g_lane >= 0) {
+          v = cz[static_cast<size_t>(g_lane) * k + r_lane];
+          t = ct[static_cast<size_t>(g_lane) * k + r_lane];
+        }
+        const bool ok = g_lane >= 0 && v >= T && t != 0x7fffffff;
+        lst.offer(ok ? v : kNegInf, ok ? t : 0x7fffffff, k);
+      }
+    }
+    __syncwarp();
+    const int req = c / b_d, j = c - req * b_d;
+    int32_t* tok = a.pool_tok + static_cast<size_t>(req) * a.P;
+    int32_t* par = a.pool_par + static_cast<size_t>(req) * a.P;
+    float2* sc = a.pool_s + static_cast<size_t>(req) * a.P;
+    const int pid = a.front[req * k + j];
+    if (lane < k) {
+      const int id = base + j * k + lane;
+      int t = lst.t;
+      float logpi = lst.v - lse;
+      if (t < 0 || t >= a.V) {
+        t = 0;
+        logpi = kNegInf;
+      }
+      const float2 sp = sc[pid];
+      const float2 sn = ff_add(sp, logpi);   // Eq. 4
+      tok[id] = t;
+      par[id] = pid;
+      sc[id] = sn;
+      const int i = req * n_layer + j * k + lane;
+      S->keys[i] = (static_cast<unsigned long long>(desc_key(sn.x)) << 32) |
+                   static_cast<unsigned int>(id);
+      S->ktok[i] = t;
+    }
+  }
+  if (d == a.B - 1) return;
+  epi_barrier();
+  // frontier of each request: the k best nodes of the new layer
+  const int total = a.batch * n_layer;
+  for (int i = tid; i < total; i += kEpiWarps * 32) {
+    const int req = i / n_layer;
+    const unsigned long long key = S->keys[i];
+    int rank = 0;
+    for (int jj = req * n_layer; jj < (req + 1) * n_layer; ++jj) rank += S->keys[jj] < key;
+    if (rank < k) {
+      a.front[req * k + rank] = static_cast<int>(key & 0xffffffffu);
+      a.xtok[req * k + rank] = S->ktok[i];
+      S->ftok[req * k + rank] = S->ktok[i];
+    }
+  }
+  epi_barrier();
+  // parent rows of the next stage: X[req * k + slot] = E_in[token]
+  constexpr int kG8 = 10;
+  const int per_row = a.H / 8;
+  const int total_v = a.batch * k * per_row;
+  const uint4* src = static_cast<const uint4*>(a.E_in);
+  uint4* dst = static_cast<uint4*>(a.X);
+  for (int i0 = tid; i0 < total_v; i0 += kEpiWarps * 32 * kG8) {
+    uint4 tmp[kG8];
+#pragma unroll
+    for (int u = 0; u < kG8; ++u) {
+      const int i = i0 + u * kEpiWarps * 32;
+      if (i < total_v) {
+        const int row = i / per_row, off = i - row * per_row;
+        tmp[u] = src[static_cast<size_t>(S->ftok[row]) * per_row + off];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kG8; ++u) {
+      const int i = i0 + u * kEpiWarps * 32;
+      if (i < total_v) {
+        const int row = i / per_row, off = i - row * per_row;
+        dst[static_cast<size_t>(row) * per_row + off] = tmp[u];
+      }
+    }
+  }
+  fence_proxy_async_global();   // the rows are read with TMA by every CTA
+  __threadfence();
+  epi_barrier();
+  if (tid == 0) st_release_gpu(&a.ready[d + 1], 1);
+}
+
+// --------------------------------------------------------------------------
+// epilogue: TMEM -> registers, online log-sum-exp and top-k per parent row
+// --------------------------------------------------------------------------
+
+__device__ void epilogue(const FusedArgs& a, FusedSmem* S, uint32_t tmem_base,
+                         volatile int* abort_v) {
+  const int warp = threadIdx.x >> 5;
+  const int ew = warp - 2;
+  const int quad = warp & 3;
+  const int lane = threadIdx.x & 31;
+  const int grid = gridDim.x;
+  const int k = a.k;
+  int acc = 0;
+  uint32_t acc_phase = 0;
+  bool bad = false;
+  for (int d = 0; d < a.B; ++d) {
+    const int b_d = d == 0 ? 1 : k;
+    const int rows = a.batch * b_d;
+    float m[kBN], s[kBN];
+    WarpList lst[kBN];
+#pragma unroll
+    for (int c = 0; c < kBN; ++c) {
+      m[c] = kNegInf;
+      s[c] = 0.0f;
+      lst[c].reset();
+    }
+    bool first = true;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < a.n_tiles; tile += grid) {
+      if (!mbar_wait_bounded(&S->acc_full[acc], acc_phase, abort_v, kLimitNs)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after_sync();
+      uint32_t r[16];
+      tmem_ld_32x32b_x16(tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                             static_cast<uint32_t>(acc * kBN),
+                         r);
+      tmem_ld_wait();
+      tc_fence_before_sync();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&S->acc_empty[acc]);
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1u;
+      const int v = tile * kBM + quad * 32 + lane;
+      const bool inb = v < a.V;
+      const float* Lrow = a.L + static_cast<size_t>(d) * a.V + (inb ? v : 0);
+#pragma unroll
+      for (int c = 0; c < kBN; ++c) {
+        if (c < rows) {
+          const int req = c / b_d;
+          float z = kNegInf;
+          int t = 0x7fffffff;
+          if (inb) {
+            const float lval = __ldg(Lrow + static_cast<size_t>(req) * a.B * a.V);
+            z = lval + __uint_as_float(r[c]);
+            t = v;
+            bad |= isnan(z) || (isinf(z) && !(isinf(lval) && lval < 0.0f));
+            lse_push(m[c], s[c], z);
+          }
+          if (first) {
+            lst[c].seed(z, t, k);
+          } else {
+            lst[c].offer(z, t, k);
+          }
+        }
+      }
+      first = false;
+    }
+    if (!ok) {
+      *abort_v = 1;
+      set_status(a.status, PCTREE_ERR_TIMEOUT);
+      break;
+    }
+    // per-thread (max, sum-exp) and per-warp lists to shared memory
+    const int tid = ew * 32 + lane;
+#pragma unroll
+    for (int c = 0; c < kBN; ++c) {
+      if (c < rows) {
+        S->u.part.m[c][tid] = m[c];
+        S->u.part.s[c][tid] = s[c];
+        if (lane < k) {
+          S->lv[ew][c][lane] = lst[c].v;
+          S->lt[ew][c][lane] = lst[c].t;
+        }
+      }
+    }
+    epi_barrier();
+    // per-CTA partials of the rows this warp owns (rolled: runs once per
+    // stage from a cold instruction cache)
+#pragma unroll 1
+    for (int c = ew; c < rows; c += kEpiWarps) {
+      float mm = kNegInf, ss = 0.0f;
+#pragma unroll
+      for (int q = 0; q < kEpiWarps; ++q)
+        lse_merge(mm, ss, S->u.part.m[c][q * 32 + lane], S->u.part.s[c][q * 32 + lane]);
+#pragma unroll 1
+      for (int o = 16; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(kFull, mm, o);
+        const float s2 = __shfl_xor_sync(kFull, ss, o);
+        lse_merge(mm, ss, m2, s2);
+      }
+      if (lane == 0) {
+        a.part_m[static_cast<size_t>(c) * grid + blockIdx.x] = mm;
+        a.part_s[static_cast<size_t>(c) * grid + blockIdx.x] = ss;
+      }
+      WarpList cl;
+      cl.seed(lane < k ? S->lv[0][c][lane] : kNegInf,
+              lane < k ? S->lt[0][c][lane] : 0x7fffffff, k);
+#pragma unroll 1
+      for (int w = 1; w < kEpiWarps; ++w)
+        cl.offer(lane < k ? S->lv[w][c][lane] : kNegInf,
+                 lane < k ? S->lt[w][c][lane] : 0x7fffffff, k);
+      if (lane < k) {   // this CTA's top-k of row c, best first
+        const size_t o = (static_cast<size_t>(c) * grid + blockIdx.x) * k + lane;
+        a.cand_z[o] = cl.v;
+        a.cand_t[o] = cl.t;
+      }
+    }
+    __threadfence();
+    epi_barrier();
+    if (ew == 0 && lane == 0) S->ticket = atomicAdd(&a.stage_cnt[d], 1);
+    epi_barrier();
+    if (S->ticket == grid - 1) {
+      __threadfence();
+      merge_stage(a, S, d);
+    }
+    epi_barrier();
+  }
+  if (bad) set_status(a.status, PCTREE_ERR_NONFINITE);
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+round_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
+                   const __grid_constant__ CUtensorMap tmap_x,
+                   const __grid_constant__ FusedArgs a) {
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* ring = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  FusedSmem* S = reinterpret_cast<FusedSmem*>(ring + kStages * kStageBytes);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&S->full[s], 1);
+      mbar_init(&S->empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&S->acc_full[i], 1);
+      mbar_init(&S->acc_empty[i], kEpiWarps);
+    }
+    mbar_init(&S->drain, 1);
+    S->abort = 0;
+    fence_barrier_init();
+    tma_prefetch_desc(&tmap_w);
+    tma_prefetch_desc(&tmap_x);
+  }
+  if (warp == 1) tmem_alloc(&S->tmem_slot, kTmemCols);
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  const uint32_t tmem_base = S->tmem_slot;
+  volatile int* abort_v = &S->abort;
+  if (warp == 0) {
+    if (lane == 0) produce(&tmap_w, &tmap_x, a, ring, S, abort_v);
+  } else if (warp == 1) {
+    if (lane == 0) mma(a, ring, S, tmem_base, abort_v);
+  } else {
+    epilogue(a, S, tmem_base, abort_v);
+  }
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  if (warp == 1) tmem_dealloc(tmem_base, kTmemCols);
+}
+
+}  // namespace
+
+size_t round_fused_smem_bytes() { return kSmemBytes; }
+
+cudaError_t launch_round_fused(const CUtensorMap* tmap_w,
+                               const CUtensorMap* tmap_x, const FusedArgs& args,
+                               int grid, cudaStream_t stream) {
+  static bool attr_done = false;
+  if (!attr_done) {
+    cudaError_t e = cudaFuncSetAttribute(round_fused_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(kSmemBytes));
+    if (e != cudaSuccess) return e;
+    attr_done = true;
+  }
+  CUtensorMap w = *tmap_w, x = *tmap_x;
+  FusedArgs a = args;
+  void* params[] = {&w, &x, &a};
+  return cudaLaunchCooperativeKernel(reinterpret_cast<void*>(round_fused_kernel),
+                                     dim3(grid), dim3(kThreads), params,
+                                     kSmemBytes, stream);
+}
+
+}  // namespace pct

@@ -45,7 +45,7 @@ __device__ void copy_row(const void* E_in, void* X, int token, int row, int H,
 
 __global__ void init_kernel(const int32_t* __restrict__ root, const void* E_in,
                             void* X, int32_t* pool_tok, int32_t* pool_par,
-                            double* pool_s, int32_t* front, int V, int H,
+                            float2* pool_s, int32_t* front, int V, int H,
                             int P, int k, int x_elem, int32_t* status) {
   const int r = blockIdx.x;
   int tok = root[r];
@@ -56,7 +56,7 @@ __global__ void init_kernel(const int32_t* __restrict__ root, const void* E_in,
   if (threadIdx.x == 0) {
     pool_tok[static_cast<size_t>(r) * P] = tok;
     pool_par[static_cast<size_t>(r) * P] = -1;
-    pool_s[static_cast<size_t>(r) * P] = 0.0;  // s(root) = 0 (Sec. 4.2)
+    pool_s[static_cast<size_t>(r) * P] = make_float2(0.0f, 0.0f);  // s(root) = 0
     front[static_cast<size_t>(r) * k] = 0;
   }
   copy_row(E_in, X, tok, r, H, x_elem, threadIdx.x, blockDim.x);
@@ -202,7 +202,7 @@ merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
              const float* __restrict__ part_s,
              const float* __restrict__ part_z,
              const int32_t* __restrict__ part_t, int32_t* pool_tok,
-             int32_t* pool_par, double* pool_s, int32_t* front,
+             int32_t* pool_par, float2* pool_s, int32_t* front,
              const void* E_in, void* X, int32_t* status) {
   const int r = blockIdx.x;
   const int lane = threadIdx.x & 31;
@@ -212,7 +212,7 @@ merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
 
   int32_t* tok = pool_tok + static_cast<size_t>(r) * P;
   int32_t* par = pool_par + static_cast<size_t>(r) * P;
-  double* sc = pool_s + static_cast<size_t>(r) * P;
+  float2* sc = pool_s + static_cast<size_t>(r) * P;
   int32_t* fr = front + static_cast<size_t>(r) * k;
   const int base = level_base(d + 1, k);
 
@@ -220,38 +220,10 @@ merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
     const int j = warp;
     const int row = r * b_d + j;
     const size_t p0 = static_cast<size_t>(row) * n_chunks;
-    // log-softmax normaliser from the chunk partials (Eq. 2), in float64
-    float Mf = kNegInf;
-    for (int c0 = 0; c0 < n_chunks; c0 += 32 * kUnroll) {
-      float mv[kUnroll];
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
-        const int c = c0 + u * 32 + lane;
-        mv[u] = c < n_chunks ? part_m[p0 + c] : kNegInf;
-      }
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u) Mf = fmaxf(Mf, mv[u]);
-    }
-    for (int o = 16; o > 0; o >>= 1) Mf = fmaxf(Mf, __shfl_xor_sync(kFull, Mf, o));
-    double S = 0.0;
-    if (Mf > kNegInf) {
-      for (int c0 = 0; c0 < n_chunks; c0 += 32 * kUnroll) {
-        float mv[kUnroll], sv[kUnroll];
-#pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-          const int c = c0 + u * 32 + lane;
-          mv[u] = c < n_chunks ? part_m[p0 + c] : kNegInf;
-          sv[u] = c < n_chunks ? part_s[p0 + c] : 0.0f;
-        }
-#pragma unroll
-        for (int u = 0; u < kUnroll; ++u)
-          if (mv[u] > kNegInf) S += (double)sv[u] * exp((double)mv[u] - (double)Mf);
-      }
-    } else if (lane == 0) {
-      set_status(status, PCTREE_ERR_NONFINITE);
-    }
-    for (int o = 16; o > 0; o >>= 1) S += __shfl_xor_sync(kFull, S, o);
-    const double lse = (double)Mf + log(S);
+    // log-softmax normaliser from the chunk partials (Eq. 2)
+    const float lse = warp_lse_from_partials<kUnroll>(part_m + p0, part_s + p0,
+                                                      n_chunks);
+    if (lse == kNegInf && lane == 0) set_status(status, PCTREE_ERR_NONFINITE);
     // top-k children of this parent over every chunk's list
     WarpList lst;
     lst.reset();
@@ -280,14 +252,14 @@ merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
     if (lane < k) {
       const int id = base + j * k + lane;
       int t = lst.t;
-      double logpi = (double)lst.v - lse;
+      float logpi = lst.v - lse;
       if (t < 0 || t >= V) {  // only when V < k (rejected on the host)
         t = 0;
-        logpi = -INFINITY;
+        logpi = kNegInf;
       }
       tok[id] = t;
       par[id] = pid;
-      sc[id] = sc[pid] + logpi;  // Eq. 4: s(child) = s(p) + log pi(child|p)
+      sc[id] = ff_add(sc[pid], logpi);  // Eq. 4: s(child) = s(p) + log pi
     }
   }
   if (d == B - 1) return;
@@ -296,7 +268,7 @@ merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
   const int n_layer = b_d * k;
   for (int i = threadIdx.x; i < n_layer; i += blockDim.x) {
     const int id = base + i;
-    sm_keys[i] = (static_cast<unsigned long long>(desc_key((float)sc[id])) << 32) |
+    sm_keys[i] = (static_cast<unsigned long long>(desc_key(sc[id].x)) << 32) |
                  static_cast<unsigned int>(id);
   }
   __syncthreads();
@@ -349,7 +321,7 @@ __global__ void __launch_bounds__(kPackThreads)
 pack_kernel(int B, int k, int N, int P, int pos_offset,
             const int32_t* __restrict__ pool_tok,
             const int32_t* __restrict__ pool_par,
-            const double* __restrict__ pool_s, pctree_tree out) {
+            const float2* __restrict__ pool_s, pctree_tree out) {
   const int r = blockIdx.x;
   const int tid = threadIdx.x;
   extern __shared__ unsigned long long sm_key[];  // P keys; later reused
@@ -363,14 +335,14 @@ pack_kernel(int B, int k, int N, int P, int pos_offset,
 
   const int32_t* tok = pool_tok + static_cast<size_t>(r) * P;
   const int32_t* par = pool_par + static_cast<size_t>(r) * P;
-  const double* sc = pool_s + static_cast<size_t>(r) * P;
+  const float2* sc = pool_s + static_cast<size_t>(r) * P;
   const int n = min(N, P);
 
   // 46-bit keys: descending fp32 score in bits 45..14, pool id in 13..0.
   // Ids grow with depth, so (score desc, id asc) is (score desc, depth asc,
   // id asc) of Sec. 4.2.
   for (int i = tid; i < P; i += blockDim.x) {
-    sm_key[i] = (static_cast<unsigned long long>(desc_key((float)sc[i])) << 14) |
+    sm_key[i] = (static_cast<unsigned long long>(desc_key(sc[i].x)) << 14) |
                 static_cast<unsigned long long>(i);
   }
   if (tid == 0) {
@@ -489,7 +461,7 @@ pack_kernel(int B, int k, int N, int P, int pos_offset,
       o_tok[a] = tok[id];
       o_par[a] = sm_par[a];
       o_dep[a] = lvl;
-      o_lp[a] = (float)sc[id];
+      o_lp[a] = sc[id].x;
       o_pos[a] = lvl + pos_offset;  // siblings share a position (Appendix A)
     } else {
       o_tok[a] = -1;
@@ -526,7 +498,7 @@ pack_kernel(int B, int k, int N, int P, int pos_offset,
     for (int i = tid; i < P; i += blockDim.x) {
       out.pool_token[static_cast<size_t>(r) * P + i] = tok[i];
       out.pool_parent[static_cast<size_t>(r) * P + i] = par[i];
-      out.pool_logp[static_cast<size_t>(r) * P + i] = (float)sc[i];
+      out.pool_logp[static_cast<size_t>(r) * P + i] = sc[i].x;
     }
   }
 }
@@ -587,7 +559,7 @@ cudaError_t launch_init(const pctree_config& c, const Layout& lay,
   init_kernel<<<c.batch, 256, 0, stream>>>(
       root, E_in, ws + lay.off_x, reinterpret_cast<int32_t*>(ws + lay.off_pool_tok),
       reinterpret_cast<int32_t*>(ws + lay.off_pool_par),
-      reinterpret_cast<double*>(ws + lay.off_pool_s),
+      reinterpret_cast<float2*>(ws + lay.off_pool_s),
       reinterpret_cast<int32_t*>(ws + lay.off_front), c.V, c.H, lay.P, c.k,
       lay.x_elem, status);
   return cudaGetLastError();
@@ -620,7 +592,7 @@ cudaError_t launch_merge(const pctree_config& c, const Layout& lay, int d,
       reinterpret_cast<const int32_t*>(ws + lay.off_pt),
       reinterpret_cast<int32_t*>(ws + lay.off_pool_tok),
       reinterpret_cast<int32_t*>(ws + lay.off_pool_par),
-      reinterpret_cast<double*>(ws + lay.off_pool_s),
+      reinterpret_cast<float2*>(ws + lay.off_pool_s),
       reinterpret_cast<int32_t*>(ws + lay.off_front), E_in, ws + lay.off_x,
       status);
   return cudaGetLastError();
@@ -640,7 +612,7 @@ cudaError_t launch_pack(const pctree_config& c, const Layout& lay,
       c.B, c.k, c.N, lay.P, c.pos_offset,
       reinterpret_cast<const int32_t*>(ws + lay.off_pool_tok),
       reinterpret_cast<const int32_t*>(ws + lay.off_pool_par),
-      reinterpret_cast<const double*>(ws + lay.off_pool_s), out);
+      reinterpret_cast<const float2*>(ws + lay.off_pool_s), out);
   return cudaGetLastError();
 }
 

@@ -109,6 +109,27 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map,
       : "memory");
 }
 
+// L2 policy for data read once per pass (the streamed head matrix): its lines
+// are the first evicted, so the stream does not flush the small, reused data
+// (base logits, parent rows, partials) and the kernel's own instructions.
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+// tma_load_2d with an L2 cache policy from createpolicy.
+__device__ __forceinline__ void tma_load_2d_hint(void* dst, const CUtensorMap* map,
+                                                 uint64_t* bar, int32_t x,
+                                                 int32_t y, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::"
+      "bytes.L2::cache_hint [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y),
+      "l"(policy)
+      : "memory");
+}
+
 // ---------------------------------------------------------------------------
 // tcgen05: tensor memory, MMA, commit, loads
 // ---------------------------------------------------------------------------
@@ -202,6 +223,71 @@ __device__ __forceinline__ void tmem_ld_32x32b_x16(uint32_t taddr,
 
 __device__ __forceinline__ void tmem_ld_wait() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+}  // namespace pct
+
+namespace pct {
+
+// ---------------------------------------------------------------------------
+// cross-CTA flags (global memory)
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_release_gpu(int* p, int v) {
+  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ int ld_relaxed_gpu(const int* p) {
+  int v;
+  asm volatile("ld.relaxed.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void fence_acq_rel_gpu() {
+  asm volatile("fence.acq_rel.gpu;" ::: "memory");
+}
+
+// Non-blocking check of a flag released by another CTA: relaxed load, and
+// one acquire fence only once the flag is seen (polling with acquire loads
+// would fence the SM's memory traffic on every poll).
+__device__ __forceinline__ bool poll_flag(const int* flag) {
+  if (ld_relaxed_gpu(flag) == 0) return false;
+  fence_acq_rel_gpu();
+  return true;
+}
+
+// Spins until *flag != 0; gives up after `limit_ns` or once `*abort` is set.
+__device__ __forceinline__ bool wait_flag_bounded(const int* flag,
+                                                  volatile int* abort,
+                                                  uint64_t limit_ns) {
+  if (poll_flag(flag)) return true;
+  const uint64_t t0 = global_timer_ns();
+  for (uint32_t it = 1;; ++it) {
+    __nanosleep(128);
+    if (poll_flag(flag)) return true;
+    if ((it & 15) == 0) {
+      if (*abort) return false;
+      if (global_timer_ns() - t0 > limit_ns) return false;
+    }
+  }
+}
+
+// Orders this thread's generic-proxy global accesses against async-proxy
+// (TMA) accesses: used between writing data that another CTA will read with
+// TMA and publishing it, and between observing such a flag and the TMA load.
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+// Barrier among `count` threads (multiple of 32) on hardware barrier `id`.
+__device__ __forceinline__ void named_barrier(int id, int count) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
 }  // namespace pct

@@ -74,6 +74,8 @@ def _load() -> ctypes.CDLL:
     lib.pctree_profile_collect.argtypes = [ctypes.POINTER(ctypes.c_int64),
                                            ctypes.POINTER(ctypes.c_double)]
     lib.pctree_profile_collect.restype = ctypes.c_int
+    lib.pctree_set_path.argtypes = [ctypes.c_int32]
+    lib.pctree_set_path.restype = ctypes.c_int
     lib.pctree_version.argtypes = []
     lib.pctree_version.restype = ctypes.c_int32
     return lib
@@ -215,6 +217,35 @@ def pctree_profile_collect():
     if rc != PCTREE_OK:
         raise PctreeError(rc, "pctree_profile_collect")
     return int(n.value), float(ms.value)
+
+
+PATH_AUTO, PATH_STAGEWISE = 0, 1
+
+
+def pctree_set_path(path: int) -> None:
+    """Select the kernel path (see pctree_set_path in include/pctree.h)."""
+    rc = LIB.pctree_set_path(path)
+    if rc != PCTREE_OK:
+        raise PctreeError(rc, "pctree_set_path")
+
+
+def uses_fused_round(cfg: Config, path: int = PATH_AUTO) -> bool:
+    """Whether a round of `cfg` runs as one fused launch (mirrors the
+    library's choice)."""
+    return (path == PATH_AUTO and cfg.weight_dtype == PCTREE_BF16 and
+            cfg.batch * cfg.k <= 16 and cfg.k <= 16)
+
+
+def kernels_per_round(cfg: Config, path: int = PATH_AUTO) -> int:
+    """Kernels of this library one pctree_draft launches."""
+    if uses_fused_round(cfg, path):
+        return 3                      # init, fused round, pack
+    launches = 2                      # init, pack
+    for d in range(cfg.B):
+        rows = cfg.batch * (1 if d == 0 else cfg.k)
+        passes = (rows + 255) // 256 if cfg.weight_dtype == PCTREE_BF16 else 1
+        launches += passes + 2        # projection, partials, merge
+    return launches
 
 
 def pctree_version() -> int:

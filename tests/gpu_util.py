@@ -27,15 +27,22 @@ def device_inputs(inp: RoundInputs, device="cuda"):
     return L, E, W, root
 
 
-def run_gpu(inp: RoundInputs, with_pool=True, accept=True) -> Dict[str, np.ndarray]:
+def run_gpu(inp: RoundInputs, with_pool=True, accept=True,
+            path: int = 0) -> Dict[str, np.ndarray]:
+    """One round through the C ABI; ``path`` 0 = automatic (fused round
+    kernel where it applies), 1 = per-stage kernels."""
     from paper_2608_02123_gb300 import pctree as P
     wl = inp.wl
     cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, inp.L.shape[0],
                         wl.pos_offset, wl.weight_dtype)
     L, E, W, root = device_inputs(inp)
     dr = P.Drafter(cfg, with_pool=with_pool)
-    tree = dr.draft(L, E, W, root)
-    torch.cuda.synchronize()
+    P.pctree_set_path(path)
+    try:
+        tree = dr.draft(L, E, W, root)
+        torch.cuda.synchronize()
+    finally:
+        P.pctree_set_path(P.PATH_AUTO)
     host = tree.to_host()
     if accept:
         target = target_for_tree(inp.greedy, host["depth"])

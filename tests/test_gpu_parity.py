@@ -43,12 +43,26 @@ SMALL = {
 }
 
 
+PATHS = {"auto": 0, "stagewise": 1}
+
+
+@pytest.mark.parametrize("path", sorted(PATHS))
 @pytest.mark.parametrize("name", sorted(SMALL))
-def test_small_parity(name):
+def test_small_parity(name, path):
     inp = draw_round(SMALL[name])
-    host = G.run_gpu(inp)
+    host = G.run_gpu(inp, path=PATHS[path])
     rep = G.compare(inp, host)
-    print(f"{name}: ambiguous={rep.ambiguous} max|dlogp|={rep.max_logp_err:.2e}")
+    print(f"{name}/{path}: ambiguous={rep.ambiguous} "
+          f"max|dlogp|={rep.max_logp_err:.2e}")
+
+
+def test_paths_agree_exactly_on_structure():
+    inp = draw_round(SMALL["weak_head_bf16"])
+    a = G.run_gpu(inp, path=0)
+    b = G.run_gpu(inp, path=1)
+    for name in ("tokens", "parent", "depth", "mask", "retrieve", "n_nodes"):
+        np.testing.assert_array_equal(a[name], b[name])
+    assert np.abs(a["logp"][:, :] - b["logp"][:, :])[np.isfinite(a["logp"])].max() <= 1e-4
 
 
 def test_second_call_reuses_workspace_cleanly():
@@ -74,37 +88,39 @@ def _tie_inputs(dtype):
                        np.zeros((1, 3), np.int32), np.zeros((1, 2), np.int32))
 
 
+@pytest.mark.parametrize("path", sorted(PATHS))
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
-def test_planted_ties_exact(dtype):
+def test_planted_ties_exact(dtype, path):
     """Exact ties everywhere: the tie-break rules alone decide, so the GPU
     must equal the oracle's own decisions with no replay."""
     inp = _tie_inputs(dtype)
-    host = G.run_gpu(inp)
+    host = G.run_gpu(inp, path=PATHS[path])
     G.compare(inp, host, strict=True)
     # root children: tokens 0, 1 (tie at 4, token order), then 2
     assert host["pool_token"][0][1:4].tolist() == [0, 1, 2]
 
 
-def test_neg_inf_logits():
+@pytest.mark.parametrize("path", sorted(PATHS))
+def test_neg_inf_logits(path):
     wl = strong(BASE, V=300, H=64, B=3, k=4, N=30, batch=1, seed=22)
     inp = draw_round(wl)
     inp.L[0, 0, :] = -np.inf
     inp.L[0, 0, [5, 77]] = [1.0, 0.5]        # two finite children only
     inp.L[0, 1, 100:] = -np.inf
-    host = G.run_gpu(inp)
+    host = G.run_gpu(inp, path=PATHS[path])
     G.compare(inp, host)
     assert np.isneginf(host["pool_logp"][0]).sum() > 0
 
 
-def test_nonfinite_and_bad_root_set_status():
-    from paper_2608_02123_gb300 import pctree as P
+@pytest.mark.parametrize("path", sorted(PATHS))
+def test_nonfinite_and_bad_root_set_status(path):
     inp = draw_round(SMALL["ragged_V_bf16"])
     inp.L[1, 2, 17] = np.nan
-    host = G.run_gpu(inp, accept=False)
+    host = G.run_gpu(inp, accept=False, path=PATHS[path])
     assert int(host["status"][0]) == -5       # PCTREE_ERR_NONFINITE
     inp = draw_round(SMALL["ragged_V_bf16"])
     inp.root[0] = inp.wl.V + 3
-    host = G.run_gpu(inp, accept=False)
+    host = G.run_gpu(inp, accept=False, path=PATHS[path])
     assert int(host["status"][0]) == -1       # PCTREE_ERR_INVALID_ARG
 
 
@@ -135,13 +151,14 @@ def _full(name, requests=None):
                       requests=reqs)
 
 
+@pytest.mark.parametrize("path", sorted(PATHS))
 @pytest.mark.parametrize("name", ["4b_b16", "4b_b16_chain", "4b_b7"])
-def test_full_size_batch1(name):
+def test_full_size_batch1(name, path):
     inp = _full(name)
-    host = G.run_gpu(inp)
+    host = G.run_gpu(inp, path=PATHS[path])
     rep = G.compare(inp, host)
-    print(f"{name}: ambiguous={rep.ambiguous} max|dlogp|={rep.max_logp_err:.2e} "
-          f"min margin={rep.min_margin:.2e}")
+    print(f"{name}/{path}: ambiguous={rep.ambiguous} "
+          f"max|dlogp|={rep.max_logp_err:.2e} min margin={rep.min_margin:.2e}")
 
 
 @pytest.mark.parametrize("name,n_check", [("8b_b7_bs16", 2), ("14b_b16_bs32", 1)])
