@@ -256,7 +256,6 @@ cudaError_t launch_markov_f32(const float* W_out, const float* X,
 cudaError_t launch_round_fused(const CUtensorMap* tmap_w,
                                const CUtensorMap* tmap_x, const FusedArgs& args,
                                int grid, cudaStream_t stream);
-size_t round_fused_smem_bytes();
 
 cudaError_t launch_init(const pctree_config& c, const Layout& lay,
                         const int32_t* root, const void* E_in,

@@ -5,19 +5,26 @@
 // Per stage d, every CTA (one per SM) streams its share of W_out tiles with
 // TMA and multiplies them on the tensor cores (tcgen05, bf16 -> f32 in TMEM)
 // against the stage's parent rows X = E_in[parent tokens] (Eq. 3), a 16-row
-// buffer in global memory loaded with one TMA box per ring slot.  The epilogue adds the shared base
-// logits L_d and keeps, per parent, a running log-sum-exp (Eq. 2) and a
-// warp-resident top-k list -- the stage logits never reach HBM.  When a CTA
-// has finished its tiles it publishes per-CTA partials; the last CTA to
-// arrive (atomic ticket, no waiting) merges them: per-parent normaliser and
-// top-k children, joint scores s(child) = s(p) + log pi (Eq. 4), the pool
-// push, the layer-wise frontier (Sec. 4.1) and the next stage's parent rows,
-// then releases a flag.  Producers keep prefetching the next stage's
-// W_out tiles while that merge runs and only hold back the parent-row loads
-// until the flag is set.
+// buffer in global memory loaded with one TMA box per ring slot.  The
+// epilogue adds the shared base logits L_d and keeps, per parent row, a
+// running log-sum-exp (Eq. 2) and a warp-resident top-k list -- the stage
+// logits never reach HBM.  When a CTA has finished its tiles it publishes
+// per-CTA partials; the last CTA to arrive (atomic ticket, no waiting) merges
+// them: per-row normaliser and top-k children, joint scores s(child) = s(p) +
+// log pi (Eq. 4), the pool push, the layer-wise frontier (Sec. 4.1) and the
+// next stage's parent rows, then releases a flag.  Producers keep
+// prefetching the next stage's W_out tiles while that merge runs and only
+// hold back the parent-row loads until the flag is set.
 //
-// Warp roles: warp 0 TMA producer, warp 1 TMEM allocator + MMA issuer,
-// warps 2..5 epilogue (TMEM lane quadrant = warp % 4) and merge.
+// Consecutive stages walk the vocabulary tiles in opposite directions, so a
+// stage begins with the tiles the previous stage read last; W_out is read
+// with an L2 evict_first policy, so those are the tiles most likely to still
+// sit in L2.
+//
+// Warp roles (320 threads): warp 0 TMA producer, warp 1 TMEM allocator + MMA
+// issuer, warps 2..9 epilogue in two groups of four, group h reading TMEM
+// accumulator buffer h (lane quadrant = warp % 4); the eight epilogue warps
+// also run the combine and the merge, one parent row per warp.
 #include <cuda_runtime.h>
 
 #include "pctree_common.cuh"
@@ -29,54 +36,77 @@ namespace {
 constexpr int kBM = 128;
 constexpr int kBK = 64;
 constexpr int kUmmaK = 16;
-constexpr int kBN = kFusedRows;                  // Markov rows per stage (max)
+constexpr int kBN = kFusedRows;                  // MMA N (Markov rows, max)
 constexpr int kMaxKF = kFusedMaxK;               // k limit of this path
-constexpr int kThreads = 192;
-constexpr int kEpiWarps = 4;
+constexpr int kEpiWarps = 8;
+constexpr int kEpiThreads = kEpiWarps * 32;
+constexpr int kThreads = 64 + kEpiThreads;
 constexpr int kABytes = kBM * kBK * 2;           // 16 KB of W_out per slot
 constexpr int kBBytes = kBN * kBK * 2;           // 2 KB of parent rows
 constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kStages = 8;
 constexpr int kTmemCols = 32;                    // two 16-column accumulators
+constexpr int kG = kFusedMaxGrid / 32;           // CTA groups of 32 in a merge
 constexpr uint64_t kLimitNs = 1000000000ull;     // 1 s per bounded wait
 constexpr float kNegInf = -INFINITY;
 
+template <int R>
 struct FusedSmem {
   uint64_t full[kStages], empty[kStages], acc_full[2], acc_empty[2], drain;
   uint32_t tmem_slot;
   int abort;
   int ticket;
-  float lv[kEpiWarps][kBN][kMaxKF];        // per-warp top-k lists per row
-  int lt[kEpiWarps][kBN][kMaxKF];
+  float lv[kEpiWarps][R][kMaxKF];          // per-warp top-k lists per row
+  int lt[kEpiWarps][R][kMaxKF];
   union {
     struct {                               // per-thread (max, sum-exp)
-      float m[kBN][kEpiWarps * 32];
-      float s[kBN][kEpiWarps * 32];
+      float m[R][kEpiThreads];
+      float s[R][kEpiThreads];
     } part;
-    struct {                               // merge: 32 CTAs' lists per warp
-      float z[kEpiWarps][kMaxKF][32];
-      int t[kEpiWarps][kMaxKF][32];
+    struct {                               // merge: first entries of 32 CTAs
+      float z[kEpiWarps][kG][32];
+      int t[kEpiWarps][kG][32];
     } stage;
   } u;
-  unsigned long long keys[kBN * kMaxKF];   // new layer: (score, id) keys
-  int ktok[kBN * kMaxKF];                  // new layer: tokens
-  int ftok[kBN];                           // next stage's parent tokens
+  unsigned long long keys[R * kMaxKF];     // new layer: (score, id) keys
+  int ktok[R * kMaxKF];                    // new layer: tokens
+  int ftok[R];                             // next stage's parent tokens
 };
 
-constexpr size_t kSmemBytes =
-    1024 + static_cast<size_t>(kStages) * kStageBytes + sizeof(FusedSmem);
+template <int R>
+constexpr size_t smem_bytes() {
+  return 1024 + static_cast<size_t>(kStages) * kStageBytes + sizeof(FusedSmem<R>);
+}
 
-__device__ __forceinline__ void epi_barrier() { named_barrier(1, kEpiWarps * 32); }
+__device__ __forceinline__ void epi_barrier() { named_barrier(1, kEpiThreads); }
+
+// i-th tile (0-based) of this CTA in stage d, and the kc-th K chunk of a
+// tile: even stages walk forward, odd stages backward, so each stage visits
+// (tile, chunk) in the exact reverse of the previous stage's order.
+__device__ __forceinline__ int tile_at(int d, int i, int n_my) {
+  const int j = (d & 1) ? n_my - 1 - i : i;
+  return blockIdx.x + j * gridDim.x;
+}
+
+__device__ __forceinline__ int chunk_at(int d, int kc, int n_k) {
+  return (d & 1) ? n_k - 1 - kc : kc;
+}
+
+__device__ __forceinline__ int my_tiles(int n_tiles) {
+  return (n_tiles - static_cast<int>(blockIdx.x) + gridDim.x - 1) / gridDim.x;
+}
 
 // --------------------------------------------------------------------------
 // producer: W_out tiles (A) and parent rows (B) into the shared-memory ring
 // --------------------------------------------------------------------------
 
+template <int R>
 __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
-                        const FusedArgs& a, unsigned char* ring, FusedSmem* S,
-                        volatile int* abort_v) {
-  const int grid = gridDim.x;
+                        const FusedArgs& a, unsigned char* ring,
+                        FusedSmem<R>* S, volatile int* abort_v) {
+  const int n_my = my_tiles(a.n_tiles);
   const uint64_t stream_policy = l2_policy_evict_first();
+  constexpr uint32_t tx = kABytes + kBBytes;
   int stage = 0;
   uint32_t phase = 0;
   int armed[kStages];
@@ -84,23 +114,22 @@ __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
   for (int s = 0; s < kStages; ++s) armed[s] = -1;
   int pend_stage[kStages], pend_kc[kStages];
   bool ok = true;
+  auto issue_rows = [&](int st, int kx) {
+    tma_load_2d(ring + st * kStageBytes + kABytes, tmap_x, &S->full[st],
+                kx * kBK, 0);
+  };
+
 
   for (int d = 0; d < a.B && ok; ++d) {
-    constexpr uint32_t tx = kABytes + kBBytes;
     bool have = d == 0;   // stage 0 rows were written before the launch
     int n_pend = 0;
-    auto acquire_rows = [&]() {
-      fence_proxy_async_global();   // rows written by another CTA's merge
-    };
-    auto issue_rows = [&](int st, int kc) {
-      tma_load_2d(ring + st * kStageBytes + kABytes, tmap_x, &S->full[st],
-                  kc * kBK, 0);
-    };
-    for (int tile = blockIdx.x; tile < a.n_tiles && ok; tile += grid) {
+    for (int i = 0; i < n_my && ok; ++i) {
+      const int tile = tile_at(d, i, n_my);
       for (int kc = 0; kc < a.n_k; ++kc) {
         if (!have) {
           bool rdy = poll_flag(&a.ready[d]);
           if (!rdy && n_pend == kStages) {
+            // ring full of slots waiting for the parent rows
             if (!wait_flag_bounded(&a.ready[d], abort_v, kLimitNs)) {
               ok = false;
               break;
@@ -108,7 +137,7 @@ __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
             rdy = true;
           }
           if (rdy) {
-            acquire_rows();
+            fence_proxy_async_global();   // rows written by another CTA
             have = true;
             for (int p = 0; p < n_pend; ++p) issue_rows(pend_stage[p], pend_kc[p]);
             n_pend = 0;
@@ -118,14 +147,15 @@ __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
           ok = false;
           break;
         }
+        const int kx = chunk_at(d, kc, a.n_k);
         mbar_arrive_expect_tx(&S->full[stage], tx);
         tma_load_2d_hint(ring + stage * kStageBytes, tmap_w, &S->full[stage],
-                         kc * kBK, tile * kBM, stream_policy);
+                         kx * kBK, tile * kBM, stream_policy);
         if (have) {
-          issue_rows(stage, kc);
+          issue_rows(stage, kx);
         } else {
           pend_stage[n_pend] = stage;
-          pend_kc[n_pend] = kc;
+          pend_kc[n_pend] = kx;
           ++n_pend;
         }
         armed[stage] = static_cast<int>(phase);
@@ -139,7 +169,7 @@ __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
       if (!wait_flag_bounded(&a.ready[d], abort_v, kLimitNs)) {
         ok = false;
       } else {
-        acquire_rows();
+        fence_proxy_async_global();
         for (int p = 0; p < n_pend; ++p) issue_rows(pend_stage[p], pend_kc[p]);
       }
     }
@@ -160,17 +190,18 @@ __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
 // MMA issuer
 // --------------------------------------------------------------------------
 
-__device__ void mma(const FusedArgs& a, unsigned char* ring, FusedSmem* S,
+template <int R>
+__device__ void mma(const FusedArgs& a, unsigned char* ring, FusedSmem<R>* S,
                     uint32_t tmem_base, volatile int* abort_v) {
   constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN);
-  const int grid = gridDim.x;
+  const int n_my = my_tiles(a.n_tiles);
   int stage = 0;
   uint32_t phase = 0;
   int acc = 0;
   uint32_t acc_phase = 0;
   bool ok = true;
   for (int d = 0; d < a.B && ok; ++d) {
-    for (int tile = blockIdx.x; tile < a.n_tiles && ok; tile += grid) {
+    for (int i = 0; i < n_my && ok; ++i) {
       if (!mbar_wait_bounded(&S->acc_empty[acc], acc_phase ^ 1u, abort_v, kLimitNs)) {
         ok = false;
         break;
@@ -213,13 +244,15 @@ __device__ void mma(const FusedArgs& a, unsigned char* ring, FusedSmem* S,
 }
 
 // --------------------------------------------------------------------------
-// merge of stage d by the last CTA (the four epilogue warps)
+// merge of stage d by the last CTA (the eight epilogue warps)
 // --------------------------------------------------------------------------
 
-__device__ void merge_stage(const FusedArgs& a, FusedSmem* S, int d) {
-  const int ew = (threadIdx.x >> 5) - 2;   // 0..3
+template <int R>
+__device__ void merge_stage(const CUtensorMap* tmap_w, const FusedArgs& a,
+                            FusedSmem<R>* S, int d) {
+  const int ew = (threadIdx.x >> 5) - 2;   // 0..7
   const int lane = threadIdx.x & 31;
-  const int tid = ew * 32 + lane;          // 0..127
+  const int tid = ew * 32 + lane;          // 0..255
   const int grid = gridDim.x;
   const int b_d = d == 0 ? 1 : a.k;
   const int rows = a.batch * b_d;
@@ -227,6 +260,7 @@ __device__ void merge_stage(const FusedArgs& a, FusedSmem* S, int d) {
   const int n_layer = b_d * k;
   const int base = level_base(d + 1, k);
   if (d > 0) (void)ld_acquire_gpu(&a.ready[d]);   // pool of earlier stages
+#pragma unroll 1
   for (int c = ew; c < rows; c += kEpiWarps) {
     // log-softmax normaliser of parent row c over all CTAs' partials (Eq. 2)
     const float lse = warp_lse_from_partials<8>(
@@ -240,7 +274,6 @@ __device__ void merge_stage(const FusedArgs& a, FusedSmem* S, int d) {
     // offered.  Loops stay rolled: this code runs once per stage.
     const float* cz = a.cand_z + static_cast<size_t>(c) * grid * k;
     const int32_t* ct = a.cand_t + static_cast<size_t>(c) * grid * k;
-    constexpr int kG = kFusedMaxGrid / 32;
     float(*sz)[32] = S->u.stage.z[ew];
     int(*st)[32] = S->u.stage.t[ew];
 #pragma unroll
@@ -299,8 +332,7 @@ __device__ void merge_stage(const FusedArgs& a, FusedSmem* S, int d) {
         t = 0;
         logpi = kNegInf;
       }
-      const float2 sp = sc[pid];
-      const float2 sn = ff_add(sp, logpi);   // Eq. 4
+      const float2 sn = ff_add(sc[pid], logpi);   // Eq. 4
       tok[id] = t;
       par[id] = pid;
       sc[id] = sn;
@@ -314,7 +346,7 @@ __device__ void merge_stage(const FusedArgs& a, FusedSmem* S, int d) {
   epi_barrier();
   // frontier of each request: the k best nodes of the new layer
   const int total = a.batch * n_layer;
-  for (int i = tid; i < total; i += kEpiWarps * 32) {
+  for (int i = tid; i < total; i += kEpiThreads) {
     const int req = i / n_layer;
     const unsigned long long key = S->keys[i];
     int rank = 0;
@@ -327,24 +359,24 @@ __device__ void merge_stage(const FusedArgs& a, FusedSmem* S, int d) {
   }
   epi_barrier();
   // parent rows of the next stage: X[req * k + slot] = E_in[token]
-  constexpr int kG8 = 10;
+  constexpr int kU = 10;
   const int per_row = a.H / 8;
   const int total_v = a.batch * k * per_row;
   const uint4* src = static_cast<const uint4*>(a.E_in);
   uint4* dst = static_cast<uint4*>(a.X);
-  for (int i0 = tid; i0 < total_v; i0 += kEpiWarps * 32 * kG8) {
-    uint4 tmp[kG8];
+  for (int i0 = tid; i0 < total_v; i0 += kEpiThreads * kU) {
+    uint4 tmp[kU];
 #pragma unroll
-    for (int u = 0; u < kG8; ++u) {
-      const int i = i0 + u * kEpiWarps * 32;
+    for (int u = 0; u < kU; ++u) {
+      const int i = i0 + u * kEpiThreads;
       if (i < total_v) {
         const int row = i / per_row, off = i - row * per_row;
         tmp[u] = src[static_cast<size_t>(S->ftok[row]) * per_row + off];
       }
     }
 #pragma unroll
-    for (int u = 0; u < kG8; ++u) {
-      const int i = i0 + u * kEpiWarps * 32;
+    for (int u = 0; u < kU; ++u) {
+      const int i = i0 + u * kEpiThreads;
       if (i < total_v) {
         const int row = i / per_row, off = i - row * per_row;
         dst[static_cast<size_t>(row) * per_row + off] = tmp[u];
@@ -361,70 +393,86 @@ __device__ void merge_stage(const FusedArgs& a, FusedSmem* S, int d) {
 // epilogue: TMEM -> registers, online log-sum-exp and top-k per parent row
 // --------------------------------------------------------------------------
 
-__device__ void epilogue(const FusedArgs& a, FusedSmem* S, uint32_t tmem_base,
+template <int R>
+__device__ __forceinline__ void load_acc(uint32_t taddr, float (&acc)[R]) {
+  if constexpr (R == 8) {
+    uint32_t r[8];
+    tmem_ld_32x32b_x8(taddr, r);
+    tmem_ld_wait();
+#pragma unroll
+    for (int c = 0; c < 8; ++c) acc[c] = __uint_as_float(r[c]);
+  } else {
+    uint32_t r[16];
+    tmem_ld_32x32b_x16(taddr, r);
+    tmem_ld_wait();
+#pragma unroll
+    for (int c = 0; c < 16; ++c) acc[c] = __uint_as_float(r[c]);
+  }
+}
+
+template <int R>
+__device__ void epilogue(const CUtensorMap* tmap_w, const FusedArgs& a,
+                         FusedSmem<R>* S, uint32_t tmem_base,
                          volatile int* abort_v) {
   const int warp = threadIdx.x >> 5;
-  const int ew = warp - 2;
-  const int quad = warp & 3;
+  const int ew = warp - 2;                 // 0..7
+  const int grp = ew >> 2;                 // accumulator buffer of this warp
+  const int quad = warp & 3;               // TMEM lanes 32*quad .. +31
   const int lane = threadIdx.x & 31;
+  const int tid = ew * 32 + lane;
   const int grid = gridDim.x;
   const int k = a.k;
-  int acc = 0;
+  const int n_my = my_tiles(a.n_tiles);
   uint32_t acc_phase = 0;
+  int g_tile = 0;                          // tiles issued by the MMA so far
   bool bad = false;
   for (int d = 0; d < a.B; ++d) {
     const int b_d = d == 0 ? 1 : k;
     const int rows = a.batch * b_d;
-    float m[kBN], s[kBN];
-    WarpList lst[kBN];
+    float m[R], s[R];
+    WarpList lst[R];
 #pragma unroll
-    for (int c = 0; c < kBN; ++c) {
+    for (int c = 0; c < R; ++c) {
       m[c] = kNegInf;
       s[c] = 0.0f;
       lst[c].reset();
     }
-    bool first = true;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < a.n_tiles; tile += grid) {
-      if (!mbar_wait_bounded(&S->acc_full[acc], acc_phase, abort_v, kLimitNs)) {
+    for (int i = 0; i < n_my; ++i, ++g_tile) {
+      if ((g_tile & 1) != grp) continue;
+      const int tile = tile_at(d, i, n_my);
+      if (!mbar_wait_bounded(&S->acc_full[grp], acc_phase, abort_v, kLimitNs)) {
         ok = false;
         break;
       }
+      acc_phase ^= 1u;
       tc_fence_after_sync();
-      uint32_t r[16];
-      tmem_ld_32x32b_x16(tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
-                             static_cast<uint32_t>(acc * kBN),
-                         r);
-      tmem_ld_wait();
+      float acc[R];
+      load_acc<R>(tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                      static_cast<uint32_t>(grp * kBN),
+                  acc);
       tc_fence_before_sync();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&S->acc_empty[acc]);
-      acc ^= 1;
-      if (acc == 0) acc_phase ^= 1u;
+      if (lane == 0) mbar_arrive(&S->acc_empty[grp]);
       const int v = tile * kBM + quad * 32 + lane;
       const bool inb = v < a.V;
       const float* Lrow = a.L + static_cast<size_t>(d) * a.V + (inb ? v : 0);
 #pragma unroll
-      for (int c = 0; c < kBN; ++c) {
+      for (int c = 0; c < R; ++c) {
         if (c < rows) {
           const int req = c / b_d;
           float z = kNegInf;
           int t = 0x7fffffff;
           if (inb) {
             const float lval = __ldg(Lrow + static_cast<size_t>(req) * a.B * a.V);
-            z = lval + __uint_as_float(r[c]);
+            z = lval + acc[c];
             t = v;
             bad |= isnan(z) || (isinf(z) && !(isinf(lval) && lval < 0.0f));
             lse_push(m[c], s[c], z);
           }
-          if (first) {
-            lst[c].seed(z, t, k);
-          } else {
-            lst[c].offer(z, t, k);
-          }
+          lst[c].offer(z, t, k);
         }
       }
-      first = false;
     }
     if (!ok) {
       *abort_v = 1;
@@ -432,9 +480,8 @@ __device__ void epilogue(const FusedArgs& a, FusedSmem* S, uint32_t tmem_base,
       break;
     }
     // per-thread (max, sum-exp) and per-warp lists to shared memory
-    const int tid = ew * 32 + lane;
 #pragma unroll
-    for (int c = 0; c < kBN; ++c) {
+    for (int c = 0; c < R; ++c) {
       if (c < rows) {
         S->u.part.m[c][tid] = m[c];
         S->u.part.s[c][tid] = s[c];
@@ -445,8 +492,7 @@ __device__ void epilogue(const FusedArgs& a, FusedSmem* S, uint32_t tmem_base,
       }
     }
     epi_barrier();
-    // per-CTA partials of the rows this warp owns (rolled: runs once per
-    // stage from a cold instruction cache)
+    // per-CTA partials, one row per warp (rolled: runs once per stage)
 #pragma unroll 1
     for (int c = ew; c < rows; c += kEpiWarps) {
       float mm = kNegInf, ss = 0.0f;
@@ -478,17 +524,18 @@ __device__ void epilogue(const FusedArgs& a, FusedSmem* S, uint32_t tmem_base,
     }
     __threadfence();
     epi_barrier();
-    if (ew == 0 && lane == 0) S->ticket = atomicAdd(&a.stage_cnt[d], 1);
+    if (tid == 0) S->ticket = atomicAdd(&a.stage_cnt[d], 1);
     epi_barrier();
     if (S->ticket == grid - 1) {
       __threadfence();
-      merge_stage(a, S, d);
+      merge_stage<R>(tmap_w, a, S, d);
     }
     epi_barrier();
   }
   if (bad) set_status(a.status, PCTREE_ERR_NONFINITE);
 }
 
+template <int R>
 __global__ void __launch_bounds__(kThreads, 1)
 round_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
                    const __grid_constant__ CUtensorMap tmap_x,
@@ -496,7 +543,7 @@ round_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
   extern __shared__ unsigned char smem_raw[];
   unsigned char* ring = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  FusedSmem* S = reinterpret_cast<FusedSmem*>(ring + kStages * kStageBytes);
+  FusedSmem<R>* S = reinterpret_cast<FusedSmem<R>*>(ring + kStages * kStageBytes);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -506,7 +553,7 @@ round_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&S->acc_full[i], 1);
-      mbar_init(&S->acc_empty[i], kEpiWarps);
+      mbar_init(&S->acc_empty[i], 4);   // the four warps of group i
     }
     mbar_init(&S->drain, 1);
     S->abort = 0;
@@ -521,11 +568,11 @@ round_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
   const uint32_t tmem_base = S->tmem_slot;
   volatile int* abort_v = &S->abort;
   if (warp == 0) {
-    if (lane == 0) produce(&tmap_w, &tmap_x, a, ring, S, abort_v);
+    if (lane == 0) produce<R>(&tmap_w, &tmap_x, a, ring, S, abort_v);
   } else if (warp == 1) {
-    if (lane == 0) mma(a, ring, S, tmem_base, abort_v);
+    if (lane == 0) mma<R>(a, ring, S, tmem_base, abort_v);
   } else {
-    epilogue(a, S, tmem_base, abort_v);
+    epilogue<R>(&tmap_w, a, S, tmem_base, abort_v);
   }
   tc_fence_before_sync();
   __syncthreads();
@@ -533,27 +580,32 @@ round_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
   if (warp == 1) tmem_dealloc(tmem_base, kTmemCols);
 }
 
-}  // namespace
-
-size_t round_fused_smem_bytes() { return kSmemBytes; }
-
-cudaError_t launch_round_fused(const CUtensorMap* tmap_w,
-                               const CUtensorMap* tmap_x, const FusedArgs& args,
-                               int grid, cudaStream_t stream) {
+template <int R>
+cudaError_t launch_r(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
+                     const FusedArgs& args, int grid, cudaStream_t stream) {
   static bool attr_done = false;
   if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(round_fused_kernel,
+    cudaError_t e = cudaFuncSetAttribute(round_fused_kernel<R>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(kSmemBytes));
+                                         static_cast<int>(smem_bytes<R>()));
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
   CUtensorMap w = *tmap_w, x = *tmap_x;
   FusedArgs a = args;
   void* params[] = {&w, &x, &a};
-  return cudaLaunchCooperativeKernel(reinterpret_cast<void*>(round_fused_kernel),
+  return cudaLaunchCooperativeKernel(reinterpret_cast<void*>(round_fused_kernel<R>),
                                      dim3(grid), dim3(kThreads), params,
-                                     kSmemBytes, stream);
+                                     smem_bytes<R>(), stream);
+}
+
+}  // namespace
+
+cudaError_t launch_round_fused(const CUtensorMap* tmap_w,
+                               const CUtensorMap* tmap_x, const FusedArgs& args,
+                               int grid, cudaStream_t stream) {
+  if (args.batch * args.k <= 8) return launch_r<8>(tmap_w, tmap_x, args, grid, stream);
+  return launch_r<16>(tmap_w, tmap_x, args, grid, stream);
 }
 
 }  // namespace pct
