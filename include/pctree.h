@@ -174,6 +174,34 @@ PCTREE_API pctree_status pctree_draft(const pctree_config* cfg, const float* bas
                            void* stream);
 
 /*
+ * The same drafting round as pctree_draft, without a caller-provided
+ * workspace.  The paper has no counterpart: this is a library convenience.
+ * It serves callers that cannot allocate device memory when they draft -- a
+ * host framework that owns a fixed memory budget and forbids side
+ * allocations, a plug-in that only receives the buffers its host hands it, a
+ * latency-critical serving loop where cudaMalloc / cudaFree would
+ * synchronise the device.  Inputs and outputs are as for pctree_draft.
+ * Scratch: a fixed 16 MiB array inside the library, reserved on every GPU
+ * that loads it until the process exits; a round whose
+ * pctree_workspace_bytes exceeds 16 MiB returns PCTREE_ERR_WORKSPACE before
+ * any work (batch-1 Qwen3-shaped rounds need about 5 MB).  The first call on
+ * a device, with that device current, looks up the array's address; make
+ * that first call before any stream capture begins.  Every call on a device
+ * shares the array, which keeps the previous call's contents (the round
+ * clears what must start at zero); calls whose GPU work overlaps -- other
+ * streams, other host threads -- race on it and must not be issued.  The
+ * call allocates nothing: no cudaMalloc, cudaFree or allocating library
+ * routine.
+ */
+PCTREE_API pctree_status pctree_draft_noalloc(const pctree_config* cfg,
+                                              const float* base_logits,
+                                              const void* head_emb,
+                                              const void* head_out,
+                                              const int32_t* root_token,
+                                              const pctree_tree* out,
+                                              void* stream);
+
+/*
  * Greedy tree acceptance (Sec. 4.2 "standard greedy tree rule"; Appendix A).
  * Starting at the root, repeatedly accept the child whose token equals the
  * target model's token at the current node, until no child matches.

@@ -64,6 +64,9 @@ def _load() -> ctypes.CDLL:
     lib.pctree_draft.argtypes = [cfgp, vp, vp, vp, vp, ctypes.POINTER(_Tree),
                                  vp, ctypes.c_size_t, vp]
     lib.pctree_draft.restype = ctypes.c_int
+    lib.pctree_draft_noalloc.argtypes = [cfgp, vp, vp, vp, vp,
+                                         ctypes.POINTER(_Tree), vp]
+    lib.pctree_draft_noalloc.restype = ctypes.c_int
     lib.pctree_accept.argtypes = [cfgp, ctypes.POINTER(_Tree), vp, vp, vp, vp,
                                   vp]
     lib.pctree_accept.restype = ctypes.c_int
@@ -187,6 +190,27 @@ def pctree_draft(cfg: Config, base_logits: torch.Tensor, head_emb: torch.Tensor,
                           _stream_ptr(stream))
     if rc != PCTREE_OK:
         raise PctreeError(rc, "pctree_draft")
+
+
+def pctree_draft_noalloc(cfg: Config, base_logits: torch.Tensor,
+                         head_emb: torch.Tensor, head_out: torch.Tensor,
+                         root_token: torch.Tensor, tree: Tree,
+                         stream: Optional[torch.cuda.Stream] = None) -> None:
+    """Enqueue one drafting round without a workspace: the library's fixed
+    16 MiB device array serves as scratch, for callers that cannot allocate
+    device memory when they draft (see pctree_draft_noalloc in
+    include/pctree.h)."""
+    for name, t in (("base_logits", base_logits), ("head_emb", head_emb),
+                    ("head_out", head_out), ("root_token", root_token)):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous CUDA tensor")
+    ts = tree.c_struct()
+    rc = LIB.pctree_draft_noalloc(ctypes.byref(cfg), base_logits.data_ptr(),
+                                  head_emb.data_ptr(), head_out.data_ptr(),
+                                  root_token.data_ptr(), ctypes.byref(ts),
+                                  _stream_ptr(stream))
+    if rc != PCTREE_OK:
+        raise PctreeError(rc, "pctree_draft_noalloc")
 
 
 def pctree_accept(cfg: Config, tree: Tree, target_tokens: torch.Tensor,
