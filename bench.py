@@ -34,7 +34,8 @@ from workloads import WORKLOADS, draw_head, draw_request  # noqa: E402
 
 METRIC = ("tree-draft rounds/sec & µs/round (V=151936, B=16, N=64); "
           "% of HBM roofline")
-N_SETS = 16          # rotating request inputs
+N_SETS = 16          # rotating input sets (at most)
+L2_BYTES = 129 * 1024 * 1024
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -46,6 +47,9 @@ def parse_args():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="4b_b16", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--path", default="auto", choices=["auto", "stagewise"],
+                    help="kernel path: fused round where it applies, or the "
+                         "per-stage kernels for every round")
     return ap.parse_args()
 
 
@@ -55,6 +59,38 @@ def measured_peaks():
         with open(path) as f:
             return json.load(f), "measured"
     return {"hbm_gbs": FALLBACK_HBM_GBS}, "fallback"
+
+
+FUSED_SOURCES = ("paper_2608_02123_gb300/csrc/round_fused.cu",
+                 "paper_2608_02123_gb300/csrc/sm103_ptx.cuh",
+                 "paper_2608_02123_gb300/csrc/pctree_common.cuh")
+
+
+def recorded_traffic(wl, fused):
+    """DRAM bytes per launch from the committed ncu summary of this kernel
+    and workload, or None when the kernel changed since the capture."""
+    if not fused:
+        return None
+    import hashlib
+    h = hashlib.sha256()
+    for f in FUSED_SOURCES:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    path = os.path.join(ROOT, "profiles",
+                        f"round_fused_kernel_qwen3_4b_V{wl.V}_H{wl.H}_B{wl.B}"
+                        f"_k{wl.k}_N{wl.N}.md")
+    if not os.path.exists(path):
+        return None
+    fields = {}
+    with open(path) as fh:
+        for line in fh:
+            if ":" in line and line.strip().split(":")[0] in (
+                    "traffic_bytes_per_launch", "kernel_sources_sha256_16"):
+                key, val = line.strip().split(":", 1)
+                fields[key] = val.strip()
+    if fields.get("kernel_sources_sha256_16") != h.hexdigest()[:16]:
+        return None
+    return int(fields["traffic_bytes_per_launch"])
 
 
 def stage_bytes(wl, d):
@@ -222,30 +258,45 @@ def run_ours(args, wl, rank, world, local_rank):
 
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
-    E_bits, W_bits = draw_head(wl)
-    E = torch.from_numpy(E_bits.view(np.int16)).to(dev).view(torch.bfloat16)
-    W = torch.from_numpy(W_bits.view(np.int16)).to(dev).view(torch.bfloat16)
+    E_host, W_host = draw_head(wl)
+    if wl.weight_dtype == "bf16":
+        E = torch.from_numpy(E_host.view(np.int16)).to(dev).view(torch.bfloat16)
+        W = torch.from_numpy(W_host.view(np.int16)).to(dev).view(torch.bfloat16)
+    else:
+        E = torch.from_numpy(E_host).to(dev)
+        W = torch.from_numpy(W_host).to(dev)
+    # rotating input sets, each a whole batch of distinct requests; enough
+    # sets that their base logits exceed the L2 three times over
+    batch_bytes = wl.batch * wl.B * wl.V * 4
+    n_sets = max(2, min(N_SETS, -(-3 * L2_BYTES // batch_bytes)))
+    per_rank = n_sets * wl.batch
+    many = wl.with_(batch=per_rank * world)
     sets = []
-    for i in range(N_SETS):
-        r = rank * N_SETS + i
-        L, root, greedy, _ = draw_request(wl.with_(batch=N_SETS * world), r)
-        sets.append((L, root, greedy))
-    L_dev = [torch.from_numpy(L[None]).to(dev) for L, _, _ in sets]
-    root_dev = [torch.tensor([root], dtype=torch.int32, device=dev)
-                for _, root, _ in sets]
-    greedy_dev = [torch.from_numpy(g[None].astype(np.int64)).to(dev)
+    for i in range(n_sets):
+        reqs = [draw_request(many, rank * per_rank + i * wl.batch + b)
+                for b in range(wl.batch)]
+        sets.append((np.stack([q[0] for q in reqs]),
+                     np.asarray([q[1] for q in reqs], np.int32),
+                     np.stack([q[2] for q in reqs])))
+    L_dev = [torch.from_numpy(L).to(dev) for L, _, _ in sets]
+    root_dev = [torch.from_numpy(root).to(dev) for _, root, _ in sets]
+    greedy_dev = [torch.from_numpy(g.astype(np.int64)).to(dev)
                   for _, _, g in sets]
-    cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, wl.batch)
+    cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, wl.batch, wl.pos_offset,
+                        wl.weight_dtype)
+    path = P.PATH_AUTO if args.path == "auto" else P.PATH_STAGEWISE
+    P.pctree_set_path(path)
+    fused = P.uses_fused_round(cfg, path)
     dr = P.Drafter(cfg, dev)
     stream = torch.cuda.current_stream()
 
     def target_of(i):
         # synthetic target model: node i at depth t wants g[t] as its child
         depth = dr.tree.depth.long().clamp_min(0)
-        return torch.gather(greedy_dev[i % N_SETS], 1, depth).to(torch.int32)
+        return torch.gather(greedy_dev[i % n_sets], 1, depth).to(torch.int32)
 
     def step(i):
-        dr.draft(L_dev[i % N_SETS], E, W, root_dev[i % N_SETS], stream)
+        dr.draft(L_dev[i % n_sets], E, W, root_dev[i % n_sets], stream)
         dr.accept(target_of(i), stream)
 
     for i in range(args.warmup):
@@ -275,9 +326,8 @@ def run_ours(args, wl, rank, world, local_rank):
     ms = start.elapsed_time(end)
 
     # end to end through the public API: pinned host inputs in, tree out
-    L_host = [torch.from_numpy(L[None]).pin_memory() for L, _, _ in sets]
-    root_host = [torch.tensor([root], dtype=torch.int32).pin_memory()
-                 for _, root, _ in sets]
+    L_host = [torch.from_numpy(L).pin_memory() for L, _, _ in sets]
+    root_host = [torch.from_numpy(root).pin_memory() for _, root, _ in sets]
     out_names = ("n_nodes", "tokens", "parent", "depth", "logp",
                  "position_ids", "mask", "retrieve", "n_leaves", "status")
     out_host = {n: torch.empty_like(getattr(dr.tree, n), device="cpu").pin_memory()
@@ -291,8 +341,8 @@ def run_ours(args, wl, rank, world, local_rank):
     root_stage = torch.empty_like(root_dev[0])
 
     def e2e_step(i):
-        L_stage.copy_(L_host[i % N_SETS], non_blocking=True)
-        root_stage.copy_(root_host[i % N_SETS], non_blocking=True)
+        L_stage.copy_(L_host[i % n_sets], non_blocking=True)
+        root_stage.copy_(root_host[i % n_sets], non_blocking=True)
         dr.draft(L_stage, E, W, root_stage, stream)
         dr.accept(target_of(i), stream)
         for n in out_names:
@@ -328,7 +378,7 @@ def run_ours(args, wl, rank, world, local_rank):
     proj_bytes = args.steps * bytes_round          # timed launches' bytes
     achieved = proj_bytes / (proj_ms / 1e3) / 1e9 if proj_ms > 0 else None
     us_round = ms * 1e3 / args.steps
-    kernels_per_step = P.kernels_per_round(cfg) + 1    # + accept
+    kernels_per_step = P.kernels_per_round(cfg, path) + 1    # + accept
     line = {
         "metric": METRIC, "value": value, "unit": "rounds/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
@@ -338,28 +388,30 @@ def run_ours(args, wl, rank, world, local_rank):
         "config": {"workload": wl.name, "V": wl.V, "H": wl.H, "B": wl.B,
                    "k": wl.k, "N": wl.N, "batch": wl.batch,
                    "parallelism": f"replicas x{world}",
-                   "l2": "inputs larger than L2: W_out (778 MB) streamed per "
-                         "stage; base logits rotate over 16 request sets"},
+                   "kernel_path": args.path,
+                   "l2": f"inputs larger than L2: W_out "
+                         f"({wl.V * wl.H * (2 if wl.weight_dtype == 'bf16' else 4) / 1e6:.0f} MB) "
+                         f"streamed per stage; base logits rotate over "
+                         f"{n_sets} input sets"},
         "us_per_round": us_round,
         "round_hbm_fraction": (bytes_round / (us_round * 1e-6) / 1e9) / peak,
         "roofline": {"bound": "hbm",
-                     "kernel": ("round_fused_kernel" if P.uses_fused_round(cfg)
+                     "kernel": ("round_fused_kernel" if fused
                                 else "markov_tc_kernel"),
                      "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak if achieved else None,
                      "peak_source": peak_kind,
                      "launches": launches,
                      "avg_launch_us": proj_ms * 1e3 / launches if launches else None,
-                     "traffic": None},
+                     "traffic": recorded_traffic(wl, fused)},
         "e2e": {"value": rounds / (e2e_ms / 1e3), "unit": "rounds/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": kernels_per_step * args.steps,
         "clocks": clk,
     }
     if world == 1 and not args.no_cpu_baseline:
-        E_bits_host, W_bits_host = E_bits, W_bits
-        runner = OracleRunner(wl, E_bits_host, W_bits_host,
-                              [(L, root) for L, root, _ in sets[:4]])
+        runner = OracleRunner(wl, E_host, W_host,
+                              [(L[0], int(root[0])) for L, root, _ in sets[:4]])
         line["cpu_baseline"] = cpu_baseline(runner, wl)
     print(json.dumps(line), flush=True)
 
