@@ -1,7 +1,8 @@
 """PCTree drafting-round oracle.  TEST INFRASTRUCTURE ONLY.
 
 A plain, slow, float64 restatement of one PCTree drafting round, written from
-the paper: the parent-conditioned Markov expansion (Sec. 4.1, Eqs. 2-4), the
+the paper: the parent-conditioned Markov expansion (Sec. 4.1, Eqs. 2-4) and
+the Shared-Markov control of the mechanism study (Sec. 5.3), the
 layer-wise frontier pruning and global budgeted selection (Sec. 4.1-4.2,
 Algorithm 1), the tree tensors (Sec. 4.2; Appendix A "Tensor implementation")
 and the greedy tree acceptance (Sec. 4.2; Appendix A).
@@ -309,10 +310,20 @@ def _check_stage(Z: np.ndarray, L_d: np.ndarray) -> None:
         raise NonFiniteInput("non-finite Markov bias")
 
 
+MODES = ("parent", "shared")
+
+
 def draft(L: np.ndarray, E_in: np.ndarray, W_out: np.ndarray, root: int,
           B: int, k: int, N: int, pos_offset: int = 0,
-          hint: Optional[Choices] = None, delta: float = DELTA) -> Round:
-    """One PCTree drafting round for one request.
+          hint: Optional[Choices] = None, delta: float = DELTA,
+          mode: str = "parent") -> Round:
+    """One drafting round for one request.
+
+    ``mode="parent"``: PCTree -- every frontier parent gets its own Markov
+    bias (Eqs. 2-3).  ``mode="shared"``: the Shared-Markov tree of the
+    mechanism study (Sec. 5.3): the greedy DSpark chain of Eq. 1 is built
+    alongside, and its distribution q_d at depth d serves every parent at
+    that depth; frontier, budget, selection and packing are unchanged.
 
     ``L`` is ``[B][V]`` (float32 or float64); ``E_in``/``W_out`` are ``[V][H]``
     as floats or bf16 bits (uint16; pass ``W_out`` pre-decoded with
@@ -322,20 +333,27 @@ def draft(L: np.ndarray, E_in: np.ndarray, W_out: np.ndarray, root: int,
     V = L.shape[1]
     if not (1 <= k <= V and N >= 1 and B >= 1 and 0 <= root < V):
         raise ValueError("invalid round parameters")
+    if mode not in MODES:
+        raise ValueError(mode)
     _check_logits(np.asarray(L, dtype=np.float64))
     pool = Pool([root], [-1], [0], [0.0], [()])       # root: score 0, id 0
     frontier = [0]
+    chain = root                                      # greedy chain (shared)
     margins = {"children": math.inf, "frontier": math.inf, "global": math.inf}
     n_amb = 0
     calls = []
     for d in range(B):                                # stage d builds level d+1
-        parents = [pool.token[i] for i in frontier]
+        if mode == "shared":
+            parents = [chain]                         # one batch-1 call, Eq. 1
+        else:
+            parents = [pool.token[i] for i in frontier]
         calls.append(len(parents))
         Z = stage_logits(L[d], E_in, W_out, parents)  # one batched call, Eq. 3
         _check_stage(Z, L[d])
         layer: List[int] = []
+        first_kids: List[int] = []
         for slot, pid in enumerate(frontier):
-            z = Z[slot]
+            z = Z[0 if mode == "shared" else slot]
             logpi, _ = log_softmax(z)                 # Eq. 2
             mine = local_topk(z, k)
             zs = np.sort(z)[::-1]
@@ -358,6 +376,8 @@ def draft(L: np.ndarray, E_in: np.ndarray, W_out: np.ndarray, root: int,
                                   cands, zval, delta, ordered=True)
                     n_amb += 1
                     kids = list(theirs)
+            if slot == 0:
+                first_kids = list(kids)
             for v in kids:                            # Eq. 4, pushed to pool
                 pool.token.append(v)
                 pool.parent.append(pid)
@@ -365,6 +385,8 @@ def draft(L: np.ndarray, E_in: np.ndarray, W_out: np.ndarray, root: int,
                 pool.s.append(pool.s[pid] + float(logpi[v]))
                 pool.path.append(pool.path[pid] + (v,))
                 layer.append(len(pool.token) - 1)
+        if mode == "shared":
+            chain = first_kids[0]                     # argmax of q_d (Eq. 1)
         if d < B - 1:
             mine = layer_frontier(layer, pool.s, k)
             ranked = sorted((pool.s[i] for i in layer), reverse=True)
@@ -496,7 +518,7 @@ def accept(tree: Tree, target: np.ndarray, B: int) -> Tuple[np.ndarray, int, int
 def draft_batch(L: np.ndarray, E_in: np.ndarray, W_out: np.ndarray,
                 roots: Sequence[int], B: int, k: int, N: int,
                 pos_offset: int = 0, hints: Optional[Sequence[Choices]] = None,
-                delta: float = DELTA) -> List[Round]:
+                delta: float = DELTA, mode: str = "parent") -> List[Round]:
     return [draft(L[r], E_in, W_out, int(roots[r]), B, k, N, pos_offset,
-                  None if hints is None else hints[r], delta)
+                  None if hints is None else hints[r], delta, mode)
             for r in range(L.shape[0])]

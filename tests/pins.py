@@ -174,7 +174,8 @@ def greedy_chain(L, E_in, W_out, root: int, B: int) -> List[int]:
     return out
 
 
-def check_chain(seed: int, V: int = 40, H: int = 5, B: int = 6) -> None:
+def check_chain(seed: int, V: int = 40, H: int = 5, B: int = 6,
+                mode: str = "parent") -> None:
     rng = np.random.default_rng(seed)
     L = rng.normal(size=(B, V)) * 2.0
     E_in = rng.normal(size=(V, H))
@@ -182,7 +183,7 @@ def check_chain(seed: int, V: int = 40, H: int = 5, B: int = 6) -> None:
     root = int(rng.integers(V))
     chain = greedy_chain(L, E_in, W_out, root, B)
     for N in (B + 1, B, 3, 1):
-        rnd = O.draft(L, E_in, W_out, root, B, k=1, N=N)
+        rnd = O.draft(L, E_in, W_out, root, B, k=1, N=N, mode=mode)
         n = min(N, B + 1)
         assert rnd.tree.n_nodes == n
         assert rnd.tree.tokens[:n].tolist() == [root] + chain[:n - 1]
@@ -356,3 +357,79 @@ def check_accept(seed: int) -> None:
         acc, length, bonus = O.accept(t, target, B)
         walk, wb = walk_accept(t, target)
         assert acc[:length + 1].tolist() == walk and bonus == wb
+
+
+# ----------------------------------------------------------------------------
+# Shared-Markov control (Sec. 5.3): one distribution per depth for all parents
+# ----------------------------------------------------------------------------
+
+def check_shared_bruteforce(seed: int, V: int, B: int, N: int, k: int) -> bool:
+    """Shared mode: every node at depth d+1 takes q_d, the distribution of
+    the greedy chain's depth-d step (Eq. 1).  With pruning unable to bind,
+    the kept set is the N most probable nodes of the full tree under those
+    shared distributions, computed exactly."""
+    assert N - 1 <= k <= V
+    L, E_in, W_out, root, cond = bigram_case(seed, V, B)
+    chain, prev = [], root
+    for d in range(B):
+        row = cond[d][prev]
+        best = max(range(V), key=lambda v: (row[v], -v))
+        if sorted(row, reverse=True)[0] == sorted(row, reverse=True)[1]:
+            return False                    # exact tie in the chain argmax
+        chain.append(row)
+        prev = best
+    probs = {(): Fraction(1)}
+    for depth in range(1, B + 1):
+        for path in product(range(V), repeat=depth):
+            probs[path] = probs[path[:-1]] * chain[depth - 1][path[-1]]
+    ranked = sorted(probs.items(), key=lambda kv: (-kv[1], len(kv[0])))
+    vals = [p for _, p in ranked[:N + 1]]
+    if len(set(vals)) != len(vals):
+        return False
+    if N < len(ranked) and (vals[N - 1] - vals[N]) / vals[N - 1] < 1e-9:
+        return False
+    want = {path for path, _ in ranked[:N]}
+    rnd = O.draft(L, E_in, W_out, root, B, k, N, mode="shared")
+    got = {rnd.pool.path[i] for i in rnd.selected}
+    assert got == want, f"kept {sorted(got)} != most probable {sorted(want)}"
+    for i, path in enumerate(rnd.pool.path):
+        assert abs(rnd.pool.s[i] - math.log(probs[path])) < 1e-12
+    assert rnd.markov_calls == [1] * B
+    return True
+
+
+def check_shared_equals_parent_without_bias(seed: int) -> None:
+    """With W_out = 0 the head adds nothing, so parent-conditioned and shared
+    scoring are the same distribution and must build the same tree."""
+    rng = np.random.default_rng(seed)
+    V, H, B, k, N = 40, 4, 5, 3, 12
+    L = rng.normal(size=(B, V)) * 2
+    E_in, W_out = rng.normal(size=(V, H)), np.zeros((V, H))
+    root = int(rng.integers(V))
+    a = O.draft(L, E_in, W_out, root, B, k, N, mode="parent")
+    b = O.draft(L, E_in, W_out, root, B, k, N, mode="shared")
+    assert a.pool.path == b.pool.path and a.pool.s == b.pool.s
+    assert (a.tree.tokens == b.tree.tokens).all()
+
+
+def check_shared_children_identical(seed: int) -> None:
+    """Every parent of a layer gets the same ranked children with the same
+    log-probabilities; the depth-1 layer equals parent mode's."""
+    rnd, _ = random_round(seed)
+    rng = np.random.default_rng(seed)
+    V, H, B, k, N = 60, 6, 5, 3, 12
+    L = rng.normal(size=(B, V)) * 3.0
+    E_in = rng.normal(size=(V, H))
+    W_out = rng.normal(size=(V, H)) * 0.8
+    root = int(rng.integers(V))
+    sh = O.draft(L, E_in, W_out, root, B, k, N, mode="shared")
+    pa = O.draft(L, E_in, W_out, root, B, k, N, mode="parent")
+    assert sh.pool.token[1:1 + k] == pa.pool.token[1:1 + k]
+    by_parent = {}
+    for i in range(1, len(sh.pool.token)):
+        p = sh.pool.parent[i]
+        by_parent.setdefault(p, []).append(
+            (sh.pool.token[i], sh.pool.s[i] - sh.pool.s[p]))
+    for depth in range(1, B):
+        lists = [v for p, v in by_parent.items() if sh.pool.depth[p] == depth]
+        assert all(lst == lists[0] for lst in lists), depth

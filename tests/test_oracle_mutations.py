@@ -108,3 +108,16 @@ def test_mask_without_self_is_caught(monkeypatch):
         return order, t
     monkeypatch.setattr(O, "pack", wrong)
     assert _fails(lambda: pins.check_structure(0))
+
+
+def test_shared_mode_conditioned_per_parent_is_caught(monkeypatch):
+    real = O.draft
+
+    def wrong(*args, **kw):                 # shared mode silently ignored
+        if kw.get("mode") == "shared":
+            kw["mode"] = "parent"
+        return real(*args, **kw)
+    monkeypatch.setattr(O, "draft", wrong)
+    assert _fails(lambda: [pins.check_shared_bruteforce(s, 5, 3, 5, 4)
+                           for s in range(6)],
+                  lambda: pins.check_shared_children_identical(0))

@@ -163,3 +163,27 @@ def test_golden_tiny_round_regression():
     target = target_for_tree(inp.greedy, t.depth[None, :])[0]
     acc, length, bonus = O.accept(t, target, wl.B)
     assert [acc.tolist(), length, bonus] == gold["accept"]
+
+
+# --- Shared-Markov control (Sec. 5.3) --------------------------------------
+
+@pytest.mark.parametrize("V,B,N,k", [(5, 3, 5, 4), (8, 3, 8, 7), (4, 4, 4, 3)])
+def test_shared_bruteforce_topN(V, B, N, k):
+    done = sum(pins.check_shared_bruteforce(seed, V, B, N, k)
+               for seed in range(12))
+    assert done >= 8
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_shared_equals_parent_without_bias(seed):
+    pins.check_shared_equals_parent_without_bias(seed)
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_shared_children_identical(seed):
+    pins.check_shared_children_identical(seed)
+
+
+@pytest.mark.parametrize("seed", range(2))
+def test_shared_k1_is_greedy_chain(seed):
+    pins.check_chain(seed, mode="shared")
