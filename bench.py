@@ -47,6 +47,8 @@ def parse_args():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="4b_b16", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--mode", default="parent", choices=["parent", "shared"],
+                    help="child scoring: PCTree, or the Shared-Markov control")
     ap.add_argument("--path", default="auto", choices=["auto", "stagewise"],
                     help="kernel path: fused round where it applies, or the "
                          "per-stage kernels for every round")
@@ -190,7 +192,7 @@ class OracleRunner:
     def run(self, i, stages):
         L, root = self.sets[i % len(self.sets)]
         self.O.draft(L[:stages], self.E_in, self.W, root, stages, self.wl.k,
-                     self.wl.N)
+                     self.wl.N, mode=self.wl.mode)
 
 
 def cpu_baseline(runner, wl, budget_s=12.0):
@@ -283,7 +285,7 @@ def run_ours(args, wl, rank, world, local_rank):
     greedy_dev = [torch.from_numpy(g.astype(np.int64)).to(dev)
                   for _, _, g in sets]
     cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, wl.batch, wl.pos_offset,
-                        wl.weight_dtype)
+                        wl.weight_dtype, wl.mode)
     path = P.PATH_AUTO if args.path == "auto" else P.PATH_STAGEWISE
     P.pctree_set_path(path)
     fused = P.uses_fused_round(cfg, path)
@@ -388,7 +390,7 @@ def run_ours(args, wl, rank, world, local_rank):
         "config": {"workload": wl.name, "V": wl.V, "H": wl.H, "B": wl.B,
                    "k": wl.k, "N": wl.N, "batch": wl.batch,
                    "parallelism": f"replicas x{world}",
-                   "kernel_path": args.path,
+                   "kernel_path": args.path, "mode": wl.mode,
                    "l2": f"inputs larger than L2: W_out "
                          f"({wl.V * wl.H * (2 if wl.weight_dtype == 'bf16' else 4) / 1e6:.0f} MB) "
                          f"streamed per stage; base logits rotate over "
@@ -418,7 +420,7 @@ def run_ours(args, wl, rank, world, local_rank):
 
 def main():
     args = parse_args()
-    wl = WORKLOADS[args.workload]
+    wl = WORKLOADS[args.workload].with_(mode=args.mode)
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

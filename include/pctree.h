@@ -57,6 +57,18 @@ typedef enum {
 
 typedef enum { PCTREE_F32 = 0, PCTREE_BF16 = 1 } pctree_dtype;
 
+/* Scoring of the tree's children.
+ *   PCTREE_MODE_PARENT  PCTree: every frontier parent gets its own Markov bias
+ *                       (Eqs. 2-3).
+ *   PCTREE_MODE_SHARED  the Shared-Markov control of the mechanism study
+ *                       (Sec. 5.3): the greedy DSpark chain of Eq. 1 is built
+ *                       alongside the tree and its distribution at depth d
+ *                       serves every parent at that depth (one batch-1 Markov
+ *                       call per stage and request); frontier, budget,
+ *                       selection and packing are unchanged.
+ * k = 1 with either mode is DSpark's single chain (Sec. 4.2). */
+typedef enum { PCTREE_MODE_PARENT = 0, PCTREE_MODE_SHARED = 1 } pctree_mode;
+
 /* Compiled limits. */
 #define PCTREE_MAX_K 32        /* per-parent top-k and frontier width        */
 #define PCTREE_MAX_N 1024      /* node budget, root included                 */
@@ -79,11 +91,12 @@ typedef enum { PCTREE_F32 = 0, PCTREE_BF16 = 1 } pctree_dtype;
  *   pos_offset   verified prefix length: position id = depth + pos_offset
  *                (Appendix A).
  *   weight_dtype storage type of both head matrices (pctree_dtype).
+ *   mode         child scoring (pctree_mode).
  * The candidate pool holds 1 + k + (B-1) k^2 nodes (Sec. 4.1); it must not
  * exceed PCTREE_MAX_POOL.
  */
 typedef struct {
-  int32_t V, H, B, k, N, batch, pos_offset, weight_dtype;
+  int32_t V, H, B, k, N, batch, pos_offset, weight_dtype, mode;
 } pctree_config;
 
 /*

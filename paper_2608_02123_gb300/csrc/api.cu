@@ -29,6 +29,8 @@ pctree_status check_config(const pctree_config* c) {
   if (c->k > c->V) return PCTREE_ERR_INVALID_ARG;
   if (c->weight_dtype != PCTREE_F32 && c->weight_dtype != PCTREE_BF16)
     return PCTREE_ERR_INVALID_ARG;
+  if (c->mode != PCTREE_MODE_PARENT && c->mode != PCTREE_MODE_SHARED)
+    return PCTREE_ERR_INVALID_ARG;
   if (c->weight_dtype == PCTREE_BF16 && (c->H % 8) != 0)
     return PCTREE_ERR_INVALID_ARG;
   if (c->k > PCTREE_MAX_K || c->N > PCTREE_MAX_N) return PCTREE_ERR_UNSUPPORTED;
@@ -42,7 +44,7 @@ pctree_status check_config(const pctree_config* c) {
 
 Layout make_layout(const pctree_config& c) {
   Layout l{};
-  l.rows_max = c.batch * c.k;
+  l.rows_max = c.batch * (c.mode == PCTREE_MODE_SHARED ? 1 : c.k);
   l.rows_pad = static_cast<int>(align_up(l.rows_max, 16));
   l.bn = l.rows_pad <= 16 ? 16 : l.rows_pad <= 32 ? 32 : l.rows_pad <= 64 ? 64
          : l.rows_pad <= 128 ? 128 : 256;
@@ -189,6 +191,7 @@ pctree_status draft_fused(const pctree_config& c, const Layout& lay,
   a.B = c.B;
   a.k = c.k;
   a.batch = c.batch;
+  a.shared = c.mode == PCTREE_MODE_SHARED ? 1 : 0;
   a.P = lay.P;
   a.n_k = (c.H + 63) / 64;
   a.n_tiles = n_tiles;
@@ -227,7 +230,7 @@ using namespace pct;
 
 extern "C" {
 
-int32_t pctree_version(void) { return 100; }
+int32_t pctree_version(void) { return 101; }
 
 const char* pctree_status_string(int32_t s) {
   switch (s) {
@@ -308,19 +311,19 @@ pctree_status pctree_draft(const pctree_config* cfg, const float* base_logits,
   float* Z = reinterpret_cast<float*>(ws + lay.off_z);
   const long long l_req_stride = static_cast<long long>(c.B) * c.V;
   for (int d = 0; d < c.B; ++d) {
-    const int b_d = d == 0 ? 1 : c.k;  // frontier size b_d (Sec. 4.1)
-    const int rows = c.batch * b_d;
+    const int rpq = rows_per_request(c, d);  // b_d (Sec. 4.1), or 1
+    const int rows = c.batch * rpq;
     const float* L_d = base_logits + static_cast<size_t>(d) * c.V;
     prof_record(0, stream);
     cudaError_t e;
     if (c.weight_dtype == PCTREE_BF16) {
       e = launch_markov_bf16(&tmap_w, &tmap_x, L_d, l_req_stride, Z, lay.ldz,
-                             c.V, c.H, rows, b_d, lay.bn, num_sms, out->status,
+                             c.V, c.H, rows, rpq, lay.bn, num_sms, out->status,
                              stream);
     } else {
       e = launch_markov_f32(static_cast<const float*>(head_out),
                             reinterpret_cast<const float*>(ws + lay.off_x), L_d,
-                            l_req_stride, Z, lay.ldz, c.V, c.H, rows, b_d,
+                            l_req_stride, Z, lay.ldz, c.V, c.H, rows, rpq,
                             out->status, stream);
     }
     prof_record(1, stream);

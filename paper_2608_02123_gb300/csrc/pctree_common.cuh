@@ -44,6 +44,7 @@ constexpr int kFusedMaxGrid = 256;
 struct FusedArgs {
   const float* L;        // [batch][B][V] base logits
   int V, H, B, k, batch, P, n_k, n_tiles;
+  int shared;            // 1: Shared-Markov control (one chain row per request)
   int32_t* pool_tok;     // [batch][P]
   int32_t* pool_par;     // [batch][P]
   float2* pool_s;        // [batch][P] joint score as (hi, lo)
@@ -265,6 +266,12 @@ cudaError_t launch_init(const pctree_config& c, const Layout& lay,
 cudaError_t launch_partials(const Layout& lay, int k, int V, int rows,
                             unsigned char* ws, int32_t* status,
                             cudaStream_t stream);
+
+// Markov rows per request at stage d: its frontier (PCTree) or the single
+// chain parent (Shared-Markov control).
+inline int rows_per_request(const pctree_config& c, int d) {
+  return c.mode == PCTREE_MODE_SHARED ? 1 : (d == 0 ? 1 : c.k);
+}
 
 cudaError_t launch_merge(const pctree_config& c, const Layout& lay, int d,
                          const void* E_in, unsigned char* ws,

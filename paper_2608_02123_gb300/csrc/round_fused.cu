@@ -1,6 +1,7 @@
 // One whole PCTree drafting round (Algorithm 1, stages d = 0..B-1) in a single
 // persistent, cooperative launch, for rounds with at most 16 Markov rows per
-// stage (batch * k <= 16, k <= 16) -- the batch-1 drafting of Sec. 5.
+// stage (batch * k <= 16, k <= 16) -- the batch-1 drafting of Sec. 5 -- with
+// either child scoring (PCTree, or the Shared-Markov control of Sec. 5.3).
 //
 // Per stage d, every CTA (one per SM) streams its share of W_out tiles with
 // TMA and multiplies them on the tensor cores (tcgen05, bf16 -> f32 in TMEM)
@@ -71,6 +72,7 @@ struct FusedSmem {
   unsigned long long keys[R * kMaxKF];     // new layer: (score, id) keys
   int ktok[R * kMaxKF];                    // new layer: tokens
   int ftok[R];                             // next stage's parent tokens
+  int ctok[R];                             // chain tokens (Shared-Markov)
 };
 
 template <int R>
@@ -255,7 +257,8 @@ __device__ void merge_stage(const CUtensorMap* tmap_w, const FusedArgs& a,
   const int tid = ew * 32 + lane;          // 0..255
   const int grid = gridDim.x;
   const int b_d = d == 0 ? 1 : a.k;
-  const int rows = a.batch * b_d;
+  const int rpq = a.shared ? 1 : b_d;      // Markov rows per request
+  const int rows = a.batch * rpq;
   const int k = a.k;
   const int n_layer = b_d * k;
   const int base = level_base(d + 1, k);
@@ -319,27 +322,36 @@ __device__ void merge_stage(const CUtensorMap* tmap_w, const FusedArgs& a,
       }
     }
     __syncwarp();
-    const int req = c / b_d, j = c - req * b_d;
+    const int req = c / rpq, j0 = c - req * rpq;
     int32_t* tok = a.pool_tok + static_cast<size_t>(req) * a.P;
     int32_t* par = a.pool_par + static_cast<size_t>(req) * a.P;
     float2* sc = a.pool_s + static_cast<size_t>(req) * a.P;
-    const int pid = a.front[req * k + j];
-    if (lane < k) {
-      const int id = base + j * k + lane;
-      int t = lst.t;
-      float logpi = lst.v - lse;
-      if (t < 0 || t >= a.V) {
-        t = 0;
-        logpi = kNegInf;
+    int t = lst.t;
+    float logpi = lst.v - lse;
+    if (t < 0 || t >= a.V) {
+      t = 0;
+      logpi = kNegInf;
+    }
+    // PCTree: this row's children belong to frontier slot j0.  Shared-Markov:
+    // the chain row's children go to every slot of the request.
+    const int j_lo = a.shared ? 0 : j0, j_hi = a.shared ? b_d : j0 + 1;
+    for (int j = j_lo; j < j_hi; ++j) {
+      const int pid = a.front[req * k + j];
+      if (lane < k) {
+        const int id = base + j * k + lane;
+        const float2 sn = ff_add(sc[pid], logpi);   // Eq. 4
+        tok[id] = t;
+        par[id] = pid;
+        sc[id] = sn;
+        const int i = req * n_layer + j * k + lane;
+        S->keys[i] = (static_cast<unsigned long long>(desc_key(sn.x)) << 32) |
+                     static_cast<unsigned int>(id);
+        S->ktok[i] = t;
       }
-      const float2 sn = ff_add(sc[pid], logpi);   // Eq. 4
-      tok[id] = t;
-      par[id] = pid;
-      sc[id] = sn;
-      const int i = req * n_layer + j * k + lane;
-      S->keys[i] = (static_cast<unsigned long long>(desc_key(sn.x)) << 32) |
-                   static_cast<unsigned int>(id);
-      S->ktok[i] = t;
+    }
+    if (a.shared) {                        // the chain continues (Eq. 1)
+      const int top = __shfl_sync(kFull, t, 0);
+      if (lane == 0) S->ctok[req] = top;
     }
   }
   if (d == a.B - 1) return;
@@ -358,10 +370,12 @@ __device__ void merge_stage(const CUtensorMap* tmap_w, const FusedArgs& a,
     }
   }
   epi_barrier();
-  // parent rows of the next stage: X[req * k + slot] = E_in[token]
+  // parent rows of the next stage: X[req * k + slot] = E_in[token] (PCTree)
+  // or X[req] = E_in[chain token] (Shared-Markov)
+  const int* row_tok = a.shared ? S->ctok : S->ftok;
   constexpr int kU = 10;
   const int per_row = a.H / 8;
-  const int total_v = a.batch * k * per_row;
+  const int total_v = a.batch * (a.shared ? 1 : k) * per_row;
   const uint4* src = static_cast<const uint4*>(a.E_in);
   uint4* dst = static_cast<uint4*>(a.X);
   for (int i0 = tid; i0 < total_v; i0 += kEpiThreads * kU) {
@@ -371,7 +385,7 @@ __device__ void merge_stage(const CUtensorMap* tmap_w, const FusedArgs& a,
       const int i = i0 + u * kEpiThreads;
       if (i < total_v) {
         const int row = i / per_row, off = i - row * per_row;
-        tmp[u] = src[static_cast<size_t>(S->ftok[row]) * per_row + off];
+        tmp[u] = src[static_cast<size_t>(row_tok[row]) * per_row + off];
       }
     }
 #pragma unroll
@@ -427,8 +441,8 @@ __device__ void epilogue(const CUtensorMap* tmap_w, const FusedArgs& a,
   int g_tile = 0;                          // tiles issued by the MMA so far
   bool bad = false;
   for (int d = 0; d < a.B; ++d) {
-    const int b_d = d == 0 ? 1 : k;
-    const int rows = a.batch * b_d;
+    const int rpq = a.shared ? 1 : (d == 0 ? 1 : k);   // rows per request
+    const int rows = a.batch * rpq;
     float m[R], s[R];
     WarpList lst[R];
 #pragma unroll
@@ -460,7 +474,7 @@ __device__ void epilogue(const CUtensorMap* tmap_w, const FusedArgs& a,
 #pragma unroll
       for (int c = 0; c < R; ++c) {
         if (c < rows) {
-          const int req = c / b_d;
+          const int req = c / rpq;
           float z = kNegInf;
           int t = 0x7fffffff;
           if (inb) {

@@ -197,7 +197,8 @@ __device__ void gather_rows(const void* E_in, void* X, const int* tok,
 }
 
 __global__ void __launch_bounds__(1024)
-merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
+merge_kernel(int d, int B, int k, int b_d, int rpq, int shared, int V, int H,
+             int P, int n_chunks,
              int x_elem, const float* __restrict__ part_m,
              const float* __restrict__ part_s,
              const float* __restrict__ part_z,
@@ -209,6 +210,7 @@ merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
   const int warp = threadIdx.x >> 5;
   extern __shared__ unsigned long long sm_keys[];  // b_d * k layer keys
   __shared__ int sm_tok[PCTREE_MAX_K];
+  __shared__ int sm_chain;
 
   int32_t* tok = pool_tok + static_cast<size_t>(r) * P;
   int32_t* par = pool_par + static_cast<size_t>(r) * P;
@@ -216,9 +218,11 @@ merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
   int32_t* fr = front + static_cast<size_t>(r) * k;
   const int base = level_base(d + 1, k);
 
-  if (warp < b_d) {
+  // one warp per Markov row: a frontier slot (PCTree) or the chain parent
+  // (Shared-Markov, rpq = 1)
+  if (warp < rpq) {
     const int j = warp;
-    const int row = r * b_d + j;
+    const int row = r * rpq + j;
     const size_t p0 = static_cast<size_t>(row) * n_chunks;
     // log-softmax normaliser from the chunk partials (Eq. 2)
     const float lse = warp_lse_from_partials<kUnroll>(part_m + p0, part_s + p0,
@@ -248,19 +252,26 @@ merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
         }
       }
     }
-    const int pid = fr[j];
-    if (lane < k) {
-      const int id = base + j * k + lane;
-      int t = lst.t;
-      float logpi = lst.v - lse;
-      if (t < 0 || t >= V) {  // only when V < k (rejected on the host)
-        t = 0;
-        logpi = kNegInf;
-      }
-      tok[id] = t;
-      par[id] = pid;
-      sc[id] = ff_add(sc[pid], logpi);  // Eq. 4: s(child) = s(p) + log pi
+    int t = lst.t;
+    float logpi = lst.v - lse;
+    if (t < 0 || t >= V) {  // only when V < k (rejected on the host)
+      t = 0;
+      logpi = kNegInf;
     }
+    // PCTree: the row's children belong to slot j; Shared-Markov: the chain
+    // row's children go to every slot of the request.
+    const int j_lo = shared ? 0 : j, j_hi = shared ? b_d : j + 1;
+    for (int jj = j_lo; jj < j_hi; ++jj) {
+      const int pid = fr[jj];
+      if (lane < k) {
+        const int id = base + jj * k + lane;
+        tok[id] = t;
+        par[id] = pid;
+        sc[id] = ff_add(sc[pid], logpi);  // Eq. 4: s(child) = s(p) + log pi
+      }
+    }
+    const int top = __shfl_sync(kFull, t, 0);
+    if (lane == 0 && j == 0) sm_chain = top;   // argmax of the row (Eq. 1)
   }
   if (d == B - 1) return;
   __syncthreads();
@@ -283,7 +294,14 @@ merge_kernel(int d, int B, int k, int b_d, int V, int H, int P, int n_chunks,
   }
   __syncthreads();
   // Markov input rows of the next stage: X[r * k + slot] = E_in[token]
-  gather_rows(E_in, X, sm_tok, k, r * k, H, x_elem);
+  // (PCTree) or X[r] = E_in[chain token] (Shared-Markov)
+  if (shared) {
+    if (threadIdx.x == 0) sm_tok[0] = sm_chain;
+    __syncthreads();
+    gather_rows(E_in, X, sm_tok, 1, r, H, x_elem);
+  } else {
+    gather_rows(E_in, X, sm_tok, k, r * k, H, x_elem);
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -582,10 +600,12 @@ cudaError_t launch_merge(const pctree_config& c, const Layout& lay, int d,
                          const void* E_in, unsigned char* ws,
                          int32_t* status, cudaStream_t stream) {
   const int b_d = d == 0 ? 1 : c.k;
+  const int rpq = rows_per_request(c, d);
   const size_t smem = static_cast<size_t>(b_d) * c.k * sizeof(unsigned long long);
-  const int threads = b_d * 32 > 256 ? b_d * 32 : 256;
+  const int threads = rpq * 32 > 256 ? rpq * 32 : 256;
   merge_kernel<<<c.batch, threads, smem, stream>>>(
-      d, c.B, c.k, b_d, c.V, c.H, lay.P, lay.n_chunks, lay.x_elem,
+      d, c.B, c.k, b_d, rpq, c.mode == PCTREE_MODE_SHARED ? 1 : 0, c.V, c.H,
+      lay.P, lay.n_chunks, lay.x_elem,
       reinterpret_cast<const float*>(ws + lay.off_pm),
       reinterpret_cast<const float*>(ws + lay.off_ps),
       reinterpret_cast<const float*>(ws + lay.off_pz),

@@ -38,7 +38,7 @@ class Config(ctypes.Structure):
                 ("B", ctypes.c_int32), ("k", ctypes.c_int32),
                 ("N", ctypes.c_int32), ("batch", ctypes.c_int32),
                 ("pos_offset", ctypes.c_int32),
-                ("weight_dtype", ctypes.c_int32)]
+                ("weight_dtype", ctypes.c_int32), ("mode", ctypes.c_int32)]
 
 
 class _Tree(ctypes.Structure):
@@ -88,10 +88,16 @@ LIB = _load()
 LIB_PATH = _LIB_PATH
 
 
+MODE_PARENT, MODE_SHARED = 0, 1
+
+
 def make_config(V: int, H: int, B: int, k: int, N: int, batch: int = 1,
-                pos_offset: int = 0, weight_dtype: str = "bf16") -> Config:
+                pos_offset: int = 0, weight_dtype: str = "bf16",
+                mode: str = "parent") -> Config:
+    """``mode``: "parent" (PCTree) or "shared" (the Shared-Markov control)."""
     return Config(V, H, B, k, N, batch, pos_offset,
-                  PCTREE_BF16 if weight_dtype == "bf16" else PCTREE_F32)
+                  PCTREE_BF16 if weight_dtype == "bf16" else PCTREE_F32,
+                  MODE_SHARED if mode == "shared" else MODE_PARENT)
 
 
 def pctree_check_config(cfg: Config) -> int:
@@ -266,7 +272,8 @@ def kernels_per_round(cfg: Config, path: int = PATH_AUTO) -> int:
         return 3                      # init, fused round, pack
     launches = 2                      # init, pack
     for d in range(cfg.B):
-        rows = cfg.batch * (1 if d == 0 else cfg.k)
+        rpq = 1 if (cfg.mode == MODE_SHARED or d == 0) else cfg.k
+        rows = cfg.batch * rpq
         passes = (rows + 255) // 256 if cfg.weight_dtype == PCTREE_BF16 else 1
         launches += passes + 2        # projection, partials, merge
     return launches

@@ -34,7 +34,7 @@ def run_gpu(inp: RoundInputs, with_pool=True, accept=True,
     from paper_2608_02123_gb300 import pctree as P
     wl = inp.wl
     cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, inp.L.shape[0],
-                        wl.pos_offset, wl.weight_dtype)
+                        wl.pos_offset, wl.weight_dtype, wl.mode)
     L, E, W, root = device_inputs(inp)
     dr = P.Drafter(cfg, with_pool=with_pool)
     P.pctree_set_path(path)
@@ -109,7 +109,7 @@ def compare(inp: RoundInputs, host: Dict[str, np.ndarray],
         assert int(host["status"][0]) == 0, host["status"]
         hint = None if strict else gpu_choices(host, r)
         rnd = O.draft(inp.L[r], E64, W64, int(inp.root[r]), wl.B, wl.k, wl.N,
-                      wl.pos_offset, hint=hint)
+                      wl.pos_offset, hint=hint, mode=wl.mode)
         t = rnd.tree
         rep.requests += 1
         rep.ambiguous += rnd.n_ambiguous

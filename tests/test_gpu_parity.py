@@ -40,6 +40,13 @@ SMALL = {
                               k=6, N=24, batch=4, seed=20),
     "f32_pos_offset": WORKLOADS["tiny"].with_(V=3001, H=37, B=5, k=3, N=20,
                                               batch=2, seed=21, pos_offset=123),
+    # Shared-Markov control (Sec. 5.3)
+    "shared_ragged_bf16": strong(BASE, V=3000, H=256, B=5, k=4, N=16, batch=3,
+                                 seed=23, mode="shared"),
+    "shared_batched_bf16": strong(BASE, V=2000, H=64, B=4, k=8, N=40,
+                                  batch=12, seed=24, mode="shared"),
+    "shared_f32": WORKLOADS["tiny"].with_(V=1500, H=40, B=4, k=3, N=10,
+                                          batch=2, seed=25, mode="shared"),
 }
 
 
@@ -145,6 +152,9 @@ def test_host_errors_need_no_work():
 
 @functools.lru_cache(maxsize=1)
 def _full(name, requests=None):
+    if name == "4b_b16_shared":
+        wl = WORKLOADS["4b_b16"].with_(mode="shared")
+        return draw_round(wl)
     wl = WORKLOADS[name]
     reqs = None if requests is None else range(requests)
     return draw_round(wl.with_(batch=wl.batch if requests is None else requests),
@@ -152,7 +162,8 @@ def _full(name, requests=None):
 
 
 @pytest.mark.parametrize("path", sorted(PATHS))
-@pytest.mark.parametrize("name", ["4b_b16", "4b_b16_chain", "4b_b7"])
+@pytest.mark.parametrize("name", ["4b_b16", "4b_b16_chain", "4b_b7",
+                                  "4b_b16_shared"])
 def test_full_size_batch1(name, path):
     inp = _full(name)
     host = G.run_gpu(inp, path=PATHS[path])

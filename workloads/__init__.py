@@ -58,6 +58,7 @@ class Workload:
     target_p: float     # probability that the target's token is the likely one
     seed: int
     pos_offset: int = 0  # verified-prefix length added to tree depths
+    mode: str = "parent"  # "parent" (PCTree) or "shared" (Shared-Markov)
 
     def with_(self, **kw) -> "Workload":
         return dataclasses.replace(self, **kw)
