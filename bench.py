@@ -49,6 +49,10 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--mode", default="parent", choices=["parent", "shared"],
                     help="child scoring: PCTree, or the Shared-Markov control")
+    ap.add_argument("--sweep", action="store_true",
+                    help="k/N sweep (B in {7,16}, k in {1,2,4,8}, N in "
+                         "{8..128}) on the workload's shapes, batch 1: one "
+                         "JSON line per point instead of the benchmark line")
     ap.add_argument("--path", default="auto", choices=["auto", "stagewise"],
                     help="kernel path: fused round where it applies, or the "
                          "per-stage kernels for every round")
@@ -418,9 +422,82 @@ def run_ours(args, wl, rank, world, local_rank):
     print(json.dumps(line), flush=True)
 
 
+# ---------------------------------------------------------------------------
+# k / N sweep (the shapes of the paper's ablations, Sec. 5.4)
+# ---------------------------------------------------------------------------
+
+SWEEP_B = (7, 16)
+SWEEP_K = (1, 2, 4, 8)
+SWEEP_N = (8, 16, 24, 32, 48, 64, 96, 128)
+
+
+def run_sweep(args, wl, local_rank):
+    import torch
+
+    from paper_2608_02123_gb300 import pctree as P
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    base = wl.with_(B=max(SWEEP_B), batch=1)
+    E_host, W_host = draw_head(base)
+    E = torch.from_numpy(E_host.view(np.int16)).to(dev).view(torch.bfloat16)
+    W = torch.from_numpy(W_host.view(np.int16)).to(dev).view(torch.bfloat16)
+    n_sets = N_SETS
+    many = base.with_(batch=n_sets)
+    reqs = [draw_request(many, i) for i in range(n_sets)]
+    peak = float(measured_peaks()[0]["hbm_gbs"])
+    steps = max(args.steps // 4, 10)
+    stream = torch.cuda.current_stream()
+    for B in SWEEP_B:
+        L_dev = [torch.from_numpy(np.ascontiguousarray(q[0][None, :B])).to(dev)
+                 for q in reqs]
+        root_dev = [torch.tensor([q[1]], dtype=torch.int32, device=dev)
+                    for q in reqs]
+        g_dev = [torch.from_numpy(np.concatenate([q[2][:B], q[2][-1:]])[None]
+                                  .astype(np.int64)).to(dev) for q in reqs]
+        for k in SWEEP_K:
+            for N in SWEEP_N:
+                wk = base.with_(B=B, k=k, N=N)
+                cfg = P.make_config(wk.V, wk.H, B, k, N, 1, 0, "bf16", wk.mode)
+                dr = P.Drafter(cfg, dev)
+                taus = []
+
+                def step(i, keep=False):
+                    dr.draft(L_dev[i % n_sets], E, W, root_dev[i % n_sets], stream)
+                    depth = dr.tree.depth.long().clamp_min(0)
+                    tgt = torch.gather(g_dev[i % n_sets], 1, depth).to(torch.int32)
+                    dr.accept(tgt, stream)
+                    if keep:
+                        taus.append(dr.accepted_len.clone())
+
+                for i in range(3):
+                    step(i)
+                torch.cuda.synchronize()
+                start = torch.cuda.Event(enable_timing=True)
+                end = torch.cuda.Event(enable_timing=True)
+                start.record(stream)
+                for i in range(steps):
+                    step(i, keep=True)
+                end.record(stream)
+                torch.cuda.synchronize()
+                dr.check_status()
+                ms = start.elapsed_time(end) / steps
+                tau = float(torch.stack(taus).float().mean()) + 1.0
+                print(json.dumps({
+                    "sweep": "kN", "workload": wk.name, "mode": wk.mode,
+                    "B": B, "k": k, "N": N, "us_per_round": ms * 1e3,
+                    "rounds_per_s": 1e3 / ms,
+                    "round_hbm_fraction": round_bytes(wk) / (ms * 1e-3) / 1e9 / peak,
+                    "fused": P.uses_fused_round(cfg),
+                    "mean_tau_synthetic_target": tau}), flush=True)
+
+
 def main():
     args = parse_args()
     wl = WORKLOADS[args.workload].with_(mode=args.mode)
+    if args.sweep:
+        run_sweep(args, wl, int(os.environ.get("LOCAL_RANK", "0")))
+        return
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

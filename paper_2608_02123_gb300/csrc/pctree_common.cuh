@@ -144,30 +144,30 @@ struct WarpList {
     if (lane >= k) reset();
   }
   // Offers one candidate per lane (lanes with nothing pass the sentinel).
+  // Every candidate better than the list's k-th entry at the start of the
+  // call is inserted in turn; one that an earlier insert has pushed below
+  // the k-th place lands at position >= k and is dropped by insert().
   __device__ __forceinline__ void offer(float cv, int ct, int k) {
-    float tv = __shfl_sync(kFull, v, k - 1);
-    int tt = __shfl_sync(kFull, t, k - 1);
+    const float tv = __shfl_sync(kFull, v, k - 1);
+    const int tt = __shfl_sync(kFull, t, k - 1);
     unsigned m = __ballot_sync(kFull, cand_better(cv, ct, tv, tt));
     while (m) {
       const int src = __ffs(m) - 1;
-      const float sv = __shfl_sync(kFull, cv, src);
-      const int st = __shfl_sync(kFull, ct, src);
-      insert(sv, st, k);
-      tv = __shfl_sync(kFull, v, k - 1);
-      tt = __shfl_sync(kFull, t, k - 1);
-      m &= ~(1u << src);
-      m &= __ballot_sync(kFull, cand_better(cv, ct, tv, tt));
+      m &= m - 1;
+      insert(__shfl_sync(kFull, cv, src), __shfl_sync(kFull, ct, src), k);
     }
   }
 };
 
-// Online (max, sum exp) pair; m = -inf means "no finite value yet".
+// Online (max, sum exp) pair; m = -inf means "no finite value yet".  The
+// terms exp(x), x <= 0, use the fast exponential: its relative error (a few
+// 1e-7) stays far below the 1e-4 tolerance on log-probabilities.
 __device__ __forceinline__ void lse_push(float& m, float& s, float z) {
   if (z > m) {
-    s = s * expf(m - z) + 1.0f;
+    s = s * __expf(m - z) + 1.0f;
     m = z;
   } else if (z > -__int_as_float(0x7f800000)) {
-    s += expf(z - m);
+    s += __expf(z - m);
   }
 }
 

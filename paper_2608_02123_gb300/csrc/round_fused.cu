@@ -452,6 +452,7 @@ __device__ void epilogue(const CUtensorMap* tmap_w, const FusedArgs& a,
       lst[c].reset();
     }
     bool ok = true;
+    bool first = true;                     // first tile of this stage
     for (int i = 0; i < n_my; ++i, ++g_tile) {
       if ((g_tile & 1) != grp) continue;
       const int tile = tile_at(d, i, n_my);
@@ -471,6 +472,8 @@ __device__ void epilogue(const CUtensorMap* tmap_w, const FusedArgs& a,
       const int v = tile * kBM + quad * 32 + lane;
       const bool inb = v < a.V;
       const float* Lrow = a.L + static_cast<size_t>(d) * a.V + (inb ? v : 0);
+      int cur_req = -1;
+      float lval = 0.0f;
 #pragma unroll
       for (int c = 0; c < R; ++c) {
         if (c < rows) {
@@ -478,15 +481,23 @@ __device__ void epilogue(const CUtensorMap* tmap_w, const FusedArgs& a,
           float z = kNegInf;
           int t = 0x7fffffff;
           if (inb) {
-            const float lval = __ldg(Lrow + static_cast<size_t>(req) * a.B * a.V);
+            if (req != cur_req) {   // one base-logit load per request
+              cur_req = req;
+              lval = __ldg(Lrow + static_cast<size_t>(req) * a.B * a.V);
+            }
             z = lval + acc[c];
             t = v;
             bad |= isnan(z) || (isinf(z) && !(isinf(lval) && lval < 0.0f));
             lse_push(m[c], s[c], z);
           }
-          lst[c].offer(z, t, k);
+          if (first) {
+            lst[c].seed(z, t, k);   // a sort instead of 32 serial inserts
+          } else {
+            lst[c].offer(z, t, k);
+          }
         }
       }
+      first = false;
     }
     if (!ok) {
       *abort_v = 1;

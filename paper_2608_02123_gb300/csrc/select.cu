@@ -427,15 +427,20 @@ pack_kernel(int B, int k, int N, int P, int pos_offset,
     const bool at = my_lvl == t;
     unsigned long long key2 = 0ull;
     if (at) {
-      const int pp = t == 0 ? -1 : pidx[par[my_id]];
+      const int pid = par[my_id];
+      const int pp = (t == 0 || pid < 0 || pid >= P) ? -1 : pidx[pid];
       key2 = (static_cast<unsigned long long>(static_cast<unsigned int>(pp + 1)) << 32) |
              static_cast<unsigned int>(tok[my_id]);
     }
     int n_t;
     block_excl_scan(at ? 1 : 0, sm_warp, &n_t);
     if (n_t == 0) break;
-    // rank among the nodes of this level (<= n of them)
+    // rank among the nodes of this level (<= n of them).  Siblings carry
+    // distinct tokens, so (parent, token) is unique; the pool id breaks ties
+    // anyway so that every packed slot is written exactly once whatever the
+    // pool holds (e.g. after a round already flagged non-finite).
     __shared__ unsigned long long sm_k2[PCTREE_MAX_N];
+    __shared__ int sm_kid[PCTREE_MAX_N];
     __shared__ int sm_lvl_slot;
     if (tid == 0) sm_lvl_slot = 0;
     __syncthreads();
@@ -443,11 +448,13 @@ pack_kernel(int B, int k, int N, int P, int pos_offset,
     if (at) {
       slot = atomicAdd(&sm_lvl_slot, 1);
       sm_k2[slot] = key2;
+      sm_kid[slot] = my_id;
     }
     __syncthreads();
     if (at) {
       int rank = 0;
-      for (int j = 0; j < n_t; ++j) rank += sm_k2[j] < key2;
+      for (int j = 0; j < n_t; ++j)
+        rank += sm_k2[j] < key2 || (sm_k2[j] == key2 && sm_kid[j] < my_id);
       const int a = placed + rank;
       pidx[my_id] = a;
       sm_sel[a] = my_id;  // safe: slots of this level are read via my_id only
@@ -456,14 +463,20 @@ pack_kernel(int B, int k, int N, int P, int pos_offset,
     __syncthreads();
   }
   // per packed node: parent index, child flags
+  // A parent is packed before its children (ids grow with depth and the
+  // selection is ancestor-closed), so sm_par[a] < a; anything else is
+  // recorded as "no parent", which keeps every walk below finite.
   for (int a = tid; a < n; a += blockDim.x) {
     const int id = sm_sel[a];
-    sm_par[a] = a == 0 ? -1 : pidx[par[id]];
+    const int pid = par[id];
+    int pa = (a == 0 || pid < 0 || pid >= P) ? -1 : pidx[pid];
+    if (pa >= a) pa = -1;
+    sm_par[a] = pa;
     sm_haschild[a] = 0;
   }
   __syncthreads();
   for (int a = tid; a < n; a += blockDim.x)
-    if (a > 0) sm_haschild[sm_par[a]] = 1;
+    if (sm_par[a] >= 0) sm_haschild[sm_par[a]] = 1;
   __syncthreads();
   int32_t* o_tok = out.tokens + static_cast<size_t>(r) * N;
   int32_t* o_par = out.parent + static_cast<size_t>(r) * N;
@@ -505,7 +518,7 @@ pack_kernel(int B, int k, int N, int P, int pos_offset,
     if (is_leaf) {
       int32_t* row = o_ret + static_cast<size_t>(leaf_rank) * (B + 1);
       int dpt = level_of(sm_sel[tid], k);
-      for (int b = tid; b >= 0; b = sm_par[b]) row[dpt--] = b;
+      for (int b = tid; b >= 0 && dpt >= 0; b = sm_par[b]) row[dpt--] = b;
     }
   }
   if (tid == 0) {
