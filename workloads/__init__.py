@@ -242,3 +242,113 @@ def target_for_tree(greedy: np.ndarray, depth: np.ndarray) -> np.ndarray:
         valid = (depth[r] >= 0) & (depth[r] < greedy.shape[1])
         out[r, valid] = greedy[r, depth[r, valid]]
     return out
+
+
+# ----------------------------------------------------------------------------
+# accepted-row compaction inputs (caches after a tree verification)
+# ----------------------------------------------------------------------------
+
+@dataclasses.dataclass(frozen=True)
+class CompactWorkload:
+    """Shapes of the per-token caches a verification forward leaves behind.
+
+    A cache plane holds one row of ``row_bytes`` per (request, slot); each
+    layer has ``planes`` of them (K and V).  ``hidden_bytes`` is one target
+    hidden-state row.  Slots per request: ``prefix_max + N``.
+    """
+
+    name: str
+    layers: int
+    planes: int
+    row_bytes: int
+    hidden_bytes: int
+    B: int
+    N: int
+    batch: int
+    prefix_max: int
+    seed: int
+
+    @property
+    def slots(self) -> int:
+        return self.prefix_max + self.N
+
+    def cache_bytes(self) -> int:
+        return self.layers * self.planes * self.batch * self.slots * self.row_bytes
+
+
+# Qwen3 KV shapes: 8 KV heads x head_dim 128 in bf16 = 2048 bytes per token
+# and plane; 36 layers (4B, 8B) or 40 (14B); hidden 2560 / 4096 / 5120 bf16.
+COMPACT_WORKLOADS: Dict[str, CompactWorkload] = {
+    "small": CompactWorkload("small_L3_row64_B5_N16_bs3", layers=3, planes=2,
+                             row_bytes=64, hidden_bytes=96, B=5, N=16,
+                             batch=3, prefix_max=40, seed=20),
+    "ragged": CompactWorkload("ragged_L2_row16_B9_N12_bs5", layers=2,
+                              planes=3, row_bytes=16, hidden_bytes=32, B=9,
+                              N=12, batch=5, prefix_max=7, seed=21),
+    "4b_b16": CompactWorkload("qwen3_4b_L36_kv2048_B16_N64_bs1", layers=36,
+                              planes=2, row_bytes=2048, hidden_bytes=5120,
+                              B=16, N=64, batch=1, prefix_max=2048, seed=22),
+    "8b_b7_bs16": CompactWorkload("qwen3_8b_L36_kv2048_B7_N64_bs16",
+                                  layers=36, planes=2, row_bytes=2048,
+                                  hidden_bytes=8192, B=7, N=64, batch=16,
+                                  prefix_max=1024, seed=23),
+    "14b_b16_bs32": CompactWorkload("qwen3_14b_L40_kv2048_B16_N128_bs32",
+                                    layers=40, planes=2, row_bytes=2048,
+                                    hidden_bytes=10240, B=16, N=128,
+                                    batch=32, prefix_max=1024, seed=24),
+}
+
+
+@dataclasses.dataclass
+class CompactInputs:
+    cw: CompactWorkload
+    accepted_idx: np.ndarray   # [batch][B+1] int32, -1 padded
+    accepted_len: np.ndarray   # [batch] int32
+    prefix_len: np.ndarray     # [batch] int32
+    cache: Optional[np.ndarray]       # uint8 [layers][planes][batch][slots][row]
+    hidden_in: Optional[np.ndarray]   # uint8 [batch][N][hidden_bytes]
+    hidden_out: Optional[np.ndarray]  # uint8 [batch][B+1][hidden_bytes]
+
+
+def draw_accepted_paths(cw: CompactWorkload, rng: np.random.Generator):
+    """Accepted paths as the greedy tree rule returns them: the root (0)
+    followed by ``len`` strictly increasing packed indices below N, -1
+    padded.  Lengths mix 0, B (capped at N-1) and uniform values."""
+    B, N = cw.B, cw.N
+    top = min(B, N - 1)
+    acc = np.full((cw.batch, B + 1), -1, dtype=np.int32)
+    lens = np.zeros(cw.batch, dtype=np.int32)
+    for r in range(cw.batch):
+        u = rng.random()
+        n = 0 if u < 0.1 else top if u < 0.2 else int(rng.integers(1, top + 1))
+        nodes = np.sort(rng.choice(np.arange(1, N), size=n, replace=False))
+        acc[r, 0] = 0
+        acc[r, 1:n + 1] = nodes
+        lens[r] = n
+    return acc, lens
+
+
+def draw_compaction(cw: CompactWorkload, seed: Optional[int] = None,
+                    fill: bool = True) -> CompactInputs:
+    """Seeded compaction inputs.  Request 0 has the longest prefix allowed
+    (its tree ends at the last slot) and request 1, if any, an empty one.
+    ``fill=False`` skips the random cache and hidden-state bytes."""
+    ss = np.random.SeedSequence(cw.seed if seed is None else seed)
+    s_path, s_cache, s_hid = ss.spawn(3)
+    rng = np.random.default_rng(s_path)
+    acc, lens = draw_accepted_paths(cw, rng)
+    prefix = rng.integers(0, cw.prefix_max + 1, size=cw.batch).astype(np.int32)
+    prefix[0] = cw.prefix_max
+    if cw.batch > 1:
+        prefix[1] = 0
+    cache = hid_in = hid_out = None
+    if fill:
+        shape = (cw.layers, cw.planes, cw.batch, cw.slots, cw.row_bytes)
+        cache = np.random.default_rng(s_cache).integers(
+            0, 256, size=shape, dtype=np.uint8)
+        g = np.random.default_rng(s_hid)
+        hid_in = g.integers(0, 256, size=(cw.batch, cw.N, cw.hidden_bytes),
+                            dtype=np.uint8)
+        hid_out = g.integers(0, 256, size=(cw.batch, cw.B + 1, cw.hidden_bytes),
+                             dtype=np.uint8)
+    return CompactInputs(cw, acc, lens, prefix, cache, hid_in, hid_out)
