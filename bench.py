@@ -30,7 +30,8 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
-from workloads import WORKLOADS, draw_head, draw_request  # noqa: E402
+from workloads import (COMPACT_WORKLOADS, WORKLOADS, draw_compaction,  # noqa: E402
+                       draw_head, draw_request)
 
 METRIC = ("tree-draft rounds/sec & µs/round (V=151936, B=16, N=64); "
           "% of HBM roofline")
@@ -53,6 +54,12 @@ def parse_args():
                     help="k/N sweep (B in {7,16}, k in {1,2,4,8}, N in "
                          "{8..128}) on the workload's shapes, batch 1: one "
                          "JSON line per point instead of the benchmark line")
+    ap.add_argument("--op", default="round", choices=["round", "compact"],
+                    help="round: the drafting round (the benchmark line); "
+                         "compact: the accepted-row KV/hidden-state compaction "
+                         "after acceptance, on --compact-workload")
+    ap.add_argument("--compact-workload", default="14b_b16_bs32",
+                    choices=sorted(COMPACT_WORKLOADS))
     ap.add_argument("--path", default="auto", choices=["auto", "stagewise"],
                     help="kernel path: fused round where it applies, or the "
                          "per-stage kernels for every round")
@@ -492,9 +499,103 @@ def run_sweep(args, wl, local_rank):
                     "mean_tau_synthetic_target": tau}), flush=True)
 
 
+def compact_bytes(cw, acc, lens):
+    """Algorithmic bytes of one compaction: every moved cache row read and
+    written once (nodes with a[j] == j at the head of the path stay), every
+    gathered hidden-state row read and written once."""
+    total = 0
+    for r in range(cw.batch):
+        L = int(lens[r])
+        j = 1
+        while j <= L and acc[r, j] == j:
+            j += 1
+        total += (L + 1 - j) * cw.layers * cw.planes * cw.row_bytes * 2
+        total += (L + 1) * cw.hidden_bytes * 2
+    return total
+
+
+def run_compact(args, local_rank):
+    """Accepted-row compaction (the step after acceptance) on one GPU: a
+    cache of the workload's shape resident in HBM, accepted paths and
+    prefix lengths rotating over 16 seeded sets, so a launch's rows were
+    last touched 15 launches (and, at the large workloads, over 1 GB of
+    other rows) earlier: inputs larger than L2, no flush."""
+    import torch
+
+    from paper_2608_02123_gb300 import pctree as P
+
+    cw = COMPACT_WORKLOADS[args.compact_workload]
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(cw.seed)
+    cache = torch.randint(0, 256, (cw.cache_bytes(),), dtype=torch.uint8,
+                          device=dev, generator=gen)
+    hin = torch.randint(0, 256, (cw.batch, cw.N, cw.hidden_bytes),
+                        dtype=torch.uint8, device=dev, generator=gen)
+    hout = torch.zeros((cw.batch, cw.B + 1, cw.hidden_bytes), dtype=torch.uint8,
+                       device=dev)
+    sets = [draw_compaction(cw, seed=cw.seed * 1000 + i, fill=False)
+            for i in range(N_SETS)]
+    acc = [torch.from_numpy(c.accepted_idx).to(dev) for c in sets]
+    lens = [torch.from_numpy(c.accepted_len).to(dev) for c in sets]
+    pre = [torch.from_numpy(c.prefix_len).to(dev) for c in sets]
+    nbytes = [compact_bytes(cw, c.accepted_idx, c.accepted_len) for c in sets]
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    lay = P.compact_layout(cw.batch, cw.B, cw.N, cw.layers, cw.planes,
+                           cw.slots, cw.row_bytes, hidden_bytes=cw.hidden_bytes)
+    stream = torch.cuda.current_stream()
+
+    def step(i):
+        j = i % N_SETS
+        P.pctree_compact(lay, acc[j], lens[j], pre[j], cache, hin, hout,
+                         status, stream)
+
+    for i in range(max(args.warmup, 3)):
+        step(i)
+    torch.cuda.synchronize()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    start.record(stream)
+    for i in range(args.steps):
+        step(i)
+    end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if int(status.item()) != 0:
+        raise RuntimeError(f"pctree_compact status {int(status.item())}")
+    total_ms = start.elapsed_time(end)
+    moved = sum(nbytes[i % N_SETS] for i in range(args.steps))
+    peaks, src = measured_peaks()
+    peak = float(peaks["hbm_gbs"])
+    achieved = moved / (total_ms * 1e-3) / 1e9
+    us = total_ms * 1e3 / args.steps
+    print(json.dumps({
+        "metric": "accepted-row compaction µs/round (KV planes + hidden states)",
+        "value": us, "unit": "us/round", "higher_is_better": False,
+        "n_gpus": 1, "steps": args.steps, "warmup": max(args.warmup, 3),
+        "dtype": "u8", "data": "synthetic (seeded cache bytes and accepted paths)",
+        "config": {"workload": cw.name, "layers": cw.layers,
+                   "planes": cw.planes, "row_bytes": cw.row_bytes,
+                   "hidden_bytes": cw.hidden_bytes, "B": cw.B, "N": cw.N,
+                   "batch": cw.batch, "slots": cw.slots,
+                   "l2": "16 rotating path sets; rows larger than L2 between reuses"},
+        "bytes_per_round": moved / args.steps,
+        "roofline": {"bound": "hbm", "kernel": "compact_kernel",
+                     "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "peak_source": src,
+                     "traffic": None},
+        "gpu_launches": args.steps, "clocks": clk}), flush=True)
+
+
 def main():
     args = parse_args()
     wl = WORKLOADS[args.workload].with_(mode=args.mode)
+    if args.op == "compact":
+        run_compact(args, int(os.environ.get("LOCAL_RANK", "0")))
+        return
     if args.sweep:
         run_sweep(args, wl, int(os.environ.get("LOCAL_RANK", "0")))
         return

@@ -233,6 +233,72 @@ PCTREE_API pctree_status pctree_accept(const pctree_config* cfg, const pctree_tr
                             int32_t* accepted_idx, int32_t* accepted_len,
                             int32_t* bonus_token, void* stream);
 
+/*
+ * Accepted-row compaction (Appendix A "Tensor implementation": once the
+ * longest accepted row is known, the KV tensors and the target's hidden
+ * states are gathered along it and placed right after the verified prefix).
+ * This is the step after pctree_accept.
+ *
+ * The verification forward wrote one row per packed tree node i into slot
+ * T + i of every cache plane, T = prefix_len[r] the request's verified
+ * prefix.  For accepted nodes a = accepted_idx[r][0 .. L], L =
+ * accepted_len[r] (a[0] = 0 is the root):
+ *   every plane:   slot T + j  <-  slot T + a[j]       (j = 0 .. L, in place)
+ *   hidden states: hidden_out[r][j] <- hidden_in[r][a[j]]   (j = 0 .. L)
+ * Every other slot and hidden_out row keeps its content.  The caller's next
+ * verified prefix is T + L + 1 (root and accepted tokens); the bonus token
+ * becomes the next root.
+ *
+ * A cache plane is a block of byte rows addressed as
+ *   cache + layer * layer_stride + plane * plane_stride
+ *         + r * request_stride + slot * slot_stride
+ * (layer < layers, plane < planes, e.g. planes = 2 for K and V), which
+ * covers the usual contiguous layouts ([layers][2][batch][slots][heads*dim],
+ * [batch][layers][2][slots][...], ...).  Rows of distinct (layer, plane,
+ * request, slot) must not overlap.  Rows are moved as raw bytes: any
+ * element type.
+ */
+typedef struct {
+  int32_t batch;          /* requests                                       */
+  int32_t B;              /* draft depth: accepted_idx rows hold B+1 ints   */
+  int32_t N;              /* packed tree size (nodes written after prefix)  */
+  int32_t layers;         /* cache layers (0 with planes = 0: hidden only)  */
+  int32_t planes;         /* cache planes per layer                         */
+  int32_t max_slots;      /* slots per (layer, plane, request); T + N <= it */
+  int64_t row_bytes;      /* bytes of one slot's row, multiple of 16        */
+  int64_t slot_stride;    /* byte strides, each a multiple of 16            */
+  int64_t request_stride;
+  int64_t plane_stride;
+  int64_t layer_stride;
+  int64_t hidden_bytes;   /* one hidden-state row, multiple of 16; 0 = none */
+} pctree_compact_layout;
+
+/*
+ *   accepted_idx  [batch][B+1] int32, as written by pctree_accept
+ *   accepted_len  [batch] int32
+ *   prefix_len    [batch] int32, verified prefix length T of each request
+ *   cache         base of the cache planes (16-byte aligned; NULL allowed
+ *                 only when layers * planes == 0)
+ *   hidden_in     [batch][N][hidden_bytes] (16-byte aligned; NULL allowed
+ *                 only when hidden_bytes == 0)
+ *   hidden_out    [batch][B+1][hidden_bytes], must not overlap hidden_in
+ *   status        one device int32, or NULL.  A request whose accepted path
+ *                 is not one pctree_accept can return (a[0] != 0, indices
+ *                 not strictly increasing or >= N, L outside [0, B]) or
+ *                 whose T < 0 or T + N > max_slots is left untouched and
+ *                 PCTREE_ERR_INVALID_ARG is stored to *status; otherwise
+ *                 *status is not written (clear it before the call).
+ * Returns PCTREE_ERR_INVALID_ARG for a bad layout, pointer or alignment
+ * (nothing enqueued) and PCTREE_ERR_CUDA if the launch fails.  Memory
+ * bound: reads and writes each moved row once.
+ */
+PCTREE_API pctree_status pctree_compact(const pctree_compact_layout* layout,
+                                        const int32_t* accepted_idx,
+                                        const int32_t* accepted_len,
+                                        const int32_t* prefix_len, void* cache,
+                                        const void* hidden_in, void* hidden_out,
+                                        int32_t* status, void* stream);
+
 /* Human-readable name of a status code. */
 PCTREE_API const char* pctree_status_string(int32_t status);
 

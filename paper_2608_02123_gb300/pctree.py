@@ -41,6 +41,18 @@ class Config(ctypes.Structure):
                 ("weight_dtype", ctypes.c_int32), ("mode", ctypes.c_int32)]
 
 
+class CompactLayout(ctypes.Structure):
+    """pctree_compact_layout: shapes and byte strides of the cache planes."""
+    _fields_ = [("batch", ctypes.c_int32), ("B", ctypes.c_int32),
+                ("N", ctypes.c_int32), ("layers", ctypes.c_int32),
+                ("planes", ctypes.c_int32), ("max_slots", ctypes.c_int32),
+                ("row_bytes", ctypes.c_int64), ("slot_stride", ctypes.c_int64),
+                ("request_stride", ctypes.c_int64),
+                ("plane_stride", ctypes.c_int64),
+                ("layer_stride", ctypes.c_int64),
+                ("hidden_bytes", ctypes.c_int64)]
+
+
 class _Tree(ctypes.Structure):
     _fields_ = [(name, ctypes.c_void_p) for name in (
         "n_nodes", "tokens", "parent", "depth", "logp", "position_ids",
@@ -70,6 +82,9 @@ def _load() -> ctypes.CDLL:
     lib.pctree_accept.argtypes = [cfgp, ctypes.POINTER(_Tree), vp, vp, vp, vp,
                                   vp]
     lib.pctree_accept.restype = ctypes.c_int
+    lib.pctree_compact.argtypes = [ctypes.POINTER(CompactLayout), vp, vp, vp,
+                                   vp, vp, vp, vp, vp]
+    lib.pctree_compact.restype = ctypes.c_int
     lib.pctree_status_string.argtypes = [ctypes.c_int32]
     lib.pctree_status_string.restype = ctypes.c_char_p
     lib.pctree_profile_enable.argtypes = [ctypes.c_int32]
@@ -231,6 +246,38 @@ def pctree_accept(cfg: Config, tree: Tree, target_tokens: torch.Tensor,
                            _stream_ptr(stream))
     if rc != PCTREE_OK:
         raise PctreeError(rc, "pctree_accept")
+
+
+def compact_layout(batch: int, B: int, N: int, layers: int, planes: int,
+                   max_slots: int, row_bytes: int, hidden_bytes: int = 0,
+                   slot_stride: Optional[int] = None,
+                   request_stride: Optional[int] = None,
+                   plane_stride: Optional[int] = None,
+                   layer_stride: Optional[int] = None) -> CompactLayout:
+    """Layout of caches shaped ``[layers][planes][batch][max_slots][row]``
+    unless strides (bytes) are given."""
+    ss = row_bytes if slot_stride is None else slot_stride
+    rs = ss * max_slots if request_stride is None else request_stride
+    ps = rs * batch if plane_stride is None else plane_stride
+    ls = ps * planes if layer_stride is None else layer_stride
+    return CompactLayout(batch, B, N, layers, planes, max_slots, row_bytes,
+                         ss, rs, ps, ls, hidden_bytes)
+
+
+def pctree_compact(layout: CompactLayout, accepted_idx: torch.Tensor,
+                   accepted_len: torch.Tensor, prefix_len: torch.Tensor,
+                   cache: Optional[torch.Tensor],
+                   hidden_in: Optional[torch.Tensor] = None,
+                   hidden_out: Optional[torch.Tensor] = None,
+                   status: Optional[torch.Tensor] = None,
+                   stream: Optional[torch.cuda.Stream] = None) -> None:
+    """Enqueue the accepted-row compaction (see pctree_compact)."""
+    rc = LIB.pctree_compact(ctypes.byref(layout), accepted_idx.data_ptr(),
+                            accepted_len.data_ptr(), prefix_len.data_ptr(),
+                            _ptr(cache), _ptr(hidden_in), _ptr(hidden_out),
+                            _ptr(status), _stream_ptr(stream))
+    if rc != PCTREE_OK:
+        raise PctreeError(rc, "pctree_compact")
 
 
 def pctree_profile_enable(on: bool) -> None:

@@ -93,3 +93,32 @@ def test_status_strings(P):
     assert P.pctree_status_string(0) == "ok"
     assert "timed out" in P.pctree_status_string(-4)
     assert P.pctree_version() >= 100
+
+
+def test_compact_rejects_bad_layouts_on_the_host(P):
+    lib, fake = P.LIB, 4096
+    good = P.compact_layout(2, 5, 16, 3, 2, 40, 64, hidden_bytes=96)
+
+    def call(lay, cache=fake, hin=fake, hout=fake * 64, acc=fake):
+        return lib.pctree_compact(ctypes.byref(lay), acc, fake, fake, cache,
+                                  hin, hout, None, None)
+
+    def variant(**kw):
+        f = {n: getattr(good, n) for n, _ in P.CompactLayout._fields_}
+        f.update(kw)
+        return P.CompactLayout(**f)
+
+    assert call(good, acc=None) == -1
+    assert call(good, cache=None) == -1
+    assert call(good, cache=fake + 8) == -1                 # misaligned
+    assert call(good, hin=None) == -1
+    assert call(good, hout=fake + 64) == -1                 # overlaps hidden_in
+    for kw in [dict(batch=0), dict(B=0), dict(N=0), dict(max_slots=15),
+               dict(row_bytes=8), dict(row_bytes=72), dict(slot_stride=48),
+               dict(request_stride=40), dict(plane_stride=-16),
+               dict(layer_stride=8), dict(hidden_bytes=20),
+               dict(layers=-1)]:
+        assert call(variant(**kw)) == -1, kw
+    # nothing to move: no planes and no hidden states
+    assert call(variant(layers=0, hidden_bytes=0), cache=None, hin=None,
+                hout=None) == 0
