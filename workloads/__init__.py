@@ -352,3 +352,119 @@ def draw_compaction(cw: CompactWorkload, seed: Optional[int] = None,
         hid_out = g.integers(0, 256, size=(cw.batch, cw.B + 1, cw.hidden_bytes),
                              dtype=np.uint8)
     return CompactInputs(cw, acc, lens, prefix, cache, hid_in, hid_out)
+
+
+# ----------------------------------------------------------------------------
+# tree-verification attention inputs (one target layer)
+# ----------------------------------------------------------------------------
+
+@dataclasses.dataclass(frozen=True)
+class AttnWorkload:
+    """One attention layer of the target's tree-verification forward:
+    ``Hq`` query heads sharing ``Hkv`` KV heads of size ``D``; ``N`` tree
+    nodes of depth at most ``B`` after a prefix of up to ``prefix_max``."""
+
+    name: str
+    batch: int
+    N: int
+    Hq: int
+    Hkv: int
+    D: int
+    B: int
+    prefix_max: int
+    seed: int
+    q_scale: float = 1.5
+    k_scale: float = 1.5
+
+    @property
+    def slots(self) -> int:
+        return self.prefix_max + self.N
+
+
+ATTN_WORKLOADS: Dict[str, AttnWorkload] = {
+    "small": AttnWorkload("small_bs2_N16_Hq8_Hkv2", batch=2, N=16, Hq=8,
+                          Hkv=2, D=128, B=5, prefix_max=200, seed=40),
+    "ragged": AttnWorkload("ragged_bs3_N24_Hq10_Hkv2", batch=3, N=24, Hq=10,
+                           Hkv=2, D=128, B=7, prefix_max=70, seed=41),
+    # Qwen3 attention shapes: 32 query / 8 KV heads (4B, 8B), 40 / 8 (14B),
+    # head_dim 128; the trees of the drafting workloads
+    "4b_b16": AttnWorkload("qwen3_4b_Hq32_Hkv8_D128_N64_B16_bs1", batch=1,
+                           N=64, Hq=32, Hkv=8, D=128, B=16, prefix_max=2048,
+                           seed=42),
+    "8b_b7_bs16": AttnWorkload("qwen3_8b_Hq32_Hkv8_D128_N64_B7_bs16",
+                               batch=16, N=64, Hq=32, Hkv=8, D=128, B=7,
+                               prefix_max=1024, seed=43),
+    "14b_b16_bs32": AttnWorkload("qwen3_14b_Hq40_Hkv8_D128_N128_B16_bs32",
+                                 batch=32, N=128, Hq=40, Hkv=8, D=128, B=16,
+                                 prefix_max=1024, seed=44),
+}
+
+
+@dataclasses.dataclass
+class AttnInputs:
+    aw: AttnWorkload
+    q: np.ndarray            # bf16 bits [batch][N][Hq][D]
+    k: np.ndarray            # bf16 bits [batch][slots][Hkv][D]
+    v: np.ndarray            # bf16 bits [batch][slots][Hkv][D]
+    prefix_len: np.ndarray   # [batch] int32
+    n_nodes: np.ndarray      # [batch] int32
+    parent: np.ndarray       # [batch][N] int32, -1 at the root and padding
+
+
+def draw_tree_parents(N: int, B: int, rng: np.random.Generator):
+    """A random tree in breadth-first packed order: node 0 is the root,
+    every other node's parent is an earlier node of depth < B, picked with
+    weight favouring shallow nodes (bushy near the root, like budgeted
+    drafting trees).  Returns ``(n_nodes, parent [N])``."""
+    n = int(rng.integers(max(1, N // 2), N + 1))
+    parent = np.full(N, -1, dtype=np.int32)
+    depth = np.zeros(N, dtype=np.int64)
+    for i in range(1, n):
+        cand = np.flatnonzero(depth[:i] < B)
+        w = 1.0 / (1.0 + depth[cand]) ** 2
+        p = int(rng.choice(cand, p=w / w.sum()))
+        parent[i] = p
+        depth[i] = depth[p] + 1
+    # breadth-first packing: parents before children, depth non-decreasing
+    order = sorted(range(n), key=lambda i: (depth[i], i))
+    pos = {old: new for new, old in enumerate(order)}
+    out = np.full(N, -1, dtype=np.int32)
+    for old in order[1:]:
+        out[pos[old]] = pos[int(parent[old])]
+    return n, out
+
+
+def draw_attention(aw: AttnWorkload, seed: Optional[int] = None,
+                   fill: bool = True) -> AttnInputs:
+    """Seeded inputs of one tree-verification attention layer.  Request 0
+    has the longest prefix allowed, request 1 (if any) an empty one; Q, K,
+    V are normal with the workload's scales, rounded to bf16; cache slots
+    past a request's tree hold random values too (they must be ignored)."""
+    ss = np.random.SeedSequence(aw.seed if seed is None else seed)
+    s_tree, s_q, s_k, s_v = ss.spawn(4)
+    rng = np.random.default_rng(s_tree)
+    prefix = rng.integers(0, aw.prefix_max + 1, size=aw.batch).astype(np.int32)
+    prefix[0] = aw.prefix_max
+    if aw.batch > 1:
+        prefix[1] = 0
+    n_nodes = np.zeros(aw.batch, dtype=np.int32)
+    parent = np.full((aw.batch, aw.N), -1, dtype=np.int32)
+    for r in range(aw.batch):           # request 0 fills the node budget
+        draw = _full_tree if r == 0 else draw_tree_parents
+        n_nodes[r], parent[r] = draw(aw.N, aw.B, rng)
+    q = k = v = None
+    if fill:
+        def normal(seq, shape, scale):
+            rows = int(np.prod(shape[:-1]))
+            return _draw_matrix(seq, rows, shape[-1], scale, "bf16").reshape(shape)
+        q = normal(s_q, (aw.batch, aw.N, aw.Hq, aw.D), aw.q_scale)
+        k = normal(s_k, (aw.batch, aw.slots, aw.Hkv, aw.D), aw.k_scale)
+        v = normal(s_v, (aw.batch, aw.slots, aw.Hkv, aw.D), 1.0)
+    return AttnInputs(aw, q, k, v, prefix, n_nodes, parent)
+
+
+def _full_tree(N: int, B: int, rng: np.random.Generator):
+    while True:
+        n, par = draw_tree_parents(N, B, rng)
+        if n == N:
+            return n, par
