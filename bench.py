@@ -30,8 +30,9 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
-from workloads import (COMPACT_WORKLOADS, WORKLOADS, draw_compaction,  # noqa: E402
-                       draw_head, draw_request)
+from workloads import (ATTN_WORKLOADS, COMPACT_WORKLOADS, WORKLOADS,  # noqa: E402
+                       draw_attention, draw_compaction, draw_head,
+                       draw_request)
 
 METRIC = ("tree-draft rounds/sec & µs/round (V=151936, B=16, N=64); "
           "% of HBM roofline")
@@ -54,12 +55,17 @@ def parse_args():
                     help="k/N sweep (B in {7,16}, k in {1,2,4,8}, N in "
                          "{8..128}) on the workload's shapes, batch 1: one "
                          "JSON line per point instead of the benchmark line")
-    ap.add_argument("--op", default="round", choices=["round", "compact"],
+    ap.add_argument("--op", default="round",
+                    choices=["round", "compact", "attention"],
                     help="round: the drafting round (the benchmark line); "
                          "compact: the accepted-row KV/hidden-state compaction "
-                         "after acceptance, on --compact-workload")
+                         "after acceptance, on --compact-workload; attention: "
+                         "one tree-verification attention layer, on "
+                         "--attn-workload")
     ap.add_argument("--compact-workload", default="14b_b16_bs32",
                     choices=sorted(COMPACT_WORKLOADS))
+    ap.add_argument("--attn-workload", default="14b_b16_bs32",
+                    choices=sorted(ATTN_WORKLOADS))
     ap.add_argument("--path", default="auto", choices=["auto", "stagewise"],
                     help="kernel path: fused round where it applies, or the "
                          "per-stage kernels for every round")
@@ -590,9 +596,111 @@ def run_compact(args, local_rank):
         "gpu_launches": args.steps, "clocks": clk}), flush=True)
 
 
+def attention_work(ai):
+    """Algorithmic bytes and flops of one tree-attention layer: K and V of
+    every request's prefix and tree read once per KV head, Q read and the
+    output written once; 4 * D flops per (node, query head, allowed key)
+    pair (the scores and the weighted sum)."""
+    aw = ai.aw
+    nbytes, flops = 0, 0
+    for r in range(aw.batch):
+        T, n = int(ai.prefix_len[r]), int(ai.n_nodes[r])
+        nbytes += (T + n) * aw.Hkv * aw.D * 2 * 2
+        nbytes += n * aw.Hq * aw.D * 2 * 2
+        depth = np.zeros(aw.N, dtype=np.int64)
+        for i in range(1, n):
+            depth[i] = depth[ai.parent[r, i]] + 1
+        keys = T + depth[:n] + 1
+        flops += int(keys.sum()) * aw.Hq * 4 * aw.D
+    return nbytes, flops
+
+
+def run_attention(args, local_rank):
+    """One tree-verification attention layer (the target's forward that
+    verifies the packed tree) on one GPU: the workload's caches resident in
+    HBM, rotated over enough copies that a launch's K/V were last read more
+    than 3 x L2 earlier."""
+    import torch
+
+    from paper_2608_02123_gb300 import pctree as P
+
+    aw = ATTN_WORKLOADS[args.attn_workload]
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    ai = draw_attention(aw)
+
+    def up(bits):
+        return torch.from_numpy(bits.view(np.int16)).to(dev).view(torch.bfloat16)
+
+    q, k, v = up(ai.q), up(ai.k), up(ai.v)
+    kv_bytes = 2 * k.numel() * 2
+    n_sets = max(1, min(64, -(-3 * L2_BYTES // kv_bytes)))
+    ks = [k] + [k.clone() for _ in range(n_sets - 1)]
+    vs = [v] + [v.clone() for _ in range(n_sets - 1)]
+    pre = torch.from_numpy(ai.prefix_len).to(dev)
+    nn = torch.from_numpy(ai.n_nodes).to(dev)
+    par = torch.from_numpy(ai.parent).to(dev)
+    out = torch.empty_like(q)
+    cfg = P.attn_config(aw.batch, aw.N, aw.Hq, aw.Hkv, aw.slots)
+    nb = P.pctree_tree_attention_workspace_bytes(cfg)
+    ws = torch.empty(max(nb, 1), dtype=torch.uint8, device=dev) if nb else None
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(i):
+        P.pctree_tree_attention(cfg, q, ks[i % n_sets], vs[i % n_sets], pre, nn,
+                                par, out, ws, status, stream)
+
+    for i in range(max(args.warmup, 3)):
+        step(i)
+    torch.cuda.synchronize()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    start.record(stream)
+    for i in range(args.steps):
+        step(i)
+    end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if int(status.item()) != 0:
+        raise RuntimeError(f"pctree_tree_attention status {int(status.item())}")
+    ms = start.elapsed_time(end) / args.steps
+    nbytes, flops = attention_work(ai)
+    peaks, src = measured_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    tc = float(peaks.get("bf16_tflops", 1900.0))
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    tfs = flops / (ms * 1e-3) / 1e12
+    bound = "hbm" if nbytes / hbm / 1e9 >= flops / tc / 1e12 else "tensor"
+    roof = ({"bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s",
+             "frac": gbs / hbm} if bound == "hbm" else
+            {"bound": "tensor", "achieved": tfs, "peak": tc, "unit": "TFLOP/s",
+             "frac": tfs / tc})
+    roof.update({"kernel": "tree_attn_kernel", "peak_source": src,
+                 "traffic": None, "other": {"GB/s": gbs, "hbm_frac": gbs / hbm,
+                                            "TFLOP/s": tfs, "tensor_frac": tfs / tc}})
+    print(json.dumps({
+        "metric": "tree-verification attention µs/layer (prefix + ancestors, GQA)",
+        "value": ms * 1e3, "unit": "us/layer", "higher_is_better": False,
+        "n_gpus": 1, "steps": args.steps, "warmup": max(args.warmup, 3),
+        "dtype": "bf16", "data": "synthetic (seeded Q/K/V, random breadth-first trees)",
+        "config": {"workload": aw.name, "batch": aw.batch, "N": aw.N,
+                   "Hq": aw.Hq, "Hkv": aw.Hkv, "D": aw.D,
+                   "prefix_max": aw.prefix_max,
+                   "mean_prefix": float(ai.prefix_len.mean()),
+                   "l2": f"K/V rotated over {n_sets} copies (>= 3x L2)"},
+        "bytes_per_layer": nbytes, "flops_per_layer": flops,
+        "roofline": roof, "gpu_launches": args.steps, "clocks": clk}), flush=True)
+
+
 def main():
     args = parse_args()
     wl = WORKLOADS[args.workload].with_(mode=args.mode)
+    if args.op == "attention":
+        run_attention(args, int(os.environ.get("LOCAL_RANK", "0")))
+        return
     if args.op == "compact":
         run_compact(args, int(os.environ.get("LOCAL_RANK", "0")))
         return

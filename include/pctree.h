@@ -299,6 +299,61 @@ PCTREE_API pctree_status pctree_compact(const pctree_compact_layout* layout,
                                         const void* hidden_in, void* hidden_out,
                                         int32_t* status, void* stream);
 
+/*
+ * Tree-verification attention (Sec. 4.2: the packed tree is verified in one
+ * target forward; Appendix A "Tensor implementation": a node attends to the
+ * verified prefix, itself and its root-to-node ancestors).  One
+ * grouped-query attention layer of that forward, for a batch of requests:
+ *
+ *   for node i < n_nodes[r] and query head h (KV head h / G, G = Hq / Hkv):
+ *     keys  = slots 0 .. T-1 (T = prefix_len[r]) and the slots T + m of the
+ *             nodes m on the path from i to the root (i included)
+ *     out[r][i][h] = softmax_j(scale * <q[r][i][h], k[r][j][h/G]>) . v[r][j][h/G]
+ *   rows i >= n_nodes[r] are 0.
+ *
+ * The ancestor sets come from the packed parent indices (parent[i] < i,
+ * -1 at the root), the same tree pctree_draft writes (its `parent`
+ * output); they equal the rows of its ancestor mask.  Rotary embeddings
+ * (positions depth + T) are applied to q and k by the caller.
+ *
+ * Layouts, all bf16 and dense:
+ *   q, out       [batch][N][Hq][D]
+ *   k_cache,
+ *   v_cache      [batch][max_slots][Hkv][D], node i of the tree at slot T + i
+ * Limits: D = 128, Hq a multiple of Hkv, Hq / Hkv <= 128,
+ * N <= PCTREE_ATTN_MAX_N.  Cache slots past T + n_nodes are never used
+ * (their values may be anything).
+ */
+#define PCTREE_ATTN_MAX_N 256
+
+typedef struct {
+  int32_t batch, N, Hq, Hkv, D;
+  int32_t max_slots;     /* slots per request in the caches, >= N         */
+  float scale;           /* softmax scale, e.g. 1/sqrt(D)                  */
+} pctree_attn_config;
+
+/* Workspace bytes pctree_tree_attention needs (0 when a request's keys are
+ * never split over several CTAs); 256-byte aligned, any prior content. */
+PCTREE_API size_t pctree_tree_attention_workspace_bytes(const pctree_attn_config* cfg);
+
+/*
+ *   prefix_len, n_nodes  [batch] int32 (device)
+ *   parent               [batch][N] int32 (device)
+ *   status               one device int32 or NULL: set to
+ *                        PCTREE_ERR_INVALID_ARG for a request with T < 0,
+ *                        n_nodes outside [0, N] or T + n_nodes > max_slots
+ *                        (its rows are 0), PCTREE_ERR_TIMEOUT if a bounded
+ *                        wait ran out; otherwise not written.
+ * Pointers 16-byte aligned.  Returns PCTREE_ERR_INVALID_ARG /
+ * PCTREE_ERR_UNSUPPORTED / PCTREE_ERR_WORKSPACE for bad arguments (nothing
+ * enqueued) and PCTREE_ERR_CUDA if the launch fails.
+ */
+PCTREE_API pctree_status pctree_tree_attention(
+    const pctree_attn_config* cfg, const void* q, const void* k_cache,
+    const void* v_cache, const int32_t* prefix_len, const int32_t* n_nodes,
+    const int32_t* parent, void* out, void* workspace, size_t workspace_bytes,
+    int32_t* status, void* stream);
+
 /* Human-readable name of a status code. */
 PCTREE_API const char* pctree_status_string(int32_t status);
 

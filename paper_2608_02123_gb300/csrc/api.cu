@@ -81,8 +81,11 @@ Layout make_layout(const pctree_config& c) {
   return l;
 }
 
+}  // namespace
+
 // --------------------------------------------------------------------------
-// per-device facts and the driver's tensor-map encoder
+// per-device facts and the driver's tensor-map encoder (shared with the
+// other translation units through pctree_common.cuh)
 // --------------------------------------------------------------------------
 
 using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
@@ -120,6 +123,30 @@ pctree_status device_facts(int* num_sms) {
   *num_sms = g_num_sms[dev];
   return PCTREE_OK;
 }
+
+pctree_status encode_bf16_map_nd(CUtensorMap* map, const void* base, int rank,
+                                 const uint64_t* dims,
+                                 const uint64_t* strides_bytes,
+                                 const uint32_t* box) {
+  if (g_encode == nullptr || rank < 1 || rank > 5) return PCTREE_ERR_CUDA;
+  cuuint64_t d[5], st[4];
+  cuuint32_t b[5], e[5];
+  for (int i = 0; i < rank; ++i) {
+    d[i] = dims[i];
+    b[i] = box[i];
+    e[i] = 1;
+    if (i + 1 < rank) st[i] = strides_bytes[i];
+  }
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank,
+                        const_cast<void*>(base), d, st, b, e,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? PCTREE_OK : PCTREE_ERR_INVALID_ARG;
+}
+
+namespace {
 
 // 2-D bf16 tensor [rows][cols] (cols contiguous), box = box_rows x 64 with
 // the 128-byte swizzle the MMA descriptors expect.

@@ -240,6 +240,18 @@ __device__ __forceinline__ void set_status(int32_t* status, int code) {
 // Z[row][v] = L[req(row)][v] + sum_h W_out[v][h] X[row][h] for rows
 // [0, rows), req(row) = row / rows_per_req.  `L` points at depth d of
 // request 0; requests are `l_req_stride` floats apart.
+// SM count of the current device and the driver's tensor-map encoder, looked
+// up once per device (api.cu).
+pctree_status device_facts(int* num_sms);
+
+// bf16 tensor map of rank 1..5 with the 128-byte swizzle (innermost box
+// dimension 64 elements = 128 bytes); dims innermost first, strides_bytes for
+// dimensions 1..rank-1.  Requires a prior successful device_facts call.
+pctree_status encode_bf16_map_nd(CUtensorMap* map, const void* base, int rank,
+                                 const uint64_t* dims,
+                                 const uint64_t* strides_bytes,
+                                 const uint32_t* box);
+
 cudaError_t launch_markov_bf16(const CUtensorMap* tmap_w,
                                const CUtensorMap* tmap_x, const float* L,
                                long long l_req_stride, float* Z, int ldz,

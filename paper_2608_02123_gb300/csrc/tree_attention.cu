@@ -1,0 +1,637 @@
+// pctree_tree_attention: one grouped-query attention layer of the target's
+// tree-verification forward (Sec. 4.2; Appendix A "Tensor implementation"):
+// every drafted node attends to the verified prefix, itself and its
+// root-to-node ancestors.
+//
+// Work unit (one CTA): request r, KV head h, a tile of query rows and a range
+// of 128-key blocks.  The tile's rows are (node, query head of the group)
+// pairs, node-major: row t = node_local * G + g, R = G * nodes_per_tile <= 128.
+// The G query heads sharing KV head h read the same K/V blocks once.
+//
+//   warp 0      TMA producer: the Q tile once, then K and V blocks (128 keys
+//               x 128 dims, two 64-dim halves each, 128-byte swizzle) into a
+//               two-stage ring
+//   warp 1      tcgen05.mma issuer: S_b = Q K_b^T into one of two TMEM
+//               buffers (M=128, N=128 keys, K=128 dims), then O_b = P_b V_b
+//               into a third (M=128, N=128 dims, K=128 keys; V is the
+//               MN-major operand, dims contiguous)
+//   warps 2..5  softmax, one thread per TMEM lane = tile row: masked running
+//               max, P = 2^(s - m) rounded to bf16 into shared memory (the
+//               K-major A operand of the second MMA), and the running output
+//               O = O * 2^(m_old - m_new) + O_b kept in registers
+//
+// S of block b+1 is computed while the softmax works on block b and the PV
+// product of block b runs while the softmax folds block b-1.  Key blocks of
+// a request may be split over several CTAs; each writes (max, sum, O) of its
+// rows and the last CTA of the unit (an atomic ticket, no waiting) merges
+// them.  All waits are bounded (1 s) and end in PCTREE_ERR_TIMEOUT.
+#include <cuda_bf16.h>
+
+#include "pctree_common.cuh"
+#include "sm103_ptx.cuh"
+
+namespace pct {
+namespace {
+
+constexpr int kAttnThreads = 192;
+constexpr int kBK = 128;                  // keys per block
+constexpr int kHalfBytes = 128 * 128;     // 128 rows x 64 bf16 (one dim half)
+constexpr int kQOff = 0;
+constexpr int kKVOff = 2 * kHalfBytes;    // stage s: K at +s*64K, V at +32K
+constexpr int kPOff = kKVOff + 2 * 4 * kHalfBytes;
+constexpr int kTailOff = kPOff + 2 * kHalfBytes;
+constexpr int kMaskWords = PCTREE_ATTN_MAX_N / 32;
+constexpr uint64_t kAttnLimitNs = 1000000000ull;
+
+struct AttnTail {
+  uint64_t q_full;
+  uint64_t kv_full[2], kv_empty[2];
+  uint64_t s_full[2], s_empty[2];
+  uint64_t p_full, p_empty, o_full, o_empty, done;
+  uint32_t tmem_base;
+  int abort;
+  int last;
+  uint32_t anc[128][kMaskWords];          // ancestor-or-self bits per node
+};
+
+constexpr size_t kAttnSmem = kTailOff + sizeof(AttnTail) + 1024;
+
+struct AttnArgs {
+  const int32_t* prefix;
+  const int32_t* n_nodes;
+  const int32_t* parent;
+  uint16_t* out;          // bf16 [batch][N][Hq][128]
+  float* part_o;          // [unit][split][128][128]
+  float2* part_ml;        // [unit][split][128]  (max in log2 units, sum)
+  int* ticket;            // [unit]
+  int32_t* status;
+  int batch, N, Hq, Hkv, G, npt, R, nqt, max_slots, n_split, bps;
+  float scale_log2;       // softmax scale * log2(e)
+};
+
+__device__ __forceinline__ uint8_t* kv_k(uint8_t* sm, int s) {
+  return sm + kKVOff + s * 4 * kHalfBytes;
+}
+__device__ __forceinline__ uint8_t* kv_v(uint8_t* sm, int s) {
+  return sm + kKVOff + s * 4 * kHalfBytes + 2 * kHalfBytes;
+}
+
+// Records the first error in the optional status word.
+__device__ __forceinline__ void report(int32_t* status, int code) {
+  if (status != nullptr) atomicCAS(status, 0, code);
+}
+
+// Allowed-key bits of 32 consecutive slots kc0 .. kc0+31 for a row whose
+// node has ancestor-or-self bits `anc`: the whole prefix (slots < T) and
+// the tree slots T + m of its ancestors (the bits are 0 past the tree).
+__device__ __forceinline__ uint32_t allowed_bits(int kc0, int T,
+                                                 const uint32_t* anc) {
+  uint32_t bits = 0;
+  const int pm = T - kc0;                       // prefix slots in the chunk
+  if (pm >= 32) return 0xffffffffu;
+  if (pm > 0) bits = (1u << pm) - 1u;
+  const int m0 = kc0 - T;                       // tree index of slot kc0
+  if (m0 >= 0) {
+    const int w = m0 >> 5, sh = m0 & 31;
+    uint32_t lo = w < kMaskWords ? anc[w] : 0u;
+    uint32_t hi = (w + 1) < kMaskWords ? anc[w + 1] : 0u;
+    bits |= sh == 0 ? lo : ((lo >> sh) | (hi << (32 - sh)));
+  } else if (m0 > -32) {
+    bits |= anc[0] << (-m0);
+  }
+  return bits;
+}
+
+__global__ void __launch_bounds__(kAttnThreads, 1)
+tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
+                 const __grid_constant__ CUtensorMap tm_k,
+                 const __grid_constant__ CUtensorMap tm_v, AttnArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  AttnTail* T = reinterpret_cast<AttnTail*>(sm + kTailOff);
+  uint8_t* sq = sm + kQOff;
+  uint8_t* sp = sm + kPOff;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qt = blockIdx.x % a.nqt, split = blockIdx.x / a.nqt;
+  const int kvh = blockIdx.y, r = blockIdx.z;
+
+  // request facts; a request with an impossible prefix or tree size is
+  // reported and produces zero rows
+  int Tp = a.prefix[r], n = a.n_nodes[r];
+  if (Tp < 0 || n < 0 || n > a.N || static_cast<long long>(Tp) + n > a.max_slots) {
+    if (threadIdx.x == 0 && split == 0 && qt == 0 && kvh == 0)
+      report(a.status, PCTREE_ERR_INVALID_ARG);
+    Tp = 0;
+    n = 0;
+  }
+  const int n_keys = n > 0 ? Tp + n : 0;        // no queries: nothing to do
+  const int nb_r = (n_keys + kBK - 1) / kBK;
+  const int kb0 = split * a.bps;
+  const int nblk = max(0, min(kb0 + a.bps, nb_r) - kb0);
+
+  if (threadIdx.x == 0) {
+    mbar_init(&T->q_full, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&T->kv_full[s], 1);
+      mbar_init(&T->kv_empty[s], 1);
+      mbar_init(&T->s_full[s], 1);
+      mbar_init(&T->s_empty[s], 4);
+    }
+    mbar_init(&T->p_full, 4);
+    mbar_init(&T->p_empty, 1);
+    mbar_init(&T->o_full, 1);
+    mbar_init(&T->o_empty, 4);
+    mbar_init(&T->done, 1);
+    T->abort = 0;
+    fence_barrier_init();
+  }
+  // rows R..127 of the Q tile are not loaded: zero them (read by the MMA)
+  for (int i = threadIdx.x; i < 2 * (128 - a.R) * 8; i += blockDim.x) {
+    const int half = i / ((128 - a.R) * 8), rem = i % ((128 - a.R) * 8);
+    *reinterpret_cast<uint4*>(sq + half * kHalfBytes + (a.R + rem / 8) * 128 +
+                              (rem % 8) * 16) = make_uint4(0, 0, 0, 0);
+  }
+  // ancestor-or-self bits of the tile's nodes (walk up the packed parents)
+  for (int nl = threadIdx.x; nl < a.npt; nl += blockDim.x) {
+    uint32_t bits[kMaskWords];
+#pragma unroll
+    for (int w = 0; w < kMaskWords; ++w) bits[w] = 0u;
+    int x = qt * a.npt + nl;
+    if (x < n) {
+      const int32_t* par = a.parent + static_cast<size_t>(r) * a.N;
+      for (int steps = 0; steps <= n && x >= 0 && x < n; ++steps) {
+#pragma unroll
+        for (int w = 0; w < kMaskWords; ++w)
+          if ((x >> 5) == w) bits[w] |= 1u << (x & 31);
+        const int px = par[x];
+        x = px < x ? px : -1;          // parents precede children
+      }
+    }
+#pragma unroll
+    for (int w = 0; w < kMaskWords; ++w) T->anc[nl][w] = bits[w];
+  }
+  fence_proxy_async_smem();
+  if (warp == 1) tmem_alloc(&T->tmem_base, 512);
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  const uint32_t tmem = T->tmem_base;
+  volatile int* abort_v = &T->abort;
+
+  if (warp == 0 && lane == 0 && nblk > 0) {
+    // ---------------- TMA producer ----------------
+    tma_prefetch_desc(&tm_q);
+    tma_prefetch_desc(&tm_k);
+    tma_prefetch_desc(&tm_v);
+    mbar_arrive_expect_tx(&T->q_full, 2u * static_cast<uint32_t>(a.R) * 128u);
+    tma_load_4d(sq, &tm_q, &T->q_full, 0, kvh * a.G, qt * a.npt, r);
+    tma_load_4d(sq + kHalfBytes, &tm_q, &T->q_full, 64, kvh * a.G, qt * a.npt, r);
+    int issued = 0;
+    for (int b = 0; b < nblk; ++b) {
+      const int s = b & 1;
+      if (b >= 2 && !mbar_wait_bounded(&T->kv_empty[s], ((b >> 1) - 1) & 1,
+                                       abort_v, kAttnLimitNs)) {
+        *abort_v = 1;
+        break;
+      }
+      const int key0 = (kb0 + b) * kBK;
+      mbar_arrive_expect_tx(&T->kv_full[s], 4u * kHalfBytes);
+      tma_load_4d(kv_k(sm, s), &tm_k, &T->kv_full[s], 0, kvh, key0, r);
+      tma_load_4d(kv_k(sm, s) + kHalfBytes, &tm_k, &T->kv_full[s], 64, kvh, key0, r);
+      tma_load_4d(kv_v(sm, s), &tm_v, &T->kv_full[s], 0, kvh, key0, r);
+      tma_load_4d(kv_v(sm, s) + kHalfBytes, &tm_v, &T->kv_full[s], 64, kvh, key0, r);
+      ++issued;
+    }
+    // copies still in flight land before the CTA may exit
+    (void)mbar_wait_bounded(&T->q_full, 0, abort_v, kAttnLimitNs);
+    for (int b = issued - 2 > 0 ? issued - 2 : 0; b < issued; ++b)
+      (void)mbar_wait_bounded(&T->kv_full[b & 1], (b >> 1) & 1, abort_v, kAttnLimitNs);
+  } else if (warp == 1 && lane == 0 && nblk > 0) {
+    // ---------------- MMA issuer ----------------
+    constexpr uint32_t idS = idesc_bf16_f32(128, 128);
+    constexpr uint32_t idO = idesc_bf16_f32_bmn(128, 128);
+    bool ok = mbar_wait_bounded(&T->q_full, 0, abort_v, kAttnLimitNs);
+    const uint32_t q0 = smem_u32(sq), p0 = smem_u32(sp);
+    auto issue_s = [&](int b) -> bool {
+      const int s = b & 1;
+      if (!mbar_wait_bounded(&T->kv_full[s], (b >> 1) & 1, abort_v, kAttnLimitNs))
+        return false;
+      if (b >= 2 && !mbar_wait_bounded(&T->s_empty[s], ((b >> 1) - 1) & 1, abort_v,
+                                       kAttnLimitNs))
+        return false;
+      tc_fence_after_sync();
+      const uint32_t k0 = smem_u32(kv_k(sm, s));
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint32_t off = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
+        tc_mma_bf16(tmem + s * 128, desc_kmajor_sw128(q0 + off),
+                    desc_kmajor_sw128(k0 + off), idS, kk > 0 ? 1u : 0u);
+      }
+      tc_commit(&T->s_full[s]);
+      return true;
+    };
+    auto issue_o = [&](int b) -> bool {
+      const int s = b & 1;
+      if (!mbar_wait_bounded(&T->p_full, b & 1, abort_v, kAttnLimitNs)) return false;
+      if (b >= 1 && !mbar_wait_bounded(&T->o_empty, (b - 1) & 1, abort_v, kAttnLimitNs))
+        return false;
+      tc_fence_after_sync();
+      const uint32_t v0 = smem_u32(kv_v(sm, s));
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint32_t aoff = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
+        // 16 keys = 16 rows of 128 B; the dims 64..127 half is kHalfBytes on
+        tc_mma_bf16(tmem + 256, desc_kmajor_sw128(p0 + aoff),
+                    desc_mnmajor_sw128(v0 + kk * 16 * 128, kHalfBytes, 1024), idO,
+                    kk > 0 ? 1u : 0u);
+      }
+      tc_commit(&T->o_full);
+      tc_commit(&T->kv_empty[s]);
+      tc_commit(&T->p_empty);
+      return true;
+    };
+    if (ok) ok = issue_s(0);
+    for (int b = 1; ok && b < nblk; ++b) ok = issue_s(b) && issue_o(b - 1);
+    if (ok) ok = issue_o(nblk - 1);
+    if (!ok) {
+      *abort_v = 1;
+      report(a.status, PCTREE_ERR_TIMEOUT);
+    }
+    tc_commit(&T->done);               // every MMA issued above has finished
+    (void)mbar_wait_bounded(&T->done, 0, abort_v, kAttnLimitNs);
+  }
+  else if (warp >= 2) {
+    // ---------------- softmax and output, one thread per tile row ----------
+    const int quad = warp & 3;               // TMEM lanes quad*32 .. +31
+    const int t = quad * 32 + lane;          // tile row
+    const int nl = t / a.G, g = t - nl * a.G;
+    const int node = qt * a.npt + nl;
+    const bool row_ok = t < a.R && node < n;
+    const uint32_t* anc = T->anc[nl < a.npt ? nl : 0];
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+    float o[128];
+#pragma unroll
+    for (int d = 0; d < 128; ++d) o[d] = 0.0f;
+    float m_ref = -INFINITY, l_ref = 0.0f;   // o and l_ref are relative to m_ref
+    float m_run = -INFINITY;                 // running max (log2 units)
+    float m_pend = -INFINITY, l_pend = 0.0f; // block whose PV product is pending
+    bool ok = true;
+    auto fold = [&](int b) -> bool {         // o += O_b (relative to m_pend)
+      if (!mbar_wait_bounded(&T->o_full, b & 1, abort_v, kAttnLimitNs)) return false;
+      tc_fence_after_sync();
+      const float alpha = m_ref == m_pend ? 1.0f : exp2f(m_ref - m_pend);
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        uint32_t y[16];
+        tmem_ld_32x32b_x16(lane_base + 256 + c * 16, y);
+        tmem_ld_wait();
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+          o[c * 16 + j] = fmaf(o[c * 16 + j], alpha, __uint_as_float(y[j]));
+      }
+      l_ref = fmaf(l_ref, alpha, l_pend);
+      m_ref = m_pend;
+      tc_fence_before_sync();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&T->o_empty);
+      return true;
+    };
+    for (int b = 0; ok && b < nblk; ++b) {
+      const int sb = b & 1;
+      const int key0 = (kb0 + b) * kBK;
+      if (!mbar_wait_bounded(&T->s_full[sb], (b >> 1) & 1, abort_v, kAttnLimitNs)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after_sync();
+      const uint32_t s_base = lane_base + sb * 128;
+      // pass 1: the block's largest allowed score
+      uint32_t allow[4];
+      float mx = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) allow[c] = row_ok ? allowed_bits(key0 + c * 32, Tp, anc) : 0u;
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        uint32_t x[16];
+        tmem_ld_32x32b_x16(s_base + c * 16, x);
+        tmem_ld_wait();
+        const uint32_t al = allow[c >> 1] >> ((c & 1) * 16);
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+          if ((al >> j) & 1u) mx = fmaxf(mx, __uint_as_float(x[j]) * a.scale_log2);
+      }
+      const float m_new = fmaxf(m_run, mx);
+      // the last block of the request: V rows past the tree hold whatever the
+      // cache held there; zero them so that 0 * (non-finite) cannot reach O
+      const int valid = n_keys - key0;
+      if (valid < kBK) {
+        if (!mbar_wait_bounded(&T->kv_full[sb], (b >> 1) & 1, abort_v, kAttnLimitNs)) {
+          ok = false;
+          break;
+        }
+        uint8_t* v = kv_v(sm, sb);
+        for (int i = t; i < 2 * (kBK - valid) * 8; i += 128) {
+          const int half = i / ((kBK - valid) * 8), rem = i % ((kBK - valid) * 8);
+          *reinterpret_cast<uint4*>(v + half * kHalfBytes + (valid + rem / 8) * 128 +
+                                    (rem % 8) * 16) = make_uint4(0, 0, 0, 0);
+        }
+      }
+      // pass 2: P = 2^(s - m_new) in bf16, into the A operand of the PV MMA
+      if (b >= 1 && !mbar_wait_bounded(&T->p_empty, (b - 1) & 1, abort_v, kAttnLimitNs)) {
+        ok = false;
+        break;
+      }
+      float lsum = 0.0f;
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        uint32_t x[16];
+        tmem_ld_32x32b_x16(s_base + c * 16, x);
+        tmem_ld_wait();
+        const uint32_t al = allow[c >> 1] >> ((c & 1) * 16);
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {          // 8 keys = one 16-byte chunk
+          uint32_t w[4];
+#pragma unroll
+          for (int h = 0; h < 4; ++h) {
+            const int j0 = q * 8 + h * 2;
+            float p0 = 0.0f, p1 = 0.0f;
+            if ((al >> j0) & 1u)
+              p0 = exp2f(__uint_as_float(x[j0]) * a.scale_log2 - m_new);
+            if ((al >> (j0 + 1)) & 1u)
+              p1 = exp2f(__uint_as_float(x[j0 + 1]) * a.scale_log2 - m_new);
+            const __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
+            lsum += __low2float(pb) + __high2float(pb);
+            w[h] = *reinterpret_cast<const uint32_t*>(&pb);
+          }
+          const int key = c * 16 + q * 8;      // first key of the chunk
+          const int half = key >> 6, chunk = (key & 63) >> 3;
+          *reinterpret_cast<uint4*>(sp + half * kHalfBytes + t * 128 +
+                                    ((chunk ^ (t & 7)) << 4)) =
+              make_uint4(w[0], w[1], w[2], w[3]);
+        }
+      }
+      tc_fence_before_sync();
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&T->s_empty[sb]);
+        mbar_arrive(&T->p_full);
+      }
+      m_run = m_new;
+      if (b >= 1 && !fold(b - 1)) {
+        ok = false;
+        break;
+      }
+      m_pend = m_new;
+      l_pend = lsum;
+    }
+    if (ok && nblk > 0) ok = fold(nblk - 1);
+    if (!ok) {
+      *abort_v = 1;
+      report(a.status, PCTREE_ERR_TIMEOUT);
+    }
+    // one decision for all four softmax warps (they meet at named barriers
+    // below, which must see every one of them)
+    named_barrier(1, 128);
+    if (t == 0) T->last = *abort_v;
+    named_barrier(1, 128);
+    ok = T->last == 0;
+    named_barrier(1, 128);
+    // ---------------- output ----------------
+    const int unit = (r * a.Hkv + kvh) * a.nqt + qt;
+    const bool store_row = t < a.R && node < a.N;
+    uint16_t* orow = a.out + ((static_cast<size_t>(r) * a.N + node) * a.Hq + kvh * a.G + g) * 128;
+    auto write_out = [&](const float* v, float inv) {
+#pragma unroll
+      for (int d = 0; d < 128; d += 8) {
+        uint32_t w[4];
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          const __nv_bfloat162 b2 = __floats2bfloat162_rn(v[d + 2 * h] * inv, v[d + 2 * h + 1] * inv);
+          w[h] = *reinterpret_cast<const uint32_t*>(&b2);
+        }
+        *reinterpret_cast<uint4*>(orow + d) = make_uint4(w[0], w[1], w[2], w[3]);
+      }
+    };
+    if (a.n_split == 1) {
+      if (store_row && ok) write_out(o, l_ref > 0.0f ? 1.0f / l_ref : 0.0f);
+    } else if (ok) {
+      const size_t slot = static_cast<size_t>(unit) * a.n_split + split;
+      a.part_ml[slot * 128 + t] = make_float2(m_ref, l_ref);
+      if (l_ref > 0.0f) {
+        float4* po = reinterpret_cast<float4*>(a.part_o + (slot * 128 + t) * 128);
+#pragma unroll
+        for (int d = 0; d < 32; ++d)
+          po[d] = make_float4(o[4 * d], o[4 * d + 1], o[4 * d + 2], o[4 * d + 3]);
+      }
+      __threadfence();
+      named_barrier(1, 128);
+      if (t == 0) T->last = atomicAdd(a.ticket + unit, 1) == a.n_split - 1;
+      named_barrier(1, 128);
+      if (T->last) {
+        // the last CTA of the unit merges every split's rows
+        __threadfence();
+        float mstar = -INFINITY;
+        for (int sp_i = 0; sp_i < a.n_split; ++sp_i) {
+          const float2 ml = __ldcg(a.part_ml + (static_cast<size_t>(unit) * a.n_split + sp_i) * 128 + t);
+          if (ml.y > 0.0f) mstar = fmaxf(mstar, ml.x);
+        }
+#pragma unroll
+        for (int d = 0; d < 128; ++d) o[d] = 0.0f;   // reused as the merge sum
+        float lsum = 0.0f;
+        for (int sp_i = 0; sp_i < a.n_split; ++sp_i) {
+          const size_t sl = static_cast<size_t>(unit) * a.n_split + sp_i;
+          const float2 ml = __ldcg(a.part_ml + sl * 128 + t);
+          if (!(ml.y > 0.0f)) continue;
+          const float f = exp2f(ml.x - mstar);
+          lsum = fmaf(ml.y, f, lsum);
+          const float4* po = reinterpret_cast<const float4*>(a.part_o + (sl * 128 + t) * 128);
+#pragma unroll
+          for (int d = 0; d < 32; ++d) {
+            const float4 v = __ldcg(po + d);
+            o[4 * d] = fmaf(v.x, f, o[4 * d]);
+            o[4 * d + 1] = fmaf(v.y, f, o[4 * d + 1]);
+            o[4 * d + 2] = fmaf(v.z, f, o[4 * d + 2]);
+            o[4 * d + 3] = fmaf(v.w, f, o[4 * d + 3]);
+          }
+        }
+        if (store_row) write_out(o, lsum > 0.0f ? 1.0f / lsum : 0.0f);
+        if (t == 0) a.ticket[unit] = 0;      // ready for the next call
+      }
+    }
+  }
+  // ---------------- teardown ----------------
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem, 512);
+  }
+}
+}  // namespace
+}  // namespace pct
+
+namespace pct {
+namespace {
+
+// Tiling of a configuration: query tiles per (request, KV head) and the split
+// of each request's key blocks over CTAs.  Splits are chosen so that the
+// grid has about one CTA per SM of a 152-SM GB300 when there are few
+// (request, KV head, tile) units; they depend only on the configuration, so
+// the workspace size does too.
+struct AttnGeom {
+  int G, npt, R, nqt, nb_max, n_split, bps;
+  long long units;
+};
+
+AttnGeom attn_geom(const pctree_attn_config& c) {
+  AttnGeom g{};
+  g.G = c.Hq / c.Hkv;
+  g.npt = 128 / g.G < c.N ? 128 / g.G : c.N;
+  g.R = g.G * g.npt;
+  g.nqt = (c.N + g.npt - 1) / g.npt;
+  g.units = static_cast<long long>(c.batch) * c.Hkv * g.nqt;
+  g.nb_max = (c.max_slots + kBK - 1) / kBK;
+  long long want = (152 + g.units - 1) / g.units;
+  if (want > g.nb_max) want = g.nb_max;
+  if (want < 1) want = 1;
+  g.bps = static_cast<int>((g.nb_max + want - 1) / want);
+  g.n_split = (g.nb_max + g.bps - 1) / g.bps;
+  return g;
+}
+
+pctree_status attn_check(const pctree_attn_config* c) {
+  if (c == nullptr) return PCTREE_ERR_INVALID_ARG;
+  if (c->batch < 1 || c->N < 1 || c->Hq < 1 || c->Hkv < 1 || c->D < 1 ||
+      c->max_slots < c->N || !(c->scale > 0.0f) || !(c->scale < 1e30f))
+    return PCTREE_ERR_INVALID_ARG;
+  if (c->Hq % c->Hkv != 0) return PCTREE_ERR_INVALID_ARG;
+  if (c->D != 128 || c->Hq / c->Hkv > 128 || c->N > PCTREE_ATTN_MAX_N ||
+      c->batch > 65535 || c->Hkv > 65535)
+    return PCTREE_ERR_UNSUPPORTED;
+  const AttnGeom g = attn_geom(*c);
+  if (static_cast<long long>(g.nqt) * g.n_split > 0x7fffffffll)
+    return PCTREE_ERR_UNSUPPORTED;
+  return PCTREE_OK;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+struct AttnWs {
+  size_t part_o, part_ml, ticket, total;
+};
+
+AttnWs attn_ws(const pctree_attn_config& c, const AttnGeom& g) {
+  AttnWs w{};
+  if (g.n_split <= 1) return w;
+  const size_t slots = static_cast<size_t>(g.units) * g.n_split * 128;
+  w.part_o = 0;
+  w.part_ml = align256(w.part_o + slots * 128 * sizeof(float));
+  w.ticket = align256(w.part_ml + slots * sizeof(float2));
+  w.total = align256(w.ticket + static_cast<size_t>(g.units) * sizeof(int));
+  return w;
+}
+
+bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+}  // namespace pct
+
+extern "C" {
+
+size_t pctree_tree_attention_workspace_bytes(const pctree_attn_config* cfg) {
+  if (pct::attn_check(cfg) != PCTREE_OK) return 0;
+  return pct::attn_ws(*cfg, pct::attn_geom(*cfg)).total;
+}
+
+pctree_status pctree_tree_attention(const pctree_attn_config* cfg, const void* q,
+                                    const void* k_cache, const void* v_cache,
+                                    const int32_t* prefix_len,
+                                    const int32_t* n_nodes, const int32_t* parent,
+                                    void* out, void* workspace,
+                                    size_t workspace_bytes, int32_t* status,
+                                    void* stream_ptr) {
+  using namespace pct;
+  pctree_status st = attn_check(cfg);
+  if (st != PCTREE_OK) return st;
+  const pctree_attn_config& c = *cfg;
+  if (q == nullptr || k_cache == nullptr || v_cache == nullptr ||
+      prefix_len == nullptr || n_nodes == nullptr || parent == nullptr ||
+      out == nullptr || !al16(q) || !al16(k_cache) || !al16(v_cache) || !al16(out))
+    return PCTREE_ERR_INVALID_ARG;
+  const AttnGeom g = attn_geom(c);
+  const AttnWs w = attn_ws(c, g);
+  if (w.total > 0 && (workspace == nullptr || workspace_bytes < w.total ||
+                      (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0))
+    return PCTREE_ERR_WORKSPACE;
+  int num_sms = 0;
+  st = device_facts(&num_sms);
+  if (st != PCTREE_OK) return st;
+  CUtensorMap tm_q, tm_k, tm_v;
+  const uint64_t hd = 128 * 2;                       // bytes of one head row
+  {
+    const uint64_t dims[4] = {128, static_cast<uint64_t>(c.Hq),
+                              static_cast<uint64_t>(c.N), static_cast<uint64_t>(c.batch)};
+    const uint64_t str[3] = {hd, hd * c.Hq, hd * c.Hq * c.N};
+    const uint32_t box[4] = {64, static_cast<uint32_t>(g.G), static_cast<uint32_t>(g.npt), 1};
+    st = encode_bf16_map_nd(&tm_q, q, 4, dims, str, box);
+    if (st != PCTREE_OK) return st;
+  }
+  {
+    const uint64_t dims[4] = {128, static_cast<uint64_t>(c.Hkv),
+                              static_cast<uint64_t>(c.max_slots),
+                              static_cast<uint64_t>(c.batch)};
+    const uint64_t str[3] = {hd, hd * c.Hkv, hd * c.Hkv * c.max_slots};
+    const uint32_t box[4] = {64, 1, static_cast<uint32_t>(kBK), 1};
+    st = encode_bf16_map_nd(&tm_k, k_cache, 4, dims, str, box);
+    if (st != PCTREE_OK) return st;
+    st = encode_bf16_map_nd(&tm_v, v_cache, 4, dims, str, box);
+    if (st != PCTREE_OK) return st;
+  }
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_ptr);
+  AttnArgs a{};
+  a.prefix = prefix_len;
+  a.n_nodes = n_nodes;
+  a.parent = parent;
+  a.out = static_cast<uint16_t*>(out);
+  a.status = status;
+  a.batch = c.batch;
+  a.N = c.N;
+  a.Hq = c.Hq;
+  a.Hkv = c.Hkv;
+  a.G = g.G;
+  a.npt = g.npt;
+  a.R = g.R;
+  a.nqt = g.nqt;
+  a.max_slots = c.max_slots;
+  a.n_split = g.n_split;
+  a.bps = g.bps;
+  a.scale_log2 = static_cast<float>(static_cast<double>(c.scale) * 1.4426950408889634);
+  if (w.total > 0) {
+    unsigned char* ws = static_cast<unsigned char*>(workspace);
+    a.part_o = reinterpret_cast<float*>(ws + w.part_o);
+    a.part_ml = reinterpret_cast<float2*>(ws + w.part_ml);
+    a.ticket = reinterpret_cast<int*>(ws + w.ticket);
+    if (cudaMemsetAsync(a.ticket, 0, static_cast<size_t>(g.units) * sizeof(int), stream) !=
+        cudaSuccess)
+      return PCTREE_ERR_CUDA;
+  }
+  // a dummy status word is not needed: kernels test for NULL
+  static bool attr_set[64] = {false};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return PCTREE_ERR_CUDA;
+  if (!attr_set[dev]) {
+    if (cudaFuncSetAttribute(tree_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(kAttnSmem)) != cudaSuccess)
+      return PCTREE_ERR_CUDA;
+    attr_set[dev] = true;
+  }
+  const dim3 grid(static_cast<unsigned>(g.nqt * g.n_split), static_cast<unsigned>(c.Hkv),
+                  static_cast<unsigned>(c.batch));
+  tree_attn_kernel<<<grid, kAttnThreads, kAttnSmem, stream>>>(tm_q, tm_k, tm_v, a);
+  return cudaGetLastError() == cudaSuccess ? PCTREE_OK : PCTREE_ERR_CUDA;
+}
+
+}  // extern "C"

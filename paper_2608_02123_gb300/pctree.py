@@ -53,6 +53,14 @@ class CompactLayout(ctypes.Structure):
                 ("hidden_bytes", ctypes.c_int64)]
 
 
+class AttnConfig(ctypes.Structure):
+    """pctree_attn_config: one grouped-query attention layer."""
+    _fields_ = [("batch", ctypes.c_int32), ("N", ctypes.c_int32),
+                ("Hq", ctypes.c_int32), ("Hkv", ctypes.c_int32),
+                ("D", ctypes.c_int32), ("max_slots", ctypes.c_int32),
+                ("scale", ctypes.c_float)]
+
+
 class _Tree(ctypes.Structure):
     _fields_ = [(name, ctypes.c_void_p) for name in (
         "n_nodes", "tokens", "parent", "depth", "logp", "position_ids",
@@ -85,6 +93,12 @@ def _load() -> ctypes.CDLL:
     lib.pctree_compact.argtypes = [ctypes.POINTER(CompactLayout), vp, vp, vp,
                                    vp, vp, vp, vp, vp]
     lib.pctree_compact.restype = ctypes.c_int
+    ap = ctypes.POINTER(AttnConfig)
+    lib.pctree_tree_attention_workspace_bytes.argtypes = [ap]
+    lib.pctree_tree_attention_workspace_bytes.restype = ctypes.c_size_t
+    lib.pctree_tree_attention.argtypes = [ap] + [vp] * 8 + [ctypes.c_size_t,
+                                                           vp, vp]
+    lib.pctree_tree_attention.restype = ctypes.c_int
     lib.pctree_status_string.argtypes = [ctypes.c_int32]
     lib.pctree_status_string.restype = ctypes.c_char_p
     lib.pctree_profile_enable.argtypes = [ctypes.c_int32]
@@ -278,6 +292,37 @@ def pctree_compact(layout: CompactLayout, accepted_idx: torch.Tensor,
                             _ptr(status), _stream_ptr(stream))
     if rc != PCTREE_OK:
         raise PctreeError(rc, "pctree_compact")
+
+
+def attn_config(batch: int, N: int, Hq: int, Hkv: int, max_slots: int,
+                D: int = 128, scale: Optional[float] = None) -> AttnConfig:
+    """``scale`` defaults to 1/sqrt(D)."""
+    return AttnConfig(batch, N, Hq, Hkv, D, max_slots,
+                      D ** -0.5 if scale is None else scale)
+
+
+def pctree_tree_attention_workspace_bytes(cfg: AttnConfig) -> int:
+    return LIB.pctree_tree_attention_workspace_bytes(ctypes.byref(cfg))
+
+
+def pctree_tree_attention(cfg: AttnConfig, q: torch.Tensor, k_cache: torch.Tensor,
+                          v_cache: torch.Tensor, prefix_len: torch.Tensor,
+                          n_nodes: torch.Tensor, parent: torch.Tensor,
+                          out: torch.Tensor,
+                          workspace: Optional[torch.Tensor] = None,
+                          status: Optional[torch.Tensor] = None,
+                          stream: Optional[torch.cuda.Stream] = None) -> None:
+    """Enqueue one tree-verification attention layer (see
+    pctree_tree_attention)."""
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    rc = LIB.pctree_tree_attention(ctypes.byref(cfg), q.data_ptr(),
+                                   k_cache.data_ptr(), v_cache.data_ptr(),
+                                   prefix_len.data_ptr(), n_nodes.data_ptr(),
+                                   parent.data_ptr(), out.data_ptr(),
+                                   _ptr(workspace), ws_bytes, _ptr(status),
+                                   _stream_ptr(stream))
+    if rc != PCTREE_OK:
+        raise PctreeError(rc, "pctree_tree_attention")
 
 
 def pctree_profile_enable(on: bool) -> None:
