@@ -15,16 +15,19 @@
 //               buffers (M=128, N=128 keys, K=128 dims), then O_b = P_b V_b
 //               into a third (M=128, N=128 dims, K=128 keys; V is the
 //               MN-major operand, dims contiguous)
-//   warps 2..5  softmax, one thread per TMEM lane = tile row: masked running
-//               max, P = 2^(s - m) rounded to bf16 into shared memory (the
-//               K-major A operand of the second MMA), and the running output
-//               O = O * 2^(m_old - m_new) + O_b kept in registers
+//   warps 2..5  softmax, one thread per TMEM lane = tile row: each S row is
+//               read from TMEM once, masked and scaled; P = 2^(s - m_used)
+//               rounded to bf16 into shared memory (the K-major A operand of
+//               the second MMA).  O accumulates in TMEM across blocks; the
+//               reference m_used rises (O and the row sum rescaled in place,
+//               tcgen05.ld / st) only when a block's maximum exceeds it by
+//               more than 8 in log2 units, so P stays below 2^8.
 //
-// S of block b+1 is computed while the softmax works on block b and the PV
-// product of block b runs while the softmax folds block b-1.  Key blocks of
-// a request may be split over several CTAs; each writes (max, sum, O) of its
-// rows and the last CTA of the unit (an atomic ticket, no waiting) merges
-// them.  All waits are bounded (1 s) and end in PCTREE_ERR_TIMEOUT.
+// S of block b+1 is computed while the softmax works on block b.  Key blocks
+// of a request may be split over several CTAs (few requests, long
+// prefixes); each then writes (max, sum, unnormalised O) of its rows and a
+// second kernel merges the splits, spread over all SMs.  All waits are
+// bounded (1 s) and end in PCTREE_ERR_TIMEOUT.
 #include <cuda_bf16.h>
 
 #include "pctree_common.cuh"
@@ -47,11 +50,12 @@ struct AttnTail {
   uint64_t q_full;
   uint64_t kv_full[2], kv_empty[2];
   uint64_t s_full[2], s_empty[2];
-  uint64_t p_full, p_empty, o_full, o_empty, done;
+  uint64_t p_full, p_empty, o_full, done;
   uint32_t tmem_base;
   int abort;
   int last;
   uint32_t anc[128][kMaskWords];          // ancestor-or-self bits per node
+  int32_t par[PCTREE_ATTN_MAX_N];         // the request's packed parents
 };
 
 constexpr size_t kAttnSmem = kTailOff + sizeof(AttnTail) + 1024;
@@ -63,7 +67,6 @@ struct AttnArgs {
   uint16_t* out;          // bf16 [batch][N][Hq][128]
   float* part_o;          // [unit][split][128][128]
   float2* part_ml;        // [unit][split][128]  (max in log2 units, sum)
-  int* ticket;            // [unit]
   int32_t* status;
   int batch, N, Hq, Hkv, G, npt, R, nqt, max_slots, n_split, bps;
   float scale_log2;       // softmax scale * log2(e)
@@ -141,7 +144,6 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     mbar_init(&T->p_full, 4);
     mbar_init(&T->p_empty, 1);
     mbar_init(&T->o_full, 1);
-    mbar_init(&T->o_empty, 4);
     mbar_init(&T->done, 1);
     T->abort = 0;
     fence_barrier_init();
@@ -152,14 +154,18 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     *reinterpret_cast<uint4*>(sq + half * kHalfBytes + (a.R + rem / 8) * 128 +
                               (rem % 8) * 16) = make_uint4(0, 0, 0, 0);
   }
-  // ancestor-or-self bits of the tile's nodes (walk up the packed parents)
+  // ancestor-or-self bits of the tile's nodes (walk up the packed parents,
+  // staged in shared memory)
+  for (int i = threadIdx.x; i < n; i += blockDim.x)
+    T->par[i] = a.parent[static_cast<size_t>(r) * a.N + i];
+  __syncthreads();
   for (int nl = threadIdx.x; nl < a.npt; nl += blockDim.x) {
     uint32_t bits[kMaskWords];
 #pragma unroll
     for (int w = 0; w < kMaskWords; ++w) bits[w] = 0u;
     int x = qt * a.npt + nl;
     if (x < n) {
-      const int32_t* par = a.parent + static_cast<size_t>(r) * a.N;
+      const int32_t* par = T->par;
       for (int steps = 0; steps <= n && x >= 0 && x < n; ++steps) {
 #pragma unroll
         for (int w = 0; w < kMaskWords; ++w)
@@ -234,8 +240,6 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     auto issue_o = [&](int b) -> bool {
       const int s = b & 1;
       if (!mbar_wait_bounded(&T->p_full, b & 1, abort_v, kAttnLimitNs)) return false;
-      if (b >= 1 && !mbar_wait_bounded(&T->o_empty, (b - 1) & 1, abort_v, kAttnLimitNs))
-        return false;
       tc_fence_after_sync();
       const uint32_t v0 = smem_u32(kv_v(sm, s));
 #pragma unroll
@@ -244,7 +248,7 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
         // 16 keys = 16 rows of 128 B; the dims 64..127 half is kHalfBytes on
         tc_mma_bf16(tmem + 256, desc_kmajor_sw128(p0 + aoff),
                     desc_mnmajor_sw128(v0 + kk * 16 * 128, kHalfBytes, 1024), idO,
-                    kk > 0 ? 1u : 0u);
+                    (b > 0 || kk > 0) ? 1u : 0u);   // O accumulates over blocks
       }
       tc_commit(&T->o_full);
       tc_commit(&T->kv_empty[s]);
@@ -262,7 +266,10 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     (void)mbar_wait_bounded(&T->done, 0, abort_v, kAttnLimitNs);
   }
   else if (warp >= 2) {
-    // ---------------- softmax and output, one thread per tile row ----------
+    // ---------------- softmax, one thread per tile row ----------------
+    // O accumulates in TMEM through the PV MMA with P = 2^(s - m_used); the
+    // reference m_used moves (and O and l are rescaled in place) only when
+    // a block's maximum exceeds it by more than 2^8, so P stays <= 256.
     const int quad = warp & 3;               // TMEM lanes quad*32 .. +31
     const int t = quad * 32 + lane;          // tile row
     const int nl = t / a.G, g = t - nl * a.G;
@@ -270,63 +277,65 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     const bool row_ok = t < a.R && node < n;
     const uint32_t* anc = T->anc[nl < a.npt ? nl : 0];
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(quad * 32) << 16);
-    float o[128];
-#pragma unroll
-    for (int d = 0; d < 128; ++d) o[d] = 0.0f;
-    float m_ref = -INFINITY, l_ref = 0.0f;   // o and l_ref are relative to m_ref
-    float m_run = -INFINITY;                 // running max (log2 units)
-    float m_pend = -INFINITY, l_pend = 0.0f; // block whose PV product is pending
+    const float sc = a.scale_log2;
+    float m_used = -INFINITY, l_sum = 0.0f;  // O and l_sum are relative to m_used
     bool ok = true;
-    auto fold = [&](int b) -> bool {         // o += O_b (relative to m_pend)
-      if (!mbar_wait_bounded(&T->o_full, b & 1, abort_v, kAttnLimitNs)) return false;
-      tc_fence_after_sync();
-      const float alpha = m_ref == m_pend ? 1.0f : exp2f(m_ref - m_pend);
-#pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        uint32_t y[16];
-        tmem_ld_32x32b_x16(lane_base + 256 + c * 16, y);
-        tmem_ld_wait();
-#pragma unroll
-        for (int j = 0; j < 16; ++j)
-          o[c * 16 + j] = fmaf(o[c * 16 + j], alpha, __uint_as_float(y[j]));
-      }
-      l_ref = fmaf(l_ref, alpha, l_pend);
-      m_ref = m_pend;
-      tc_fence_before_sync();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&T->o_empty);
-      return true;
+    // the warp continues only if all its lanes saw the phase complete, so
+    // the warp-collective tcgen05 loads that follow never diverge
+    auto wwait = [&](uint64_t* bar, uint32_t parity) -> bool {
+      const bool got = mbar_wait_bounded(bar, parity, abort_v, kAttnLimitNs);
+      return __all_sync(kFull, got);
     };
-    for (int b = 0; ok && b < nblk; ++b) {
+    for (int b = 0; b < nblk; ++b) {
       const int sb = b & 1;
       const int key0 = (kb0 + b) * kBK;
-      if (!mbar_wait_bounded(&T->s_full[sb], (b >> 1) & 1, abort_v, kAttnLimitNs)) {
+      if (!wwait(&T->s_full[sb], (b >> 1) & 1)) {
         ok = false;
         break;
       }
       tc_fence_after_sync();
-      const uint32_t s_base = lane_base + sb * 128;
-      // pass 1: the block's largest allowed score
-      uint32_t allow[4];
-      float mx = -INFINITY;
+      float x[128];
+      {
+        uint32_t* xu = reinterpret_cast<uint32_t*>(x);
 #pragma unroll
-      for (int c = 0; c < 4; ++c) allow[c] = row_ok ? allowed_bits(key0 + c * 32, Tp, anc) : 0u;
-#pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        uint32_t x[16];
-        tmem_ld_32x32b_x16(s_base + c * 16, x);
+        for (int c = 0; c < 4; ++c)
+          tmem_ld_32x32b_x32(lane_base + sb * 128 + c * 32,
+                             *reinterpret_cast<uint32_t(*)[32]>(xu + c * 32));
         tmem_ld_wait();
-        const uint32_t al = allow[c >> 1] >> ((c & 1) * 16);
-#pragma unroll
-        for (int j = 0; j < 16; ++j)
-          if ((al >> j) & 1u) mx = fmaxf(mx, __uint_as_float(x[j]) * a.scale_log2);
       }
-      const float m_new = fmaxf(m_run, mx);
+      tc_fence_before_sync();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&T->s_empty[sb]);   // S buffer free
+      // scaled scores; keys the row may not see become -inf
+      // (eight independent running maxima keep the dependency chains short)
+      float m8[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) m8[u] = -INFINITY;
+      if (row_ok && key0 + kBK <= Tp) {      // a block of prefix keys only
+#pragma unroll
+        for (int j = 0; j < 128; ++j) {
+          x[j] *= sc;
+          m8[j & 7] = fmaxf(m8[j & 7], x[j]);
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const uint32_t al = row_ok ? allowed_bits(key0 + c * 32, Tp, anc) : 0u;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const float v = ((al >> j) & 1u) ? x[c * 32 + j] * sc : -INFINITY;
+            x[c * 32 + j] = v;
+            m8[j & 7] = fmaxf(m8[j & 7], v);
+          }
+        }
+      }
+      const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+                             fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
       // the last block of the request: V rows past the tree hold whatever the
       // cache held there; zero them so that 0 * (non-finite) cannot reach O
       const int valid = n_keys - key0;
       if (valid < kBK) {
-        if (!mbar_wait_bounded(&T->kv_full[sb], (b >> 1) & 1, abort_v, kAttnLimitNs)) {
+        if (!wwait(&T->kv_full[sb], (b >> 1) & 1)) {
           ok = false;
           break;
         }
@@ -337,56 +346,63 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
                                     (rem % 8) * 16) = make_uint4(0, 0, 0, 0);
         }
       }
-      // pass 2: P = 2^(s - m_new) in bf16, into the A operand of the PV MMA
-      if (b >= 1 && !mbar_wait_bounded(&T->p_empty, (b - 1) & 1, abort_v, kAttnLimitNs)) {
+      // the PV product of the previous block has finished: P may be
+      // rewritten and O read
+      if (b >= 1 && !wwait(&T->p_empty, (b - 1) & 1)) {
         ok = false;
         break;
       }
-      float lsum = 0.0f;
+      // move the reference up where a row needs it; tcgen05.ld / st are
+      // warp-collective, so the warp rescales together (alpha = 1 for rows
+      // that keep their reference)
+      const bool mine = mx > m_used + 8.0f;
+      const float alpha = mine ? ex2_approx(m_used - mx) : 1.0f;   // 0 from -inf
+      if (__any_sync(kFull, mine)) {
+        if (b >= 1) {
+          tc_fence_after_sync();
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        uint32_t x[16];
-        tmem_ld_32x32b_x16(s_base + c * 16, x);
-        tmem_ld_wait();
-        const uint32_t al = allow[c >> 1] >> ((c & 1) * 16);
+          for (int c = 0; c < 4; ++c) {
+            uint32_t y[32];
+            tmem_ld_32x32b_x32(lane_base + 256 + c * 32, y);
+            tmem_ld_wait();
 #pragma unroll
-        for (int q = 0; q < 2; ++q) {          // 8 keys = one 16-byte chunk
-          uint32_t w[4];
-#pragma unroll
-          for (int h = 0; h < 4; ++h) {
-            const int j0 = q * 8 + h * 2;
-            float p0 = 0.0f, p1 = 0.0f;
-            if ((al >> j0) & 1u)
-              p0 = exp2f(__uint_as_float(x[j0]) * a.scale_log2 - m_new);
-            if ((al >> (j0 + 1)) & 1u)
-              p1 = exp2f(__uint_as_float(x[j0 + 1]) * a.scale_log2 - m_new);
-            const __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
-            lsum += __low2float(pb) + __high2float(pb);
-            w[h] = *reinterpret_cast<const uint32_t*>(&pb);
+            for (int j = 0; j < 32; ++j)
+              y[j] = __float_as_uint(__uint_as_float(y[j]) * alpha);
+            tmem_st_32x32b_x32(lane_base + 256 + c * 32, y);
           }
-          const int key = c * 16 + q * 8;      // first key of the chunk
-          const int half = key >> 6, chunk = (key & 63) >> 3;
-          *reinterpret_cast<uint4*>(sp + half * kHalfBytes + t * 128 +
-                                    ((chunk ^ (t & 7)) << 4)) =
-              make_uint4(w[0], w[1], w[2], w[3]);
+          tmem_st_wait();
+        }
+        if (mine) {
+          l_sum *= alpha;
+          m_used = mx;
         }
       }
+      // P = 2^(s - m_used) in bf16, the A operand of the PV MMA
+      const float mref = m_used == -INFINITY ? 0.0f : m_used;
+      float ls[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+      for (int c = 0; c < 16; ++c) {         // 8 keys = one 16-byte chunk
+        uint32_t w[4];
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          const float p0 = ex2_approx(x[c * 8 + 2 * h] - mref);
+          const float p1 = ex2_approx(x[c * 8 + 2 * h + 1] - mref);
+          ls[h] += p0 + p1;
+          const __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
+          w[h] = *reinterpret_cast<const uint32_t*>(&pb);
+        }
+        const int half = c >> 3, chunk = c & 7;
+        *reinterpret_cast<uint4*>(sp + half * kHalfBytes + t * 128 +
+                                  ((chunk ^ (t & 7)) << 4)) =
+            make_uint4(w[0], w[1], w[2], w[3]);
+      }
+      l_sum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
       tc_fence_before_sync();
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&T->s_empty[sb]);
-        mbar_arrive(&T->p_full);
-      }
-      m_run = m_new;
-      if (b >= 1 && !fold(b - 1)) {
-        ok = false;
-        break;
-      }
-      m_pend = m_new;
-      l_pend = lsum;
+      if (lane == 0) mbar_arrive(&T->p_full);
     }
-    if (ok && nblk > 0) ok = fold(nblk - 1);
+    if (ok && nblk > 0 && !wwait(&T->o_full, (nblk - 1) & 1)) ok = false;
     if (!ok) {
       *abort_v = 1;
       report(a.status, PCTREE_ERR_TIMEOUT);
@@ -398,66 +414,61 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     named_barrier(1, 128);
     ok = T->last == 0;
     named_barrier(1, 128);
+    tc_fence_after_sync();
     // ---------------- output ----------------
+    // O is read from TMEM in four 32-column chunks; tcgen05.ld is
+    // warp-collective, so every lane loads and only valid rows store.
     const int unit = (r * a.Hkv + kvh) * a.nqt + qt;
     const bool store_row = t < a.R && node < a.N;
     uint16_t* orow = a.out + ((static_cast<size_t>(r) * a.N + node) * a.Hq + kvh * a.G + g) * 128;
-    auto write_out = [&](const float* v, float inv) {
+    auto store_chunk = [&](int c, const float (&v)[32], float inv) {
 #pragma unroll
-      for (int d = 0; d < 128; d += 8) {
+      for (int q = 0; q < 4; ++q) {
         uint32_t w[4];
 #pragma unroll
         for (int h = 0; h < 4; ++h) {
-          const __nv_bfloat162 b2 = __floats2bfloat162_rn(v[d + 2 * h] * inv, v[d + 2 * h + 1] * inv);
+          const __nv_bfloat162 b2 =
+              __floats2bfloat162_rn(v[q * 8 + 2 * h] * inv, v[q * 8 + 2 * h + 1] * inv);
           w[h] = *reinterpret_cast<const uint32_t*>(&b2);
         }
-        *reinterpret_cast<uint4*>(orow + d) = make_uint4(w[0], w[1], w[2], w[3]);
+        *reinterpret_cast<uint4*>(orow + c * 32 + q * 8) = make_uint4(w[0], w[1], w[2], w[3]);
+      }
+    };
+    auto load_chunk = [&](int c, float (&v)[32]) {
+      if (nblk > 0) {
+        uint32_t y[32];
+        tmem_ld_32x32b_x32(lane_base + 256 + c * 32, y);
+        tmem_ld_wait();
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(y[j]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = 0.0f;
       }
     };
     if (a.n_split == 1) {
-      if (store_row && ok) write_out(o, l_ref > 0.0f ? 1.0f / l_ref : 0.0f);
+      if (ok) {
+        const float inv = l_sum > 0.0f ? 1.0f / l_sum : 0.0f;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          float v[32];
+          load_chunk(c, v);
+          if (store_row) store_chunk(c, v, inv);
+        }
+      }
     } else if (ok) {
       const size_t slot = static_cast<size_t>(unit) * a.n_split + split;
-      a.part_ml[slot * 128 + t] = make_float2(m_ref, l_ref);
-      if (l_ref > 0.0f) {
-        float4* po = reinterpret_cast<float4*>(a.part_o + (slot * 128 + t) * 128);
+      a.part_ml[slot * 128 + t] = make_float2(l_sum > 0.0f ? m_used : -INFINITY, l_sum);
+      float4* po = reinterpret_cast<float4*>(a.part_o + (slot * 128 + t) * 128);
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        float v[32];
+        load_chunk(c, v);
+        if (l_sum > 0.0f) {
 #pragma unroll
-        for (int d = 0; d < 32; ++d)
-          po[d] = make_float4(o[4 * d], o[4 * d + 1], o[4 * d + 2], o[4 * d + 3]);
-      }
-      __threadfence();
-      named_barrier(1, 128);
-      if (t == 0) T->last = atomicAdd(a.ticket + unit, 1) == a.n_split - 1;
-      named_barrier(1, 128);
-      if (T->last) {
-        // the last CTA of the unit merges every split's rows
-        __threadfence();
-        float mstar = -INFINITY;
-        for (int sp_i = 0; sp_i < a.n_split; ++sp_i) {
-          const float2 ml = __ldcg(a.part_ml + (static_cast<size_t>(unit) * a.n_split + sp_i) * 128 + t);
-          if (ml.y > 0.0f) mstar = fmaxf(mstar, ml.x);
+          for (int q = 0; q < 8; ++q)
+            po[c * 8 + q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
         }
-#pragma unroll
-        for (int d = 0; d < 128; ++d) o[d] = 0.0f;   // reused as the merge sum
-        float lsum = 0.0f;
-        for (int sp_i = 0; sp_i < a.n_split; ++sp_i) {
-          const size_t sl = static_cast<size_t>(unit) * a.n_split + sp_i;
-          const float2 ml = __ldcg(a.part_ml + sl * 128 + t);
-          if (!(ml.y > 0.0f)) continue;
-          const float f = exp2f(ml.x - mstar);
-          lsum = fmaf(ml.y, f, lsum);
-          const float4* po = reinterpret_cast<const float4*>(a.part_o + (sl * 128 + t) * 128);
-#pragma unroll
-          for (int d = 0; d < 32; ++d) {
-            const float4 v = __ldcg(po + d);
-            o[4 * d] = fmaf(v.x, f, o[4 * d]);
-            o[4 * d + 1] = fmaf(v.y, f, o[4 * d + 1]);
-            o[4 * d + 2] = fmaf(v.z, f, o[4 * d + 2]);
-            o[4 * d + 3] = fmaf(v.w, f, o[4 * d + 3]);
-          }
-        }
-        if (store_row) write_out(o, lsum > 0.0f ? 1.0f / lsum : 0.0f);
-        if (t == 0) a.ticket[unit] = 0;      // ready for the next call
       }
     }
   }
@@ -470,6 +481,79 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     tmem_dealloc(tmem, 512);
   }
 }
+// Merges the key splits of every (request, KV head, tile) unit: one thread
+// per 16 output dims of a row, 16 rows per CTA.  Per row the splits' maxima
+// and sums give weights 2^(m_s - m*); the weighted partial outputs are summed
+// four splits at a time (their loads in flight together) and normalised.
+constexpr int kMergeThreads = 128;
+constexpr int kMergeRows = 16;
+
+__global__ void __launch_bounds__(kMergeThreads)
+tree_attn_merge_kernel(AttnArgs a) {
+  const int unit = blockIdx.x;
+  const int row = blockIdx.y * kMergeRows + (threadIdx.x >> 3);   // tile row
+  const int d0 = (threadIdx.x & 7) * 16;
+  const int qt = unit % a.nqt;
+  const int kvh = (unit / a.nqt) % a.Hkv;
+  const int r = unit / (a.nqt * a.Hkv);
+  const int nl = row / a.G, g = row - nl * a.G;
+  const int node = qt * a.npt + nl;
+  if (row >= a.R || node >= a.N) return;
+  const float2* ml = a.part_ml + static_cast<size_t>(unit) * a.n_split * 128 + row;
+  float mstar = -INFINITY, lsum = 0.0f;
+  for (int s = 0; s < a.n_split; ++s) {
+    const float2 v = ml[static_cast<size_t>(s) * 128];
+    if (v.y > 0.0f) mstar = fmaxf(mstar, v.x);
+  }
+  float acc[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) acc[j] = 0.0f;
+  for (int s0 = 0; s0 < a.n_split; s0 += 4) {
+    float4 v[4][4];
+    float f[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      f[u] = 0.0f;
+      if (s0 + u < a.n_split) {
+        const float2 w = ml[static_cast<size_t>(s0 + u) * 128];
+        if (w.y > 0.0f) {
+          f[u] = exp2f(w.x - mstar);
+          lsum = fmaf(w.y, f[u], lsum);
+          const float4* src = reinterpret_cast<const float4*>(
+              a.part_o + ((static_cast<size_t>(unit) * a.n_split + s0 + u) * 128 + row) * 128 + d0);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) v[u][q] = src[q];
+        }
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (f[u] != 0.0f) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          acc[4 * q] = fmaf(v[u][q].x, f[u], acc[4 * q]);
+          acc[4 * q + 1] = fmaf(v[u][q].y, f[u], acc[4 * q + 1]);
+          acc[4 * q + 2] = fmaf(v[u][q].z, f[u], acc[4 * q + 2]);
+          acc[4 * q + 3] = fmaf(v[u][q].w, f[u], acc[4 * q + 3]);
+        }
+      }
+    }
+  }
+  const float inv = lsum > 0.0f ? 1.0f / lsum : 0.0f;
+  uint16_t* orow = a.out + ((static_cast<size_t>(r) * a.N + node) * a.Hq + kvh * a.G + g) * 128 + d0;
+#pragma unroll
+  for (int q = 0; q < 2; ++q) {
+    uint32_t w[4];
+#pragma unroll
+    for (int h = 0; h < 4; ++h) {
+      const __nv_bfloat162 b2 =
+          __floats2bfloat162_rn(acc[q * 8 + 2 * h] * inv, acc[q * 8 + 2 * h + 1] * inv);
+      w[h] = *reinterpret_cast<const uint32_t*>(&b2);
+    }
+    *reinterpret_cast<uint4*>(orow + q * 8) = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+}
+
 }  // namespace
 }  // namespace pct
 
@@ -520,7 +604,7 @@ pctree_status attn_check(const pctree_attn_config* c) {
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 struct AttnWs {
-  size_t part_o, part_ml, ticket, total;
+  size_t part_o, part_ml, total;
 };
 
 AttnWs attn_ws(const pctree_attn_config& c, const AttnGeom& g) {
@@ -529,8 +613,7 @@ AttnWs attn_ws(const pctree_attn_config& c, const AttnGeom& g) {
   const size_t slots = static_cast<size_t>(g.units) * g.n_split * 128;
   w.part_o = 0;
   w.part_ml = align256(w.part_o + slots * 128 * sizeof(float));
-  w.ticket = align256(w.part_ml + slots * sizeof(float2));
-  w.total = align256(w.ticket + static_cast<size_t>(g.units) * sizeof(int));
+  w.total = align256(w.part_ml + slots * sizeof(float2));
   return w;
 }
 
@@ -613,10 +696,6 @@ pctree_status pctree_tree_attention(const pctree_attn_config* cfg, const void* q
     unsigned char* ws = static_cast<unsigned char*>(workspace);
     a.part_o = reinterpret_cast<float*>(ws + w.part_o);
     a.part_ml = reinterpret_cast<float2*>(ws + w.part_ml);
-    a.ticket = reinterpret_cast<int*>(ws + w.ticket);
-    if (cudaMemsetAsync(a.ticket, 0, static_cast<size_t>(g.units) * sizeof(int), stream) !=
-        cudaSuccess)
-      return PCTREE_ERR_CUDA;
   }
   // a dummy status word is not needed: kernels test for NULL
   static bool attr_set[64] = {false};
@@ -631,7 +710,13 @@ pctree_status pctree_tree_attention(const pctree_attn_config* cfg, const void* q
   const dim3 grid(static_cast<unsigned>(g.nqt * g.n_split), static_cast<unsigned>(c.Hkv),
                   static_cast<unsigned>(c.batch));
   tree_attn_kernel<<<grid, kAttnThreads, kAttnSmem, stream>>>(tm_q, tm_k, tm_v, a);
-  return cudaGetLastError() == cudaSuccess ? PCTREE_OK : PCTREE_ERR_CUDA;
+  if (cudaGetLastError() != cudaSuccess) return PCTREE_ERR_CUDA;
+  if (g.n_split > 1) {
+    const dim3 mgrid(static_cast<unsigned>(g.units), (g.R + kMergeRows - 1) / kMergeRows);
+    tree_attn_merge_kernel<<<mgrid, kMergeThreads, 0, stream>>>(a);
+    if (cudaGetLastError() != cudaSuccess) return PCTREE_ERR_CUDA;
+  }
+  return PCTREE_OK;
 }
 
 }  // extern "C"
