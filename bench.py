@@ -269,6 +269,38 @@ def run_reference(args, wl, rank, world):
 # the CUDA path
 # ---------------------------------------------------------------------------
 
+# ---------------------------------------------------------------------------
+# multi-rank plumbing: independent replicas, no collective on the data path
+# ---------------------------------------------------------------------------
+
+def rank_requests(rank, world, n_sets, batch):
+    """Request indices of every input set on this rank.  Ranks draw disjoint
+    requests (each GPU drafts its own), so the job's requests are
+    ``world * n_sets * batch`` distinct ones."""
+    per_rank = n_sets * batch
+    return [[rank * per_rank + i * batch + b for b in range(batch)]
+            for i in range(n_sets)]
+
+
+def max_over_ranks(values, world, device=None):
+    """Element-wise maximum of per-rank timings (the slowest rank sets the
+    job's time)."""
+    if world == 1:
+        return [float(v) for v in values]
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64,
+                     device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.tolist()]
+
+
+def job_rounds_per_s(ms_max, steps, world, batch):
+    """Whole-job throughput: every rank's rounds over the slowest rank's
+    time."""
+    return steps * world * batch / (ms_max / 1e3)
+
+
 def run_ours(args, wl, rank, world, local_rank):
     import torch
     import torch.distributed as dist
@@ -288,12 +320,10 @@ def run_ours(args, wl, rank, world, local_rank):
     # sets that their base logits exceed the L2 three times over
     batch_bytes = wl.batch * wl.B * wl.V * 4
     n_sets = max(2, min(N_SETS, -(-3 * L2_BYTES // batch_bytes)))
-    per_rank = n_sets * wl.batch
-    many = wl.with_(batch=per_rank * world)
+    many = wl.with_(batch=n_sets * wl.batch * world)
     sets = []
-    for i in range(n_sets):
-        reqs = [draw_request(many, rank * per_rank + i * wl.batch + b)
-                for b in range(wl.batch)]
+    for ids in rank_requests(rank, world, n_sets, wl.batch):
+        reqs = [draw_request(many, q) for q in ids]
         sets.append((np.stack([q[0] for q in reqs]),
                      np.asarray([q[1] for q in reqs], np.int32),
                      np.stack([q[2] for q in reqs])))
@@ -382,15 +412,11 @@ def run_ours(args, wl, rank, world, local_rank):
     e2e_ms = e_start.elapsed_time(e_end)
     clk = clocks.stop()
 
-    if world > 1:
-        t = torch.tensor([ms, e2e_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms, e2e_ms = float(t[0]), float(t[1])
+    ms, e2e_ms = max_over_ranks([ms, e2e_ms], world, dev)
     if rank != 0:
         return
 
-    rounds = args.steps * world * wl.batch
-    value = rounds / (ms / 1e3)
+    value = job_rounds_per_s(ms, args.steps, world, wl.batch)
     peaks, peak_kind = measured_peaks()
     peak = float(peaks["hbm_gbs"])
     bytes_round = round_bytes(wl)
@@ -423,7 +449,8 @@ def run_ours(args, wl, rank, world, local_rank):
                      "launches": launches,
                      "avg_launch_us": proj_ms * 1e3 / launches if launches else None,
                      "traffic": recorded_traffic(wl, fused)},
-        "e2e": {"value": rounds / (e2e_ms / 1e3), "unit": "rounds/s",
+        "e2e": {"value": job_rounds_per_s(e2e_ms, args.steps, world, wl.batch),
+                "unit": "rounds/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": kernels_per_step * args.steps,
         "clocks": clk,
