@@ -4,17 +4,17 @@
 // root-to-node ancestors.
 //
 // Work unit (one CTA): request r, KV head h, a tile of query rows and a range
-// of 128-key blocks.  The tile's rows are (node, query head of the group)
+// of 64-key blocks.  The tile's rows are (node, query head of the group)
 // pairs, node-major: row t = node_local * G + g, R = G * nodes_per_tile <= 128.
 // The G query heads sharing KV head h read the same K/V blocks once.
 //
-//   warp 0      TMA producer: the Q tile once, then K and V blocks (128 keys
+//   warp 0      TMA producer: the Q tile once, then K and V blocks (64 keys
 //               x 128 dims, two 64-dim halves each, 128-byte swizzle) into a
-//               two-stage ring
+//               four-stage ring (three blocks in flight ahead of the MMA)
 //   warp 1      tcgen05.mma issuer: S_b = Q K_b^T into one of two TMEM
-//               buffers (M=128, N=128 keys, K=128 dims), then O_b = P_b V_b
-//               into a third (M=128, N=128 dims, K=128 keys; V is the
-//               MN-major operand, dims contiguous)
+//               buffers (M=128, N=64 keys, K=128 dims), then O += P_b V_b
+//               (M=128, N=128 dims, K=64 keys; V is the MN-major operand,
+//               dims contiguous) from one of two P buffers
 //   warps 2..5  softmax, one thread per TMEM lane = tile row: each S row is
 //               read from TMEM once, masked and scaled; P = 2^(s - m_used)
 //               rounded to bf16 into shared memory (the K-major A operand of
@@ -37,20 +37,25 @@ namespace pct {
 namespace {
 
 constexpr int kAttnThreads = 192;
-constexpr int kBK = 128;                  // keys per block
-constexpr int kHalfBytes = 128 * 128;     // 128 rows x 64 bf16 (one dim half)
+constexpr int kBK = 64;                   // keys per block
+constexpr int kStages = 4;                // K/V ring depth
+constexpr int kHalfBytes = 128 * 128;     // Q: 128 rows x 64 bf16 (one dim half)
+constexpr int kKVHalf = kBK * 128;        // K or V: 64 keys x 64 bf16 (one dim half)
+constexpr int kStageBytes = 4 * kKVHalf;  // K (two halves) then V (two halves)
+constexpr int kPBytes = 128 * kBK * 2;    // P: 128 rows x 64 keys bf16
 constexpr int kQOff = 0;
-constexpr int kKVOff = 2 * kHalfBytes;    // stage s: K at +s*64K, V at +32K
-constexpr int kPOff = kKVOff + 2 * 4 * kHalfBytes;
-constexpr int kTailOff = kPOff + 2 * kHalfBytes;
+constexpr int kKVOff = 2 * kHalfBytes;
+constexpr int kPOff = kKVOff + kStages * kStageBytes;   // two P buffers
+constexpr int kTailOff = kPOff + 2 * kPBytes;
+constexpr uint32_t kOCol = 128;           // TMEM: S buffers at 0 and 64, O at 128
 constexpr int kMaskWords = PCTREE_ATTN_MAX_N / 32;
 constexpr uint64_t kAttnLimitNs = 1000000000ull;
 
 struct AttnTail {
   uint64_t q_full;
-  uint64_t kv_full[2], kv_empty[2];
+  uint64_t kv_full[kStages], kv_empty[kStages];
   uint64_t s_full[2], s_empty[2];
-  uint64_t p_full, p_empty, o_full, done;
+  uint64_t p_full, p_empty[2], done;     // p_empty[i]: PV products of blocks i, i+2, ...
   uint32_t tmem_base;
   int abort;
   int last;
@@ -73,10 +78,10 @@ struct AttnArgs {
 };
 
 __device__ __forceinline__ uint8_t* kv_k(uint8_t* sm, int s) {
-  return sm + kKVOff + s * 4 * kHalfBytes;
+  return sm + kKVOff + s * kStageBytes;
 }
 __device__ __forceinline__ uint8_t* kv_v(uint8_t* sm, int s) {
-  return sm + kKVOff + s * 4 * kHalfBytes + 2 * kHalfBytes;
+  return sm + kKVOff + s * kStageBytes + 2 * kKVHalf;
 }
 
 // Records the first error in the optional status word.
@@ -135,15 +140,16 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
 
   if (threadIdx.x == 0) {
     mbar_init(&T->q_full, 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kStages; ++s) {
       mbar_init(&T->kv_full[s], 1);
       mbar_init(&T->kv_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
       mbar_init(&T->s_full[s], 1);
       mbar_init(&T->s_empty[s], 4);
+      mbar_init(&T->p_empty[s], 1);
     }
     mbar_init(&T->p_full, 4);
-    mbar_init(&T->p_empty, 1);
-    mbar_init(&T->o_full, 1);
     mbar_init(&T->done, 1);
     T->abort = 0;
     fence_barrier_init();
@@ -178,7 +184,7 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     for (int w = 0; w < kMaskWords; ++w) T->anc[nl][w] = bits[w];
   }
   fence_proxy_async_smem();
-  if (warp == 1) tmem_alloc(&T->tmem_base, 512);
+  if (warp == 1) tmem_alloc(&T->tmem_base, 256);
   tc_fence_before_sync();
   __syncthreads();
   tc_fence_after_sync();
@@ -195,64 +201,66 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     tma_load_4d(sq + kHalfBytes, &tm_q, &T->q_full, 64, kvh * a.G, qt * a.npt, r);
     int issued = 0;
     for (int b = 0; b < nblk; ++b) {
-      const int s = b & 1;
-      if (b >= 2 && !mbar_wait_bounded(&T->kv_empty[s], ((b >> 1) - 1) & 1,
-                                       abort_v, kAttnLimitNs)) {
+      const int s = b % kStages;
+      if (b >= kStages && !mbar_wait_bounded(&T->kv_empty[s], ((b / kStages) - 1) & 1,
+                                             abort_v, kAttnLimitNs)) {
         *abort_v = 1;
         break;
       }
       const int key0 = (kb0 + b) * kBK;
-      mbar_arrive_expect_tx(&T->kv_full[s], 4u * kHalfBytes);
+      mbar_arrive_expect_tx(&T->kv_full[s], static_cast<uint32_t>(kStageBytes));
       tma_load_4d(kv_k(sm, s), &tm_k, &T->kv_full[s], 0, kvh, key0, r);
-      tma_load_4d(kv_k(sm, s) + kHalfBytes, &tm_k, &T->kv_full[s], 64, kvh, key0, r);
+      tma_load_4d(kv_k(sm, s) + kKVHalf, &tm_k, &T->kv_full[s], 64, kvh, key0, r);
       tma_load_4d(kv_v(sm, s), &tm_v, &T->kv_full[s], 0, kvh, key0, r);
-      tma_load_4d(kv_v(sm, s) + kHalfBytes, &tm_v, &T->kv_full[s], 64, kvh, key0, r);
+      tma_load_4d(kv_v(sm, s) + kKVHalf, &tm_v, &T->kv_full[s], 64, kvh, key0, r);
       ++issued;
     }
     // copies still in flight land before the CTA may exit
     (void)mbar_wait_bounded(&T->q_full, 0, abort_v, kAttnLimitNs);
-    for (int b = issued - 2 > 0 ? issued - 2 : 0; b < issued; ++b)
-      (void)mbar_wait_bounded(&T->kv_full[b & 1], (b >> 1) & 1, abort_v, kAttnLimitNs);
+    for (int b = issued - kStages > 0 ? issued - kStages : 0; b < issued; ++b)
+      (void)mbar_wait_bounded(&T->kv_full[b % kStages], (b / kStages) & 1, abort_v,
+                              kAttnLimitNs);
   } else if (warp == 1 && lane == 0 && nblk > 0) {
     // ---------------- MMA issuer ----------------
-    constexpr uint32_t idS = idesc_bf16_f32(128, 128);
+    constexpr uint32_t idS = idesc_bf16_f32(128, kBK);
     constexpr uint32_t idO = idesc_bf16_f32_bmn(128, 128);
     bool ok = mbar_wait_bounded(&T->q_full, 0, abort_v, kAttnLimitNs);
     const uint32_t q0 = smem_u32(sq), p0 = smem_u32(sp);
     auto issue_s = [&](int b) -> bool {
-      const int s = b & 1;
-      if (!mbar_wait_bounded(&T->kv_full[s], (b >> 1) & 1, abort_v, kAttnLimitNs))
+      const int s = b % kStages, sb = b & 1;
+      if (!mbar_wait_bounded(&T->kv_full[s], (b / kStages) & 1, abort_v, kAttnLimitNs))
         return false;
-      if (b >= 2 && !mbar_wait_bounded(&T->s_empty[s], ((b >> 1) - 1) & 1, abort_v,
+      if (b >= 2 && !mbar_wait_bounded(&T->s_empty[sb], ((b >> 1) - 1) & 1, abort_v,
                                        kAttnLimitNs))
         return false;
       tc_fence_after_sync();
       const uint32_t k0 = smem_u32(kv_k(sm, s));
 #pragma unroll
-      for (int kk = 0; kk < 8; ++kk) {
-        const uint32_t off = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-        tc_mma_bf16(tmem + s * 128, desc_kmajor_sw128(q0 + off),
-                    desc_kmajor_sw128(k0 + off), idS, kk > 0 ? 1u : 0u);
+      for (int kk = 0; kk < 8; ++kk) {        // 128 dims in steps of 16
+        tc_mma_bf16(tmem + sb * kBK,
+                    desc_kmajor_sw128(q0 + (kk >> 2) * kHalfBytes + (kk & 3) * 32),
+                    desc_kmajor_sw128(k0 + (kk >> 2) * kKVHalf + (kk & 3) * 32), idS,
+                    kk > 0 ? 1u : 0u);
       }
-      tc_commit(&T->s_full[s]);
+      tc_commit(&T->s_full[sb]);
       return true;
     };
     auto issue_o = [&](int b) -> bool {
-      const int s = b & 1;
+      const int s = b % kStages, pb = b & 1;
       if (!mbar_wait_bounded(&T->p_full, b & 1, abort_v, kAttnLimitNs)) return false;
       tc_fence_after_sync();
       const uint32_t v0 = smem_u32(kv_v(sm, s));
+      const uint32_t pa = p0 + pb * kPBytes;
 #pragma unroll
-      for (int kk = 0; kk < 8; ++kk) {
-        const uint32_t aoff = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-        // 16 keys = 16 rows of 128 B; the dims 64..127 half is kHalfBytes on
-        tc_mma_bf16(tmem + 256, desc_kmajor_sw128(p0 + aoff),
-                    desc_mnmajor_sw128(v0 + kk * 16 * 128, kHalfBytes, 1024), idO,
+      for (int kk = 0; kk < kBK / 16; ++kk) {
+        // A: P rows of 64 keys (128 B); B: 16 keys = 16 rows of 128 B, the
+        // dims 64..127 half kKVHalf further on
+        tc_mma_bf16(tmem + kOCol, desc_kmajor_sw128(pa + kk * 32),
+                    desc_mnmajor_sw128(v0 + kk * 16 * 128, kKVHalf, 1024), idO,
                     (b > 0 || kk > 0) ? 1u : 0u);   // O accumulates over blocks
       }
-      tc_commit(&T->o_full);
       tc_commit(&T->kv_empty[s]);
-      tc_commit(&T->p_empty);
+      tc_commit(&T->p_empty[pb]);
       return true;
     };
     if (ok) ok = issue_s(0);
@@ -287,39 +295,39 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
       return __all_sync(kFull, got);
     };
     for (int b = 0; b < nblk; ++b) {
-      const int sb = b & 1;
+      const int sb = b & 1, st = b % kStages;
       const int key0 = (kb0 + b) * kBK;
       if (!wwait(&T->s_full[sb], (b >> 1) & 1)) {
         ok = false;
         break;
       }
       tc_fence_after_sync();
-      float x[128];
+      float x[kBK];
       {
         uint32_t* xu = reinterpret_cast<uint32_t*>(x);
 #pragma unroll
-        for (int c = 0; c < 4; ++c)
-          tmem_ld_32x32b_x32(lane_base + sb * 128 + c * 32,
+        for (int c = 0; c < kBK / 32; ++c)
+          tmem_ld_32x32b_x32(lane_base + sb * kBK + c * 32,
                              *reinterpret_cast<uint32_t(*)[32]>(xu + c * 32));
         tmem_ld_wait();
       }
       tc_fence_before_sync();
       __syncwarp();
       if (lane == 0) mbar_arrive(&T->s_empty[sb]);   // S buffer free
-      // scaled scores; keys the row may not see become -inf
-      // (eight independent running maxima keep the dependency chains short)
+      // scaled scores; keys the row may not see become -inf (eight
+      // independent running maxima keep the dependency chains short)
       float m8[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u) m8[u] = -INFINITY;
       if (row_ok && key0 + kBK <= Tp) {      // a block of prefix keys only
 #pragma unroll
-        for (int j = 0; j < 128; ++j) {
+        for (int j = 0; j < kBK; ++j) {
           x[j] *= sc;
           m8[j & 7] = fmaxf(m8[j & 7], x[j]);
         }
       } else {
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+        for (int c = 0; c < kBK / 32; ++c) {
           const uint32_t al = row_ok ? allowed_bits(key0 + c * 32, Tp, anc) : 0u;
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
@@ -335,40 +343,46 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
       // cache held there; zero them so that 0 * (non-finite) cannot reach O
       const int valid = n_keys - key0;
       if (valid < kBK) {
-        if (!wwait(&T->kv_full[sb], (b >> 1) & 1)) {
+        if (!wwait(&T->kv_full[st], (b / kStages) & 1)) {
           ok = false;
           break;
         }
-        uint8_t* v = kv_v(sm, sb);
+        uint8_t* v = kv_v(sm, st);
         for (int i = t; i < 2 * (kBK - valid) * 8; i += 128) {
           const int half = i / ((kBK - valid) * 8), rem = i % ((kBK - valid) * 8);
-          *reinterpret_cast<uint4*>(v + half * kHalfBytes + (valid + rem / 8) * 128 +
+          *reinterpret_cast<uint4*>(v + half * kKVHalf + (valid + rem / 8) * 128 +
                                     (rem % 8) * 16) = make_uint4(0, 0, 0, 0);
         }
       }
-      // the PV product of the previous block has finished: P may be
-      // rewritten and O read
-      if (b >= 1 && !wwait(&T->p_empty, (b - 1) & 1)) {
+      // P buffer b & 1 was last read by the PV product of block b - 2
+      if (b >= 2 && !wwait(&T->p_empty[sb], ((b >> 1) - 1) & 1)) {
         ok = false;
         break;
       }
       // move the reference up where a row needs it; tcgen05.ld / st are
       // warp-collective, so the warp rescales together (alpha = 1 for rows
-      // that keep their reference)
+      // that keep their reference).  O must hold every block before b: the
+      // PV product of block b - 1 has to finish first (the one of block
+      // b - 3 on the same P buffer is known complete, so the phase is
+      // unambiguous).
       const bool mine = mx > m_used + 8.0f;
       const float alpha = mine ? ex2_approx(m_used - mx) : 1.0f;   // 0 from -inf
       if (__any_sync(kFull, mine)) {
         if (b >= 1) {
+          if (!wwait(&T->p_empty[(b - 1) & 1], ((b - 1) >> 1) & 1)) {
+            ok = false;
+            break;
+          }
           tc_fence_after_sync();
 #pragma unroll
           for (int c = 0; c < 4; ++c) {
             uint32_t y[32];
-            tmem_ld_32x32b_x32(lane_base + 256 + c * 32, y);
+            tmem_ld_32x32b_x32(lane_base + kOCol + c * 32, y);
             tmem_ld_wait();
 #pragma unroll
             for (int j = 0; j < 32; ++j)
               y[j] = __float_as_uint(__uint_as_float(y[j]) * alpha);
-            tmem_st_32x32b_x32(lane_base + 256 + c * 32, y);
+            tmem_st_32x32b_x32(lane_base + kOCol + c * 32, y);
           }
           tmem_st_wait();
         }
@@ -380,8 +394,9 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
       // P = 2^(s - m_used) in bf16, the A operand of the PV MMA
       const float mref = m_used == -INFINITY ? 0.0f : m_used;
       float ls[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+      uint8_t* pbuf = sp + sb * kPBytes;
 #pragma unroll
-      for (int c = 0; c < 16; ++c) {         // 8 keys = one 16-byte chunk
+      for (int c = 0; c < kBK / 8; ++c) {    // 8 keys = one 16-byte chunk
         uint32_t w[4];
 #pragma unroll
         for (int h = 0; h < 4; ++h) {
@@ -391,9 +406,7 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
           const __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
           w[h] = *reinterpret_cast<const uint32_t*>(&pb);
         }
-        const int half = c >> 3, chunk = c & 7;
-        *reinterpret_cast<uint4*>(sp + half * kHalfBytes + t * 128 +
-                                  ((chunk ^ (t & 7)) << 4)) =
+        *reinterpret_cast<uint4*>(pbuf + t * 128 + ((c ^ (t & 7)) << 4)) =
             make_uint4(w[0], w[1], w[2], w[3]);
       }
       l_sum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
@@ -402,7 +415,12 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
       __syncwarp();
       if (lane == 0) mbar_arrive(&T->p_full);
     }
-    if (ok && nblk > 0 && !wwait(&T->o_full, (nblk - 1) & 1)) ok = false;
+    // every PV product has finished: those of the last two blocks, one on
+    // each P buffer (earlier ones are known complete)
+    if (ok && nblk >= 2 && !wwait(&T->p_empty[(nblk - 2) & 1], ((nblk - 2) >> 1) & 1))
+      ok = false;
+    if (ok && nblk >= 1 && !wwait(&T->p_empty[(nblk - 1) & 1], ((nblk - 1) >> 1) & 1))
+      ok = false;
     if (!ok) {
       *abort_v = 1;
       report(a.status, PCTREE_ERR_TIMEOUT);
@@ -437,7 +455,7 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     auto load_chunk = [&](int c, float (&v)[32]) {
       if (nblk > 0) {
         uint32_t y[32];
-        tmem_ld_32x32b_x32(lane_base + 256 + c * 32, y);
+        tmem_ld_32x32b_x32(lane_base + kOCol + c * 32, y);
         tmem_ld_wait();
 #pragma unroll
         for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(y[j]);
@@ -478,7 +496,7 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
   tc_fence_after_sync();
   if (warp == 1) {
     __syncwarp();
-    tmem_dealloc(tmem, 512);
+    tmem_dealloc(tmem, 256);
   }
 }
 // Merges the key splits of every (request, KV head, tile) unit: one thread
@@ -501,9 +519,15 @@ tree_attn_merge_kernel(AttnArgs a) {
   if (row >= a.R || node >= a.N) return;
   const float2* ml = a.part_ml + static_cast<size_t>(unit) * a.n_split * 128 + row;
   float mstar = -INFINITY, lsum = 0.0f;
-  for (int s = 0; s < a.n_split; ++s) {
-    const float2 v = ml[static_cast<size_t>(s) * 128];
-    if (v.y > 0.0f) mstar = fmaxf(mstar, v.x);
+  for (int s0 = 0; s0 < a.n_split; s0 += 8) {   // eight loads in flight
+    float2 v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      v[u] = s0 + u < a.n_split ? ml[static_cast<size_t>(s0 + u) * 128]
+                                : make_float2(-INFINITY, 0.0f);
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      if (v[u].y > 0.0f) mstar = fmaxf(mstar, v[u].x);
   }
   float acc[16];
 #pragma unroll
