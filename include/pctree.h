@@ -380,6 +380,20 @@ PCTREE_API pctree_status pctree_profile_collect(int64_t* launches, double* total
 #define PCTREE_PATH_STAGEWISE 1
 PCTREE_API pctree_status pctree_set_path(int32_t path);
 
+/*
+ * Failure-detection test hook (the paper has no counterpart).  While
+ * `stage` >= 1, the fused round kernel withholds the cross-CTA release of
+ * that stage's parent rows, so every CTA's wait for it runs out after
+ * `wait_limit_ns`; the kernel then records PCTREE_ERR_TIMEOUT in
+ * out->status, drains its copies and MMAs, frees its tensor memory and
+ * returns, leaving the context usable.  `wait_limit_ns` bounds every wait
+ * of that kernel (1000 ns .. 10 s).  pctree_debug_stall_stage(-1,
+ * 1000000000) restores normal operation (no stall, 1 s bound).
+ * Process-wide, not thread-safe; returns PCTREE_ERR_INVALID_ARG for values
+ * out of range.
+ */
+PCTREE_API pctree_status pctree_debug_stall_stage(int32_t stage, int64_t wait_limit_ns);
+
 /* ABI version (major * 100 + minor). */
 PCTREE_API int32_t pctree_version(void);
 

@@ -96,6 +96,10 @@ using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t
                                    CUtensorMapFloatOOBfill);
 
 std::mutex g_mu;
+// Test hook (pctree_debug_stall_stage): a stage of the fused round whose
+// release is withheld, and the bound of every wait of that kernel.
+int g_stall_stage = -1;
+unsigned long long g_wait_limit_ns = 1000000000ull;
 EncodeTiledFn g_encode = nullptr;
 int g_num_sms[64] = {0};
 
@@ -237,6 +241,8 @@ pctree_status draft_fused(const pctree_config& c, const Layout& lay,
   a.cand_z = reinterpret_cast<float*>(ws + lay.off_fcz);
   a.cand_t = reinterpret_cast<int32_t*>(ws + lay.off_fct);
   a.status = out.status;
+  a.limit_ns = g_wait_limit_ns;
+  a.stall_stage = g_stall_stage;
   if (cudaMemsetAsync(out.status, 0, sizeof(int32_t), stream) != cudaSuccess ||
       cudaMemsetAsync(sync, 0, lay.sync_bytes, stream) != cudaSuccess)
     return PCTREE_ERR_CUDA;
@@ -377,6 +383,14 @@ pctree_status pctree_accept(const pctree_config* cfg, const pctree_tree* tree,
   return cuda_status(launch_accept(*cfg, *tree, target_tokens, accepted_idx,
                                    accepted_len, bonus_token,
                                    static_cast<cudaStream_t>(stream_ptr)));
+}
+
+pctree_status pctree_debug_stall_stage(int32_t stage, int64_t wait_limit_ns) {
+  if (stage < -1 || wait_limit_ns < 1000 || wait_limit_ns > 10000000000ll)
+    return PCTREE_ERR_INVALID_ARG;
+  g_stall_stage = stage;
+  g_wait_limit_ns = static_cast<unsigned long long>(wait_limit_ns);
+  return PCTREE_OK;
 }
 
 pctree_status pctree_set_path(int32_t path) {

@@ -59,6 +59,8 @@ struct FusedArgs {
   float* cand_z;         // [kFusedRows][grid][k] per-CTA top-k logits
   int32_t* cand_t;       // [kFusedRows][grid][k] per-CTA top-k tokens
   int32_t* status;
+  unsigned long long limit_ns;   // bound of every wait (1 s)
+  int stall_stage;       // test hook: stage whose release is withheld, or -1
 };
 
 // Pool id of the first node of level t (t >= 1).  Level 1 has k nodes, every

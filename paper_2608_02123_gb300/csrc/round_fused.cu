@@ -48,7 +48,6 @@ constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kStages = 8;
 constexpr int kTmemCols = 32;                    // two 16-column accumulators
 constexpr int kG = kFusedMaxGrid / 32;           // CTA groups of 32 in a merge
-constexpr uint64_t kLimitNs = 1000000000ull;     // 1 s per bounded wait
 constexpr float kNegInf = -INFINITY;
 
 template <int R>
@@ -57,6 +56,7 @@ struct FusedSmem {
   uint32_t tmem_slot;
   int abort;
   int ticket;
+  int stop;              // snapshot of abort the epilogue warps all act on
   float lv[kEpiWarps][R][kMaxKF];          // per-warp top-k lists per row
   int lt[kEpiWarps][R][kMaxKF];
   union {
@@ -115,6 +115,7 @@ __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
 #pragma unroll
   for (int s = 0; s < kStages; ++s) armed[s] = -1;
   int pend_stage[kStages], pend_kc[kStages];
+  int n_pend = 0;                 // slots waiting for this stage's parent rows
   bool ok = true;
   auto issue_rows = [&](int st, int kx) {
     tma_load_2d(ring + st * kStageBytes + kABytes, tmap_x, &S->full[st],
@@ -124,7 +125,7 @@ __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
 
   for (int d = 0; d < a.B && ok; ++d) {
     bool have = d == 0;   // stage 0 rows were written before the launch
-    int n_pend = 0;
+    n_pend = 0;
     for (int i = 0; i < n_my && ok; ++i) {
       const int tile = tile_at(d, i, n_my);
       for (int kc = 0; kc < a.n_k; ++kc) {
@@ -132,7 +133,7 @@ __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
           bool rdy = poll_flag(&a.ready[d]);
           if (!rdy && n_pend == kStages) {
             // ring full of slots waiting for the parent rows
-            if (!wait_flag_bounded(&a.ready[d], abort_v, kLimitNs)) {
+            if (!wait_flag_bounded(&a.ready[d], abort_v, a.limit_ns)) {
               ok = false;
               break;
             }
@@ -145,7 +146,7 @@ __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
             n_pend = 0;
           }
         }
-        if (!mbar_wait_bounded(&S->empty[stage], phase ^ 1u, abort_v, kLimitNs)) {
+        if (!mbar_wait_bounded(&S->empty[stage], phase ^ 1u, abort_v, a.limit_ns)) {
           ok = false;
           break;
         }
@@ -168,7 +169,7 @@ __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
       }
     }
     if (ok && !have) {
-      if (!wait_flag_bounded(&a.ready[d], abort_v, kLimitNs)) {
+      if (!wait_flag_bounded(&a.ready[d], abort_v, a.limit_ns)) {
         ok = false;
       } else {
         fence_proxy_async_global();
@@ -179,13 +180,17 @@ __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
   if (!ok) {
     *abort_v = 1;
     set_status(a.status, PCTREE_ERR_TIMEOUT);
+    // slots armed for W_out and a parent-row box that was never issued:
+    // load whatever the row buffer holds so that their barriers complete
+    fence_proxy_async_global();
+    for (int p = 0; p < n_pend; ++p) issue_rows(pend_stage[p], pend_kc[p]);
   }
   // every copy issued here must land before the CTA may exit
   volatile int never = 0;
   for (int s = 0; s < kStages; ++s)
     if (armed[s] >= 0)
       mbar_wait_bounded(&S->full[s], static_cast<uint32_t>(armed[s]), &never,
-                        kLimitNs);
+                        a.limit_ns);
 }
 
 // --------------------------------------------------------------------------
@@ -204,14 +209,14 @@ __device__ void mma(const FusedArgs& a, unsigned char* ring, FusedSmem<R>* S,
   bool ok = true;
   for (int d = 0; d < a.B && ok; ++d) {
     for (int i = 0; i < n_my && ok; ++i) {
-      if (!mbar_wait_bounded(&S->acc_empty[acc], acc_phase ^ 1u, abort_v, kLimitNs)) {
+      if (!mbar_wait_bounded(&S->acc_empty[acc], acc_phase ^ 1u, abort_v, a.limit_ns)) {
         ok = false;
         break;
       }
       tc_fence_after_sync();
       const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * kBN);
       for (int kc = 0; kc < a.n_k; ++kc) {
-        if (!mbar_wait_bounded(&S->full[stage], phase, abort_v, kLimitNs)) {
+        if (!mbar_wait_bounded(&S->full[stage], phase, abort_v, a.limit_ns)) {
           ok = false;
           break;
         }
@@ -242,7 +247,7 @@ __device__ void mma(const FusedArgs& a, unsigned char* ring, FusedSmem<R>* S,
   }
   tc_commit(&S->drain);
   volatile int never = 0;
-  mbar_wait_bounded(&S->drain, 0, &never, kLimitNs);
+  mbar_wait_bounded(&S->drain, 0, &never, a.limit_ns);
 }
 
 // --------------------------------------------------------------------------
@@ -400,7 +405,7 @@ __device__ void merge_stage(const CUtensorMap* tmap_w, const FusedArgs& a,
   fence_proxy_async_global();   // the rows are read with TMA by every CTA
   __threadfence();
   epi_barrier();
-  if (tid == 0) st_release_gpu(&a.ready[d + 1], 1);
+  if (tid == 0 && d + 1 != a.stall_stage) st_release_gpu(&a.ready[d + 1], 1);
 }
 
 // --------------------------------------------------------------------------
@@ -456,7 +461,9 @@ __device__ void epilogue(const CUtensorMap* tmap_w, const FusedArgs& a,
     for (int i = 0; i < n_my; ++i, ++g_tile) {
       if ((g_tile & 1) != grp) continue;
       const int tile = tile_at(d, i, n_my);
-      if (!mbar_wait_bounded(&S->acc_full[grp], acc_phase, abort_v, kLimitNs)) {
+      // the lanes agree before the warp-collective TMEM load
+      if (!__all_sync(kFull, mbar_wait_bounded(&S->acc_full[grp], acc_phase, abort_v,
+                                               a.limit_ns))) {
         ok = false;
         break;
       }
@@ -502,8 +509,13 @@ __device__ void epilogue(const CUtensorMap* tmap_w, const FusedArgs& a,
     if (!ok) {
       *abort_v = 1;
       set_status(a.status, PCTREE_ERR_TIMEOUT);
-      break;
     }
+    // one decision for all eight epilogue warps, which meet at named
+    // barriers below: a warp that gave up waits here for the others
+    epi_barrier();
+    if (tid == 0) S->stop = *abort_v;
+    epi_barrier();
+    if (S->stop) break;
     // per-thread (max, sum-exp) and per-warp lists to shared memory
 #pragma unroll
     for (int c = 0; c < R; ++c) {

@@ -108,6 +108,8 @@ def _load() -> ctypes.CDLL:
     lib.pctree_profile_collect.restype = ctypes.c_int
     lib.pctree_set_path.argtypes = [ctypes.c_int32]
     lib.pctree_set_path.restype = ctypes.c_int
+    lib.pctree_debug_stall_stage.argtypes = [ctypes.c_int32, ctypes.c_int64]
+    lib.pctree_debug_stall_stage.restype = ctypes.c_int
     lib.pctree_version.argtypes = []
     lib.pctree_version.restype = ctypes.c_int32
     return lib
@@ -422,3 +424,10 @@ class Drafter:
                                  "n_leaves", "status")}
         s.synchronize()
         return host
+
+
+def pctree_debug_stall_stage(stage: int, wait_limit_ns: int = 1_000_000_000) -> None:
+    """Failure-detection test hook (see include/pctree.h)."""
+    rc = LIB.pctree_debug_stall_stage(stage, wait_limit_ns)
+    if rc != PCTREE_OK:
+        raise PctreeError(rc, "pctree_debug_stall_stage")

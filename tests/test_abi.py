@@ -122,3 +122,11 @@ def test_compact_rejects_bad_layouts_on_the_host(P):
     # nothing to move: no planes and no hidden states
     assert call(variant(layers=0, hidden_bytes=0), cache=None, hin=None,
                 hout=None) == 0
+
+
+def test_stall_hook_argument_checks(P):
+    lib = P.LIB
+    assert lib.pctree_debug_stall_stage(-2, 10**9) == -1
+    assert lib.pctree_debug_stall_stage(1, 10) == -1
+    assert lib.pctree_debug_stall_stage(1, 2 * 10**10) == -1
+    assert lib.pctree_debug_stall_stage(-1, 10**9) == 0      # the default
