@@ -66,7 +66,9 @@ __global__ void init_kernel(const int32_t* __restrict__ root, const void* E_in,
 // partials: one CTA per (chunk of kChunk logits, row)
 // ---------------------------------------------------------------------------
 
-__global__ void __launch_bounds__(kChunkThreads)
+constexpr int kCandCap = 256;      // candidates a chunk may hold in shared memory
+
+__global__ void __launch_bounds__(kChunkThreads, 3)
 partials_kernel(const float* __restrict__ Z, int ldz, int V, int k,
                 int n_chunks, float* __restrict__ part_m,
                 float* __restrict__ part_s, float* __restrict__ part_z,
@@ -76,9 +78,10 @@ partials_kernel(const float* __restrict__ Z, int ldz, int V, int k,
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   constexpr int kWarps = kChunkThreads / 32;
-  __shared__ float sm_m[kWarps], sm_s[kWarps];
-  __shared__ float sm_v[kWarps][32];
-  __shared__ int sm_t[kWarps][32];
+  __shared__ float sm_m[kWarps], sm_s[kWarps], sm_kth[kWarps];
+  __shared__ float sm_v[kCandCap];
+  __shared__ int sm_t[kCandCap];
+  __shared__ int sm_count;
 
   const float* z_row = Z + static_cast<size_t>(row) * ldz;
   const int v0 = chunk * kChunk;
@@ -90,39 +93,44 @@ partials_kernel(const float* __restrict__ Z, int ldz, int V, int k,
     const int v = v0 + i * kChunkThreads + threadIdx.x;
     zs[i] = v < V ? z_row[v] : kNegInf;
   }
-  float m = kNegInf, s = 0.0f;
-  WarpList lst;
+  if (threadIdx.x == 0) sm_count = 0;
+  // this thread's max, then its sum of exp relative to it (no branches)
+  float tmax = kNegInf;
   bool bad = false;
 #pragma unroll
   for (int i = 0; i < kPer; ++i) {
-    const int v = v0 + i * kChunkThreads + threadIdx.x;
-    const bool in = v < V;
-    const float z = zs[i];
-    const int t = in ? v : 0x7fffffff;
-    if (in) {
-      bad |= is_nonfinite_logit(z);
-      lse_push(m, s, z);
-    }
-    if (i == 0) {
-      lst.seed(z, t, k);
-    } else {
-      lst.offer(z, t, k);
-    }
+    bad |= is_nonfinite_logit(zs[i]);
+    tmax = fmaxf(tmax, zs[i]);
+  }
+  float tsum = 0.0f;
+  if (tmax != kNegInf) {
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) tsum += __expf(zs[i] - tmax);
   }
   if (bad) set_status(status, PCTREE_ERR_NONFINITE);
-  // warp reduction of (m, s)
+  float m = tmax, s = tsum;
   for (int o = 16; o > 0; o >>= 1) {
     const float m2 = __shfl_xor_sync(kFull, m, o);
     const float s2 = __shfl_xor_sync(kFull, s, o);
     lse_merge(m, s, m2, s2);
   }
+  // a warp's k-th largest thread maximum bounds the chunk's k-th largest
+  // logit from below (k distinct threads hold a logit >= it), and so does
+  // the largest such value over the warps: only logits >= that floor can
+  // enter the chunk's top-k
+  WarpList lst;
+  lst.seed(tmax, threadIdx.x, k);
+  const float warp_kth = __shfl_sync(kFull, lst.v, k - 1);
   if (lane == 0) {
     sm_m[warp] = m;
     sm_s[warp] = s;
+    sm_kth[warp] = warp_kth;
   }
-  sm_v[warp][lane] = lst.v;
-  sm_t[warp][lane] = lst.t;
   __syncthreads();
+  float floor_z = sm_kth[0];
+#pragma unroll
+  for (int w = 1; w < kWarps; ++w) floor_z = fmaxf(floor_z, sm_kth[w]);
+  const size_t p = static_cast<size_t>(row) * n_chunks + chunk;
   if (warp == 0) {
     float mm = lane < kWarps ? sm_m[lane] : kNegInf;
     float ss = lane < kWarps ? sm_s[lane] : 0.0f;
@@ -131,17 +139,68 @@ partials_kernel(const float* __restrict__ Z, int ldz, int V, int k,
       const float s2 = __shfl_xor_sync(kFull, ss, o);
       lse_merge(mm, ss, m2, s2);
     }
-    // lane 0 keeps its own list; merge the other warps' lists into it
-    for (int w = 1; w < kWarps; ++w) {
-      const float cv = lane < k ? sm_v[w][lane] : kNegInf;
-      const int ct = lane < k ? sm_t[w][lane] : 0x7fffffff;
-      lst.offer(cv, ct, k);
-    }
-    const size_t p = static_cast<size_t>(row) * n_chunks + chunk;
     if (lane == 0) {
       part_m[p] = mm;
       part_s[p] = ss;
     }
+  }
+  // candidates (logits >= the floor) appended to shared memory, one atomic
+  // per warp and round
+#pragma unroll
+  for (int i = 0; i < kPer; ++i) {
+    const int v = v0 + i * kChunkThreads + threadIdx.x;
+    const bool pass = v < V && zs[i] >= floor_z;
+    const unsigned mask = __ballot_sync(kFull, pass);
+    if (mask) {
+      int base = 0;
+      if (lane == 0) base = atomicAdd(&sm_count, __popc(mask));
+      base = __shfl_sync(kFull, base, 0);
+      const int slot = base + __popc(mask & ((1u << lane) - 1u));
+      if (pass && slot < kCandCap) {
+        sm_v[slot] = zs[i];
+        sm_t[slot] = v;
+      }
+    }
+  }
+  __syncthreads();
+  const int count = sm_count;
+  if (count <= kCandCap) {
+    // rank of each candidate among the others (tokens are distinct)
+    for (int i = threadIdx.x; i < count; i += blockDim.x) {
+      const float cv = sm_v[i];
+      const int ct = sm_t[i];
+      int rank = 0;
+      for (int j = 0; j < count; ++j) rank += cand_better(sm_v[j], sm_t[j], cv, ct);
+      if (rank < k) {
+        part_z[p * k + rank] = cv;
+        part_t[p * k + rank] = ct;
+      }
+    }
+    // fewer candidates than k (a short last chunk): padding entries
+    for (int i = count + threadIdx.x; i < k; i += blockDim.x) {
+      part_z[p * k + i] = kNegInf;
+      part_t[p * k + i] = 0x7fffffff;
+    }
+    return;
+  }
+  // many logits at the floor (ties): every warp keeps a list of its
+  // candidates, warp 0 merges them
+  __syncthreads();
+  lst.reset();
+#pragma unroll
+  for (int i = 0; i < kPer; ++i) {
+    const int v = v0 + i * kChunkThreads + threadIdx.x;
+    const bool pass = v < V && zs[i] >= floor_z;
+    if (__any_sync(kFull, pass))
+      lst.offer(pass ? zs[i] : kNegInf, pass ? v : 0x7fffffff, k);
+  }
+  sm_v[warp * 32 + lane] = lst.v;
+  sm_t[warp * 32 + lane] = lst.t;
+  __syncthreads();
+  if (warp == 0) {
+    for (int w = 1; w < kWarps; ++w)
+      lst.offer(lane < k ? sm_v[w * 32 + lane] : kNegInf,
+                lane < k ? sm_t[w * 32 + lane] : 0x7fffffff, k);
     if (lane < k) {
       part_z[p * k + lane] = lst.v;
       part_t[p * k + lane] = lst.t;
