@@ -69,7 +69,7 @@ Layout make_layout(const pctree_config& c) {
   l.off_pool_par = take(static_cast<size_t>(c.batch) * l.P * sizeof(int32_t));
   l.off_pool_s = take(static_cast<size_t>(c.batch) * l.P * sizeof(float2));
   l.off_front = take(static_cast<size_t>(c.batch) * c.k * sizeof(int32_t));
-  l.sync_bytes = 2 * static_cast<size_t>(c.B) * sizeof(int);
+  l.sync_bytes = 2 * static_cast<size_t>(c.B) * sizeof(int);   // tickets, flags
   l.off_sync = take(l.sync_bytes);
   const size_t fparts = static_cast<size_t>(kFusedRows) * kFusedMaxGrid;
   l.off_fpm = take(fparts * sizeof(float));

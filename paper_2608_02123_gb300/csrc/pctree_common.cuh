@@ -196,8 +196,10 @@ __device__ __forceinline__ float warp_lse_from_partials(const float* pm,
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int c = c0 + u * 32 + lane;
-      mv[u] = c < n ? pm[c] : -INFINITY;
-      sv[u] = c < n ? ps[c] : 0.0f;
+      // written by other CTAs of a running kernel: read through L2, never
+      // from this SM's (non-coherent) L1
+      mv[u] = c < n ? __ldcg(pm + c) : -INFINITY;
+      sv[u] = c < n ? __ldcg(ps + c) : 0.0f;
     }
     float Mc = -INFINITY;
 #pragma unroll

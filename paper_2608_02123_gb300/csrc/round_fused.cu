@@ -287,8 +287,11 @@ __device__ void merge_stage(const CUtensorMap* tmap_w, const FusedArgs& a,
 #pragma unroll
     for (int u = 0; u < kG; ++u) {
       const int g = u * 32 + lane;
-      const float v = g < grid ? cz[static_cast<size_t>(g) * k] : kNegInf;
-      const int t = g < grid ? ct[static_cast<size_t>(g) * k] : 0x7fffffff;
+      // other CTAs wrote these during this launch: L2 loads (__ldcg), as
+      // for every cross-CTA read below -- this SM's L1 may still hold the
+      // same addresses from an earlier stage
+      const float v = g < grid ? __ldcg(cz + static_cast<size_t>(g) * k) : kNegInf;
+      const int t = g < grid ? __ldcg(ct + static_cast<size_t>(g) * k) : 0x7fffffff;
       sz[u][lane] = v;
       st[u][lane] = t;
     }
@@ -319,8 +322,8 @@ __device__ void merge_stage(const CUtensorMap* tmap_w, const FusedArgs& a,
         float v = kNegInf;
         int t = 0x7fffffff;
         if (g_lane >= 0) {
-          v = cz[static_cast<size_t>(g_lane) * k + r_lane];
-          t = ct[static_cast<size_t>(g_lane) * k + r_lane];
+          v = __ldcg(cz + static_cast<size_t>(g_lane) * k + r_lane);
+          t = __ldcg(ct + static_cast<size_t>(g_lane) * k + r_lane);
         }
         const bool ok = g_lane >= 0 && v >= T && t != 0x7fffffff;
         lst.offer(ok ? v : kNegInf, ok ? t : 0x7fffffff, k);
@@ -341,10 +344,10 @@ __device__ void merge_stage(const CUtensorMap* tmap_w, const FusedArgs& a,
     // the chain row's children go to every slot of the request.
     const int j_lo = a.shared ? 0 : j0, j_hi = a.shared ? b_d : j0 + 1;
     for (int j = j_lo; j < j_hi; ++j) {
-      const int pid = a.front[req * k + j];
+      const int pid = __ldcg(a.front + req * k + j);
       if (lane < k) {
         const int id = base + j * k + lane;
-        const float2 sn = ff_add(sc[pid], logpi);   // Eq. 4
+        const float2 sn = ff_add(__ldcg(sc + pid), logpi);   // Eq. 4
         tok[id] = t;
         par[id] = pid;
         sc[id] = sn;
@@ -507,6 +510,16 @@ __device__ void epilogue(const CUtensorMap* tmap_w, const FusedArgs& a,
       first = false;
     }
     if (!ok) {
+      *abort_v = 1;
+      set_status(a.status, PCTREE_ERR_TIMEOUT);
+    }
+    // The partials and candidate lists below overwrite those of stage d-1,
+    // which the last CTA of that stage may still be reading.  A CTA with
+    // tiles in this stage has already waited for the flag that merge
+    // releases after its reads (its parent rows needed it); check it here
+    // so the order holds for every CTA.
+    if (d > 0 && tid == 0 && !*abort_v &&
+        !wait_flag_bounded(&a.ready[d], abort_v, a.limit_ns)) {
       *abort_v = 1;
       set_status(a.status, PCTREE_ERR_TIMEOUT);
     }
