@@ -383,12 +383,25 @@ def run_ours(args, wl, rank, world, local_rank):
     P.pctree_profile_enable(True)
     start = torch.cuda.Event(enable_timing=True)
     end = torch.cuda.Event(enable_timing=True)
+    # per-step events (draft, accept) inside the bracketed timing, for the
+    # distribution of round times and the accept call on its own
+    marks = [[torch.cuda.Event(enable_timing=True) for _ in range(4)]
+             for _ in range(args.steps)]
     torch.cuda.synchronize()
     start.record(stream)
     for i in range(args.steps):
-        step(i)
+        m = marks[i]
+        m[0].record(stream)
+        dr.draft(L_dev[i % n_sets], E, W, root_dev[i % n_sets], stream)
+        m[1].record(stream)
+        tgt = target_of(i)
+        m[2].record(stream)
+        dr.accept(tgt, stream)
+        m[3].record(stream)
     end.record(stream)
     torch.cuda.synchronize()
+    draft_us = sorted(m[0].elapsed_time(m[1]) * 1e3 for m in marks)
+    accept_us = [m[2].elapsed_time(m[3]) * 1e3 for m in marks]
     launches, proj_ms = P.pctree_profile_collect()
     P.pctree_profile_enable(False)
     dr.check_status()
@@ -469,6 +482,10 @@ def run_ours(args, wl, rank, world, local_rank):
                      "launches": launches,
                      "avg_launch_us": proj_ms * 1e3 / launches if launches else None,
                      "traffic": recorded_traffic(wl, fused)},
+        "draft_us": {"p10": draft_us[len(draft_us) // 10],
+                     "p50": draft_us[len(draft_us) // 2],
+                     "p90": draft_us[(9 * len(draft_us)) // 10]},
+        "accept_us": statistics.mean(accept_us),
         "e2e": {"value": job_rounds_per_s(e2e_ms, args.steps, world, wl.batch),
                 "unit": "rounds/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
