@@ -198,7 +198,9 @@ markov_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
     uint32_t acc_phase = 0;
     bool bad = false;
     for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
-      if (!mbar_wait_bounded(&acc_full[acc], acc_phase, abort_v, kWaitLimitNs)) {
+      // the lanes agree before the warp-collective TMEM loads
+      if (!__all_sync(0xffffffffu, mbar_wait_bounded(&acc_full[acc], acc_phase, abort_v,
+                                                     kWaitLimitNs))) {
         *abort_v = 1;
         set_status(status, PCTREE_ERR_TIMEOUT);
         break;
