@@ -11,10 +11,14 @@
 //   warp 0      TMA producer: the Q tile once, then K and V blocks (64 keys
 //               x 128 dims, two 64-dim halves each, 128-byte swizzle) into a
 //               four-stage ring (three blocks in flight ahead of the MMA)
-//   warp 1      tcgen05.mma issuer: S_b = Q K_b^T into one of two TMEM
-//               buffers (M=128, N=64 keys, K=128 dims), then O += P_b V_b
-//               (M=128, N=128 dims, K=64 keys; V is the MN-major operand,
-//               dims contiguous) from one of two P buffers
+//   warp 1      S issuer: S_b = Q K_b^T (tcgen05.mma, M=128, N=64 keys,
+//               K=128 dims) into one of two TMEM buffers, up to two blocks
+//               ahead of the softmax
+//   warp 6      PV issuer: O += P_b V_b (M=128, N=128 dims, K=64 keys; V is
+//               the MN-major operand, dims contiguous) from one of two P
+//               buffers, as soon as the softmax has written P_b; its commit
+//               frees the K/V stage (S_b, the other reader, finished before
+//               the softmax could write P_b)
 //   warps 2..5  softmax, one thread per TMEM lane = tile row: each S row is
 //               read from TMEM once, masked and scaled; P = 2^(s - m_used)
 //               rounded to bf16 into shared memory (the K-major A operand of
@@ -23,7 +27,8 @@
 //               tcgen05.ld / st) only when a block's maximum exceeds it by
 //               more than 8 in log2 units, so P stays below 2^8.
 //
-// S of block b+1 is computed while the softmax works on block b.  Key blocks
+// S of blocks b+1 and b+2 is computed while the softmax works on block b:
+// two issuing threads keep the PV products off the S issue path.  Key blocks
 // of a request may be split over several CTAs (few requests, long
 // prefixes); each then writes (max, sum, unnormalised O) of its rows and a
 // second kernel merges the splits, spread over all SMs.  All waits are
@@ -36,7 +41,7 @@
 namespace pct {
 namespace {
 
-constexpr int kAttnThreads = 192;
+constexpr int kAttnThreads = 224;     // 7 warps, roles above
 constexpr int kBK = 64;                   // keys per block
 constexpr int kStages = 4;                // K/V ring depth
 constexpr int kHalfBytes = 128 * 128;     // Q: 128 rows x 64 bf16 (one dim half)
@@ -55,7 +60,7 @@ struct AttnTail {
   uint64_t q_full;
   uint64_t kv_full[kStages], kv_empty[kStages];
   uint64_t s_full[2], s_empty[2];
-  uint64_t p_full, p_empty[2], done;     // p_empty[i]: PV products of blocks i, i+2, ...
+  uint64_t p_full[2], p_empty[2], done;  // [i]: P / PV of blocks i, i+2, ...
   uint32_t tmem_base;
   int abort;
   int last;
@@ -147,10 +152,10 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     for (int s = 0; s < 2; ++s) {
       mbar_init(&T->s_full[s], 1);
       mbar_init(&T->s_empty[s], 4);
+      mbar_init(&T->p_full[s], 4);
       mbar_init(&T->p_empty[s], 1);
     }
-    mbar_init(&T->p_full, 4);
-    mbar_init(&T->done, 1);
+    mbar_init(&T->done, 2);              // one commit from each MMA issuer
     T->abort = 0;
     fence_barrier_init();
   }
@@ -221,18 +226,16 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
       (void)mbar_wait_bounded(&T->kv_full[b % kStages], (b / kStages) & 1, abort_v,
                               kAttnLimitNs);
   } else if (warp == 1 && lane == 0 && nblk > 0) {
-    // ---------------- MMA issuer ----------------
+    // ---------------- S issuer ----------------
     constexpr uint32_t idS = idesc_bf16_f32(128, kBK);
-    constexpr uint32_t idO = idesc_bf16_f32_bmn(128, 128);
     bool ok = mbar_wait_bounded(&T->q_full, 0, abort_v, kAttnLimitNs);
-    const uint32_t q0 = smem_u32(sq), p0 = smem_u32(sp);
-    auto issue_s = [&](int b) -> bool {
+    const uint32_t q0 = smem_u32(sq);
+    for (int b = 0; ok && b < nblk; ++b) {
       const int s = b % kStages, sb = b & 1;
-      if (!mbar_wait_bounded(&T->kv_full[s], (b / kStages) & 1, abort_v, kAttnLimitNs))
-        return false;
-      if (b >= 2 && !mbar_wait_bounded(&T->s_empty[sb], ((b >> 1) - 1) & 1, abort_v,
-                                       kAttnLimitNs))
-        return false;
+      ok = mbar_wait_bounded(&T->kv_full[s], (b / kStages) & 1, abort_v, kAttnLimitNs) &&
+           (b < 2 || mbar_wait_bounded(&T->s_empty[sb], ((b >> 1) - 1) & 1, abort_v,
+                                       kAttnLimitNs));
+      if (!ok) break;
       tc_fence_after_sync();
       const uint32_t k0 = smem_u32(kv_k(sm, s));
 #pragma unroll
@@ -243,11 +246,26 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
                     kk > 0 ? 1u : 0u);
       }
       tc_commit(&T->s_full[sb]);
-      return true;
-    };
-    auto issue_o = [&](int b) -> bool {
+    }
+    if (!ok) {
+      *abort_v = 1;
+      report(a.status, PCTREE_ERR_TIMEOUT);
+    }
+    tc_commit(&T->done);               // every MMA this thread issued has finished
+    (void)mbar_wait_bounded(&T->done, 0, abort_v, kAttnLimitNs);
+  } else if (warp == 6 && lane == 0 && nblk > 0) {
+    // ---------------- PV issuer ----------------
+    constexpr uint32_t idO = idesc_bf16_f32_bmn(128, 128);
+    const uint32_t p0 = smem_u32(sp);
+    bool ok = true;
+    for (int b = 0; b < nblk; ++b) {
       const int s = b % kStages, pb = b & 1;
-      if (!mbar_wait_bounded(&T->p_full, b & 1, abort_v, kAttnLimitNs)) return false;
+      // P_b, and with it S_b, is complete; the K/V stage is read by the PV
+      // product alone from here on
+      if (!mbar_wait_bounded(&T->p_full[pb], (b >> 1) & 1, abort_v, kAttnLimitNs)) {
+        ok = false;
+        break;
+      }
       tc_fence_after_sync();
       const uint32_t v0 = smem_u32(kv_v(sm, s));
       const uint32_t pa = p0 + pb * kPBytes;
@@ -261,19 +279,15 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
       }
       tc_commit(&T->kv_empty[s]);
       tc_commit(&T->p_empty[pb]);
-      return true;
-    };
-    if (ok) ok = issue_s(0);
-    for (int b = 1; ok && b < nblk; ++b) ok = issue_s(b) && issue_o(b - 1);
-    if (ok) ok = issue_o(nblk - 1);
+    }
     if (!ok) {
       *abort_v = 1;
       report(a.status, PCTREE_ERR_TIMEOUT);
     }
-    tc_commit(&T->done);               // every MMA issued above has finished
+    tc_commit(&T->done);
     (void)mbar_wait_bounded(&T->done, 0, abort_v, kAttnLimitNs);
   }
-  else if (warp >= 2) {
+  else if (warp >= 2 && warp < 6) {
     // ---------------- softmax, one thread per tile row ----------------
     // O accumulates in TMEM through the PV MMA with P = 2^(s - m_used); the
     // reference m_used moves (and O and l are rescaled in place) only when
@@ -413,7 +427,7 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
       tc_fence_before_sync();
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&T->p_full);
+      if (lane == 0) mbar_arrive(&T->p_full[sb]);
     }
     // every PV product has finished: those of the last two blocks, one on
     // each P buffer (earlier ones are known complete)
