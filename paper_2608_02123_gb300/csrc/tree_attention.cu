@@ -3,36 +3,42 @@
 // every drafted node attends to the verified prefix, itself and its
 // root-to-node ancestors.
 //
-// Work unit (one CTA): request r, KV head h, a tile of query rows and a range
-// of 64-key blocks.  The tile's rows are (node, query head of the group)
-// pairs, node-major: row t = node_local * G + g, R = G * nodes_per_tile <= 128.
-// The G query heads sharing KV head h read the same K/V blocks once.
+// Work unit (one CTA): request r, KV head h, one or two query tiles
+// (TILES) and a range of 64-key blocks.  A tile's rows are (node, query head
+// of the group) pairs, node-major: row t = node_local * G + g, R = G *
+// nodes_per_tile <= 128.  The G query heads sharing KV head h, and the
+// CTA's tiles, read each K/V block once.
 //
-//   warp 0      TMA producer: the Q tile once, then K and V blocks (64 keys
-//               x 128 dims, two 64-dim halves each, 128-byte swizzle) into a
-//               four-stage ring (three blocks in flight ahead of the MMA)
-//   warp 1      S issuer: S_b = Q K_b^T (tcgen05.mma, M=128, N=64 keys,
-//               K=128 dims) into one of two TMEM buffers, up to two blocks
-//               ahead of the softmax
-//   warp 6      PV issuer: O += P_b V_b (M=128, N=128 dims, K=64 keys; V is
-//               the MN-major operand, dims contiguous) from one of two P
-//               buffers, as soon as the softmax has written P_b; its commit
-//               frees the K/V stage (S_b, the other reader, finished before
-//               the softmax could write P_b)
-//   warps 2..5  softmax, one thread per TMEM lane = tile row: each S row is
-//               read from TMEM once, masked and scaled; P = 2^(s - m_used)
-//               rounded to bf16 into shared memory (the K-major A operand of
-//               the second MMA).  O accumulates in TMEM across blocks; the
-//               reference m_used rises (O and the row sum rescaled in place,
-//               tcgen05.ld / st) only when a block's maximum exceeds it by
-//               more than 8 in log2 units, so P stays below 2^8.
+//   warp 0      TMA producer: the Q tiles, then K and V blocks (64 keys x 128
+//               dims, two 64-dim halves each, 128-byte swizzle) into a ring
+//               (four stages for one tile, three for two); Q and the first
+//               blocks are issued before the rest of the set-up
+//   warp 1      S issuer: S_b = Q K_b^T for each tile (tcgen05.mma, M=128,
+//               N=64 keys, K=128 dims) into one of the tile's two TMEM
+//               buffers, up to two blocks ahead of its softmax
+//   warps 2..5  softmax of tile 0 (warps 6..9: tile 1): one thread per TMEM
+//               lane = tile row; each S row is read from TMEM once, masked
+//               and scaled; P = 2^(s - m_used) rounded to bf16 into a
+//               shared-memory P buffer (the K-major A operand of the second
+//               MMA).  O accumulates in TMEM across blocks; the reference
+//               m_used rises (O and the row sum rescaled in place, tcgen05.ld
+//               / st) only when a block's maximum exceeds it by more than 8
+//               in log2 units, so P stays below 2^8.
+//   last warp   PV issuer: O += P_b V_b per tile (M=128, N=128 dims, K=64
+//               keys; V is the MN-major operand, dims contiguous) as soon as
+//               the tile's P_b is written; after the CTA's tiles it frees the
+//               K/V stage (S_b, the other reader, finished before P_b existed)
 //
-// S of blocks b+1 and b+2 is computed while the softmax works on block b:
-// two issuing threads keep the PV products off the S issue path.  Key blocks
-// of a request may be split over several CTAs (few requests, long
-// prefixes); each then writes (max, sum, unnormalised O) of its rows and a
-// second kernel merges the splits, spread over all SMs.  All waits are
-// bounded (1 s) and end in PCTREE_ERR_TIMEOUT.
+// With two tiles each SM sub-partition runs one softmax warp of each, so one
+// tile's waits (TMEM loads, the PV product before its single P buffer is
+// rewritten) overlap the other's arithmetic, and the CTA set-up is paid once
+// per two tiles; TMEM then holds 2 x (two 64-column S buffers + a 128-column
+// O) = 512 columns.  One tile per CTA (chosen when two-tile CTAs would leave
+// SMs idle) double-buffers P instead.  Key blocks of a request may be split
+// over several CTAs (few requests, long prefixes); each then writes (max,
+// sum, unnormalised O) of its rows and a second kernel merges the splits,
+// spread over all SMs.  All waits are bounded (1 s) and end in
+// PCTREE_ERR_TIMEOUT.
 #include <cuda_bf16.h>
 
 #include "pctree_common.cuh"
@@ -41,34 +47,58 @@
 namespace pct {
 namespace {
 
-constexpr int kAttnThreads = 224;     // 7 warps, roles above
 constexpr int kBK = 64;                   // keys per block
-constexpr int kStages = 4;                // K/V ring depth
 constexpr int kHalfBytes = 128 * 128;     // Q: 128 rows x 64 bf16 (one dim half)
+constexpr int kQBytes = 2 * kHalfBytes;   // one Q tile
 constexpr int kKVHalf = kBK * 128;        // K or V: 64 keys x 64 bf16 (one dim half)
 constexpr int kStageBytes = 4 * kKVHalf;  // K (two halves) then V (two halves)
-constexpr int kPBytes = 128 * kBK * 2;    // P: 128 rows x 64 keys bf16
-constexpr int kQOff = 0;
-constexpr int kKVOff = 2 * kHalfBytes;
-constexpr int kPOff = kKVOff + kStages * kStageBytes;   // two P buffers
-constexpr int kTailOff = kPOff + 2 * kPBytes;
-constexpr uint32_t kOCol = 128;           // TMEM: S buffers at 0 and 64, O at 128
+constexpr int kPSub = 128 * 128;          // P: 128 rows x 64 keys bf16 (SW128)
+constexpr int kPBytes = kPSub * (kBK / 64);
 constexpr int kMaskWords = PCTREE_ATTN_MAX_N / 32;
 constexpr uint64_t kAttnLimitNs = 1000000000ull;
 
+// Layout of a CTA with TILES query tiles (1 or 2).  One tile: a four-stage
+// K/V ring and two P buffers, so P_b is written while the PV product of
+// block b-1 still runs.  Two tiles: a three-stage ring and one P buffer per
+// tile (the other tile's softmax covers that wait).
+template <int TILES>
+struct AttnCfg {
+  static constexpr int kThreads = 32 * (3 + 4 * TILES);   // roles above
+  static constexpr int kPVWarp = 2 + 4 * TILES;
+  static constexpr int kStages = TILES == 1 ? 4 : 3;
+  static constexpr int kNP = TILES == 1 ? 2 : 1;          // P buffers per tile
+  static constexpr int kQOff = 0;
+  static constexpr int kKVOff = TILES * kQBytes;
+  static constexpr int kPOff = kKVOff + kStages * kStageBytes;
+  static constexpr int kTailOff = kPOff + TILES * kNP * kPBytes;
+  // TMEM: tile j's two S buffers at columns (2j + sb) * kBK, its O (128
+  // columns) at kOCol + 128 j
+  static constexpr uint32_t kOCol = 2 * TILES * kBK;
+  static constexpr uint32_t kTmemCols = kOCol + 128 * TILES <= 256 ? 256 : 512;
+  static_assert(kOCol + 128 * TILES <= 512, "TMEM columns");
+};
+
+template <int TILES>
 struct AttnTail {
+  static constexpr int kStages = AttnCfg<TILES>::kStages, kNP = AttnCfg<TILES>::kNP;
   uint64_t q_full;
   uint64_t kv_full[kStages], kv_empty[kStages];
-  uint64_t s_full[2], s_empty[2];
-  uint64_t p_full[2], p_empty[2], done;  // [i]: P / PV of blocks i, i+2, ...
+  uint64_t s_full[TILES][2], s_empty[TILES][2];
+  uint64_t p_full[TILES][kNP], p_empty[TILES][kNP];   // P / PV of blocks pb, pb + kNP, ...
+  uint64_t done;
   uint32_t tmem_base;
   int abort;
-  int last;
-  uint32_t anc[128][kMaskWords];          // ancestor-or-self bits per node
+  int last[TILES];
+  uint32_t anc[TILES][128][kMaskWords];   // ancestor-or-self bits per node
   int32_t par[PCTREE_ATTN_MAX_N];         // the request's packed parents
 };
 
-constexpr size_t kAttnSmem = kTailOff + sizeof(AttnTail) + 1024;
+template <int TILES>
+constexpr size_t attn_smem() {
+  return AttnCfg<TILES>::kTailOff + sizeof(AttnTail<TILES>) + 1024;
+}
+static_assert(attn_smem<1>() <= 227 * 1024 && attn_smem<2>() <= 227 * 1024,
+              "shared memory per CTA");
 
 struct AttnArgs {
   const int32_t* prefix;
@@ -78,16 +108,9 @@ struct AttnArgs {
   float* part_o;          // [unit][split][128][128]
   float2* part_ml;        // [unit][split][128]  (max in log2 units, sum)
   int32_t* status;
-  int batch, N, Hq, Hkv, G, npt, R, nqt, max_slots, n_split, bps;
+  int batch, N, Hq, Hkv, G, npt, R, nqt, tpc, npair, max_slots, n_split, bps;
   float scale_log2;       // softmax scale * log2(e)
 };
-
-__device__ __forceinline__ uint8_t* kv_k(uint8_t* sm, int s) {
-  return sm + kKVOff + s * kStageBytes;
-}
-__device__ __forceinline__ uint8_t* kv_v(uint8_t* sm, int s) {
-  return sm + kKVOff + s * kStageBytes + 2 * kKVHalf;
-}
 
 // Records the first error in the optional status word.
 __device__ __forceinline__ void report(int32_t* status, int code) {
@@ -115,25 +138,33 @@ __device__ __forceinline__ uint32_t allowed_bits(int kc0, int T,
   return bits;
 }
 
-__global__ void __launch_bounds__(kAttnThreads, 1)
+template <int TILES>
+__global__ void __launch_bounds__(AttnCfg<TILES>::kThreads, 1)
 tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
                  const __grid_constant__ CUtensorMap tm_k,
                  const __grid_constant__ CUtensorMap tm_v, AttnArgs a) {
+  using C = AttnCfg<TILES>;
+  constexpr int kStages = C::kStages, kNP = C::kNP;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  AttnTail* T = reinterpret_cast<AttnTail*>(sm + kTailOff);
-  uint8_t* sq = sm + kQOff;
-  uint8_t* sp = sm + kPOff;
+  AttnTail<TILES>* T = reinterpret_cast<AttnTail<TILES>*>(sm + C::kTailOff);
+  uint8_t* sq = sm + C::kQOff;
+  uint8_t* sp = sm + C::kPOff;
+  // ring stage s: K (two dim halves) then V (two dim halves)
+  auto kv_k = [&](int s) { return sm + C::kKVOff + s * kStageBytes; };
+  auto kv_v = [&](int s) { return sm + C::kKVOff + s * kStageBytes + 2 * kKVHalf; };
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int qt = blockIdx.x % a.nqt, split = blockIdx.x / a.nqt;
+  const int pair = blockIdx.x % a.npair, split = blockIdx.x / a.npair;
   const int kvh = blockIdx.y, r = blockIdx.z;
+  const int qt0 = pair * a.tpc;                        // the CTA's first query tile
+  const int ntile = min(TILES, a.nqt - qt0);
 
   // request facts; a request with an impossible prefix or tree size is
   // reported and produces zero rows
   int Tp = a.prefix[r], n = a.n_nodes[r];
   if (Tp < 0 || n < 0 || n > a.N || static_cast<long long>(Tp) + n > a.max_slots) {
-    if (threadIdx.x == 0 && split == 0 && qt == 0 && kvh == 0)
+    if (threadIdx.x == 0 && split == 0 && pair == 0 && kvh == 0)
       report(a.status, PCTREE_ERR_INVALID_ARG);
     Tp = 0;
     n = 0;
@@ -143,38 +174,69 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
   const int kb0 = split * a.bps;
   const int nblk = max(0, min(kb0 + a.bps, nb_r) - kb0);
 
+  // K and V block b into ring stage b % kStages (producer thread only)
+  int issued = 0;
+  auto issue_kv = [&](int b) {
+    const int s = b % kStages, key0 = (kb0 + b) * kBK;
+    mbar_arrive_expect_tx(&T->kv_full[s], static_cast<uint32_t>(kStageBytes));
+    tma_load_4d(kv_k(s), &tm_k, &T->kv_full[s], 0, kvh, key0, r);
+    tma_load_4d(kv_k(s) + kKVHalf, &tm_k, &T->kv_full[s], 64, kvh, key0, r);
+    tma_load_4d(kv_v(s), &tm_v, &T->kv_full[s], 0, kvh, key0, r);
+    tma_load_4d(kv_v(s) + kKVHalf, &tm_v, &T->kv_full[s], 64, kvh, key0, r);
+  };
   if (threadIdx.x == 0) {
     mbar_init(&T->q_full, 1);
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&T->kv_full[s], 1);
       mbar_init(&T->kv_empty[s], 1);
     }
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(&T->s_full[s], 1);
-      mbar_init(&T->s_empty[s], 4);
-      mbar_init(&T->p_full[s], 4);
-      mbar_init(&T->p_empty[s], 1);
+    for (int j = 0; j < TILES; ++j) {
+      for (int s = 0; s < 2; ++s) {
+        mbar_init(&T->s_full[j][s], 1);
+        mbar_init(&T->s_empty[j][s], 4);
+      }
+      for (int pb = 0; pb < kNP; ++pb) {
+        mbar_init(&T->p_full[j][pb], 4);
+        mbar_init(&T->p_empty[j][pb], 1);
+      }
     }
     mbar_init(&T->done, 2);              // one commit from each MMA issuer
     T->abort = 0;
     fence_barrier_init();
+    if (nblk > 0) {
+      // the producer's first copies start now and overlap the rest of the
+      // set-up (ancestor bits, TMEM allocation)
+      tma_prefetch_desc(&tm_q);
+      tma_prefetch_desc(&tm_k);
+      tma_prefetch_desc(&tm_v);
+      mbar_arrive_expect_tx(&T->q_full,
+                            static_cast<uint32_t>(ntile) * 2u * static_cast<uint32_t>(a.R) * 128u);
+      for (int j = 0; j < ntile; ++j) {
+        const int node0 = (qt0 + j) * a.npt;
+        tma_load_4d(sq + j * kQBytes, &tm_q, &T->q_full, 0, kvh * a.G, node0, r);
+        tma_load_4d(sq + j * kQBytes + kHalfBytes, &tm_q, &T->q_full, 64, kvh * a.G, node0, r);
+      }
+      for (; issued < min(kStages, nblk); ++issued) issue_kv(issued);
+    }
   }
-  // rows R..127 of the Q tile are not loaded: zero them (read by the MMA)
-  for (int i = threadIdx.x; i < 2 * (128 - a.R) * 8; i += blockDim.x) {
-    const int half = i / ((128 - a.R) * 8), rem = i % ((128 - a.R) * 8);
-    *reinterpret_cast<uint4*>(sq + half * kHalfBytes + (a.R + rem / 8) * 128 +
+  // rows R..127 of each Q tile are not loaded: zero them (read by the MMA)
+  const int zq = (128 - a.R) * 8;                  // 16-byte chunks per half
+  for (int i = threadIdx.x; i < ntile * 2 * zq; i += blockDim.x) {
+    const int j = i / (2 * zq), half = (i / zq) & 1, rem = i % zq;
+    *reinterpret_cast<uint4*>(sq + j * kQBytes + half * kHalfBytes + (a.R + rem / 8) * 128 +
                               (rem % 8) * 16) = make_uint4(0, 0, 0, 0);
   }
-  // ancestor-or-self bits of the tile's nodes (walk up the packed parents,
+  // ancestor-or-self bits of the tiles' nodes (walk up the packed parents,
   // staged in shared memory)
   for (int i = threadIdx.x; i < n; i += blockDim.x)
     T->par[i] = a.parent[static_cast<size_t>(r) * a.N + i];
   __syncthreads();
-  for (int nl = threadIdx.x; nl < a.npt; nl += blockDim.x) {
+  for (int i = threadIdx.x; i < ntile * a.npt; i += blockDim.x) {
+    const int j = i / a.npt, nl = i - j * a.npt;
     uint32_t bits[kMaskWords];
 #pragma unroll
     for (int w = 0; w < kMaskWords; ++w) bits[w] = 0u;
-    int x = qt * a.npt + nl;
+    int x = (qt0 + j) * a.npt + nl;
     if (x < n) {
       const int32_t* par = T->par;
       for (int steps = 0; steps <= n && x >= 0 && x < n; ++steps) {
@@ -186,10 +248,10 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
       }
     }
 #pragma unroll
-    for (int w = 0; w < kMaskWords; ++w) T->anc[nl][w] = bits[w];
+    for (int w = 0; w < kMaskWords; ++w) T->anc[j][nl][w] = bits[w];
   }
   fence_proxy_async_smem();
-  if (warp == 1) tmem_alloc(&T->tmem_base, 256);
+  if (warp == 1) tmem_alloc(&T->tmem_base, C::kTmemCols);
   tc_fence_before_sync();
   __syncthreads();
   tc_fence_after_sync();
@@ -197,27 +259,15 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
   volatile int* abort_v = &T->abort;
 
   if (warp == 0 && lane == 0 && nblk > 0) {
-    // ---------------- TMA producer ----------------
-    tma_prefetch_desc(&tm_q);
-    tma_prefetch_desc(&tm_k);
-    tma_prefetch_desc(&tm_v);
-    mbar_arrive_expect_tx(&T->q_full, 2u * static_cast<uint32_t>(a.R) * 128u);
-    tma_load_4d(sq, &tm_q, &T->q_full, 0, kvh * a.G, qt * a.npt, r);
-    tma_load_4d(sq + kHalfBytes, &tm_q, &T->q_full, 64, kvh * a.G, qt * a.npt, r);
-    int issued = 0;
-    for (int b = 0; b < nblk; ++b) {
-      const int s = b % kStages;
-      if (b >= kStages && !mbar_wait_bounded(&T->kv_empty[s], ((b / kStages) - 1) & 1,
-                                             abort_v, kAttnLimitNs)) {
+    // ---------------- TMA producer (thread 0; Q and the first kStages
+    // blocks were issued during the set-up) ----------------
+    for (int b = issued; b < nblk; ++b) {
+      if (!mbar_wait_bounded(&T->kv_empty[b % kStages], ((b / kStages) - 1) & 1, abort_v,
+                             kAttnLimitNs)) {
         *abort_v = 1;
         break;
       }
-      const int key0 = (kb0 + b) * kBK;
-      mbar_arrive_expect_tx(&T->kv_full[s], static_cast<uint32_t>(kStageBytes));
-      tma_load_4d(kv_k(sm, s), &tm_k, &T->kv_full[s], 0, kvh, key0, r);
-      tma_load_4d(kv_k(sm, s) + kKVHalf, &tm_k, &T->kv_full[s], 64, kvh, key0, r);
-      tma_load_4d(kv_v(sm, s), &tm_v, &T->kv_full[s], 0, kvh, key0, r);
-      tma_load_4d(kv_v(sm, s) + kKVHalf, &tm_v, &T->kv_full[s], 64, kvh, key0, r);
+      issue_kv(b);
       ++issued;
     }
     // copies still in flight land before the CTA may exit
@@ -229,23 +279,28 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     // ---------------- S issuer ----------------
     constexpr uint32_t idS = idesc_bf16_f32(128, kBK);
     bool ok = mbar_wait_bounded(&T->q_full, 0, abort_v, kAttnLimitNs);
-    const uint32_t q0 = smem_u32(sq);
     for (int b = 0; ok && b < nblk; ++b) {
       const int s = b % kStages, sb = b & 1;
-      ok = mbar_wait_bounded(&T->kv_full[s], (b / kStages) & 1, abort_v, kAttnLimitNs) &&
-           (b < 2 || mbar_wait_bounded(&T->s_empty[sb], ((b >> 1) - 1) & 1, abort_v,
-                                       kAttnLimitNs));
-      if (!ok) break;
-      tc_fence_after_sync();
-      const uint32_t k0 = smem_u32(kv_k(sm, s));
+      ok = mbar_wait_bounded(&T->kv_full[s], (b / kStages) & 1, abort_v, kAttnLimitNs);
+      const uint32_t k0 = smem_u32(kv_k(s));
+      for (int j = 0; ok && j < ntile; ++j) {
+        // tile j's S buffer sb was last read by its softmax at block b - 2
+        if (b >= 2 && !mbar_wait_bounded(&T->s_empty[j][sb], ((b >> 1) - 1) & 1, abort_v,
+                                         kAttnLimitNs)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after_sync();
+        const uint32_t q0 = smem_u32(sq + j * kQBytes);
 #pragma unroll
-      for (int kk = 0; kk < 8; ++kk) {        // 128 dims in steps of 16
-        tc_mma_bf16(tmem + sb * kBK,
-                    desc_kmajor_sw128(q0 + (kk >> 2) * kHalfBytes + (kk & 3) * 32),
-                    desc_kmajor_sw128(k0 + (kk >> 2) * kKVHalf + (kk & 3) * 32), idS,
-                    kk > 0 ? 1u : 0u);
+        for (int kk = 0; kk < 8; ++kk) {      // 128 dims in steps of 16
+          tc_mma_bf16(tmem + (2 * j + sb) * kBK,
+                      desc_kmajor_sw128(q0 + (kk >> 2) * kHalfBytes + (kk & 3) * 32),
+                      desc_kmajor_sw128(k0 + (kk >> 2) * kKVHalf + (kk & 3) * 32), idS,
+                      kk > 0 ? 1u : 0u);
+        }
+        tc_commit(&T->s_full[j][sb]);
       }
-      tc_commit(&T->s_full[sb]);
     }
     if (!ok) {
       *abort_v = 1;
@@ -253,32 +308,35 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     }
     tc_commit(&T->done);               // every MMA this thread issued has finished
     (void)mbar_wait_bounded(&T->done, 0, abort_v, kAttnLimitNs);
-  } else if (warp == 6 && lane == 0 && nblk > 0) {
+  } else if (warp == C::kPVWarp && lane == 0 && nblk > 0) {
     // ---------------- PV issuer ----------------
     constexpr uint32_t idO = idesc_bf16_f32_bmn(128, 128);
-    const uint32_t p0 = smem_u32(sp);
     bool ok = true;
-    for (int b = 0; b < nblk; ++b) {
-      const int s = b % kStages, pb = b & 1;
-      // P_b, and with it S_b, is complete; the K/V stage is read by the PV
-      // product alone from here on
-      if (!mbar_wait_bounded(&T->p_full[pb], (b >> 1) & 1, abort_v, kAttnLimitNs)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after_sync();
-      const uint32_t v0 = smem_u32(kv_v(sm, s));
-      const uint32_t pa = p0 + pb * kPBytes;
+    for (int b = 0; ok && b < nblk; ++b) {
+      const int s = b % kStages;
+      const uint32_t v0 = smem_u32(kv_v(s));
+      const int pb = b % kNP;
+      for (int j = 0; j < ntile; ++j) {
+        // P_b of tile j, and with it S_b, is complete
+        if (!mbar_wait_bounded(&T->p_full[j][pb], (b / kNP) & 1, abort_v, kAttnLimitNs)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after_sync();
+        const uint32_t pa = smem_u32(sp + (j * kNP + pb) * kPBytes);
 #pragma unroll
-      for (int kk = 0; kk < kBK / 16; ++kk) {
-        // A: P rows of 64 keys (128 B); B: 16 keys = 16 rows of 128 B, the
-        // dims 64..127 half kKVHalf further on
-        tc_mma_bf16(tmem + kOCol, desc_kmajor_sw128(pa + kk * 32),
-                    desc_mnmajor_sw128(v0 + kk * 16 * 128, kKVHalf, 1024), idO,
-                    (b > 0 || kk > 0) ? 1u : 0u);   // O accumulates over blocks
+        for (int kk = 0; kk < kBK / 16; ++kk) {
+          // A: P rows of 64 keys (128 B); B: 16 keys = 16 rows of 128 B, the
+          // dims 64..127 half kKVHalf further on
+          tc_mma_bf16(tmem + C::kOCol + j * 128,
+                      desc_kmajor_sw128(pa + (kk >> 2) * kPSub + (kk & 3) * 32),
+                      desc_mnmajor_sw128(v0 + kk * 16 * 128, kKVHalf, 1024), idO,
+                      (b > 0 || kk > 0) ? 1u : 0u);   // O accumulates over blocks
+        }
+        tc_commit(&T->p_empty[j][pb]);
       }
-      tc_commit(&T->kv_empty[s]);
-      tc_commit(&T->p_empty[pb]);
+      // both tiles' S and PV products of block b have read the stage
+      if (ok) tc_commit(&T->kv_empty[s]);
     }
     if (!ok) {
       *abort_v = 1;
@@ -287,18 +345,21 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     tc_commit(&T->done);
     (void)mbar_wait_bounded(&T->done, 0, abort_v, kAttnLimitNs);
   }
-  else if (warp >= 2 && warp < 6) {
+  else if (warp >= 2 && warp < 2 + 4 * TILES && (warp - 2) / 4 < ntile) {
     // ---------------- softmax, one thread per tile row ----------------
     // O accumulates in TMEM through the PV MMA with P = 2^(s - m_used); the
     // reference m_used moves (and O and l are rescaled in place) only when
     // a block's maximum exceeds it by more than 2^8, so P stays <= 256.
+    const int j = (warp - 2) / 4;            // the tile of this warp
+    const int qt = qt0 + j;
     const int quad = warp & 3;               // TMEM lanes quad*32 .. +31
     const int t = quad * 32 + lane;          // tile row
     const int nl = t / a.G, g = t - nl * a.G;
     const int node = qt * a.npt + nl;
     const bool row_ok = t < a.R && node < n;
-    const uint32_t* anc = T->anc[nl < a.npt ? nl : 0];
+    const uint32_t* anc = T->anc[j][nl < a.npt ? nl : 0];
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+    const uint32_t s_col = lane_base + 2 * j * kBK, o_col = lane_base + C::kOCol + j * 128;
     const float sc = a.scale_log2;
     float m_used = -INFINITY, l_sum = 0.0f;  // O and l_sum are relative to m_used
     bool ok = true;
@@ -311,7 +372,7 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     for (int b = 0; b < nblk; ++b) {
       const int sb = b & 1, st = b % kStages;
       const int key0 = (kb0 + b) * kBK;
-      if (!wwait(&T->s_full[sb], (b >> 1) & 1)) {
+      if (!wwait(&T->s_full[j][sb], (b >> 1) & 1)) {
         ok = false;
         break;
       }
@@ -321,13 +382,13 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
         uint32_t* xu = reinterpret_cast<uint32_t*>(x);
 #pragma unroll
         for (int c = 0; c < kBK / 32; ++c)
-          tmem_ld_32x32b_x32(lane_base + sb * kBK + c * 32,
+          tmem_ld_32x32b_x32(s_col + sb * kBK + c * 32,
                              *reinterpret_cast<uint32_t(*)[32]>(xu + c * 32));
         tmem_ld_wait();
       }
       tc_fence_before_sync();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&T->s_empty[sb]);   // S buffer free
+      if (lane == 0) mbar_arrive(&T->s_empty[j][sb]);   // S buffer free
       // scaled scores; keys the row may not see become -inf (eight
       // independent running maxima keep the dependency chains short)
       float m8[8];
@@ -335,55 +396,58 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
       for (int u = 0; u < 8; ++u) m8[u] = -INFINITY;
       if (row_ok && key0 + kBK <= Tp) {      // a block of prefix keys only
 #pragma unroll
-        for (int j = 0; j < kBK; ++j) {
-          x[j] *= sc;
-          m8[j & 7] = fmaxf(m8[j & 7], x[j]);
+        for (int k2 = 0; k2 < kBK; ++k2) {
+          x[k2] *= sc;
+          m8[k2 & 7] = fmaxf(m8[k2 & 7], x[k2]);
         }
       } else {
 #pragma unroll
         for (int c = 0; c < kBK / 32; ++c) {
           const uint32_t al = row_ok ? allowed_bits(key0 + c * 32, Tp, anc) : 0u;
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const float v = ((al >> j) & 1u) ? x[c * 32 + j] * sc : -INFINITY;
-            x[c * 32 + j] = v;
-            m8[j & 7] = fmaxf(m8[j & 7], v);
+          for (int k2 = 0; k2 < 32; ++k2) {
+            const float v = ((al >> k2) & 1u) ? x[c * 32 + k2] * sc : -INFINITY;
+            x[c * 32 + k2] = v;
+            m8[k2 & 7] = fmaxf(m8[k2 & 7], v);
           }
         }
       }
       const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
                              fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
       // the last block of the request: V rows past the tree hold whatever the
-      // cache held there; zero them so that 0 * (non-finite) cannot reach O
+      // cache held there; zero them so that 0 * (non-finite) cannot reach O.
+      // Both tiles' warps do it: each tile's PV product then reads rows its
+      // own warps zeroed and fenced, and the other tile only ever writes the
+      // same zero bytes there.
       const int valid = n_keys - key0;
       if (valid < kBK) {
         if (!wwait(&T->kv_full[st], (b / kStages) & 1)) {
           ok = false;
           break;
         }
-        uint8_t* v = kv_v(sm, st);
+        uint8_t* v = kv_v(st);
         for (int i = t; i < 2 * (kBK - valid) * 8; i += 128) {
           const int half = i / ((kBK - valid) * 8), rem = i % ((kBK - valid) * 8);
           *reinterpret_cast<uint4*>(v + half * kKVHalf + (valid + rem / 8) * 128 +
                                     (rem % 8) * 16) = make_uint4(0, 0, 0, 0);
         }
       }
-      // P buffer b & 1 was last read by the PV product of block b - 2
-      if (b >= 2 && !wwait(&T->p_empty[sb], ((b >> 1) - 1) & 1)) {
+      // P buffer pbi was last read by the PV product of block b - kNP
+      const int pbi = b % kNP;
+      if (b >= kNP && !wwait(&T->p_empty[j][pbi], ((b / kNP) - 1) & 1)) {
         ok = false;
         break;
       }
       // move the reference up where a row needs it; tcgen05.ld / st are
       // warp-collective, so the warp rescales together (alpha = 1 for rows
-      // that keep their reference).  O must hold every block before b: the
-      // PV product of block b - 1 has to finish first (the one of block
-      // b - 3 on the same P buffer is known complete, so the phase is
-      // unambiguous).
+      // that keep their reference)
       const bool mine = mx > m_used + 8.0f;
       const float alpha = mine ? ex2_approx(m_used - mx) : 1.0f;   // 0 from -inf
       if (__any_sync(kFull, mine)) {
         if (b >= 1) {
-          if (!wwait(&T->p_empty[(b - 1) & 1], ((b - 1) >> 1) & 1)) {
+          // O must hold every block before b: the PV product of block b - 1
+          // has finished (with one P buffer, the wait above saw to that)
+          if (kNP > 1 && !wwait(&T->p_empty[j][(b - 1) % kNP], ((b - 1) / kNP) & 1)) {
             ok = false;
             break;
           }
@@ -391,12 +455,12 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
 #pragma unroll
           for (int c = 0; c < 4; ++c) {
             uint32_t y[32];
-            tmem_ld_32x32b_x32(lane_base + kOCol + c * 32, y);
+            tmem_ld_32x32b_x32(o_col + c * 32, y);
             tmem_ld_wait();
 #pragma unroll
-            for (int j = 0; j < 32; ++j)
-              y[j] = __float_as_uint(__uint_as_float(y[j]) * alpha);
-            tmem_st_32x32b_x32(lane_base + kOCol + c * 32, y);
+            for (int k2 = 0; k2 < 32; ++k2)
+              y[k2] = __float_as_uint(__uint_as_float(y[k2]) * alpha);
+            tmem_st_32x32b_x32(o_col + c * 32, y);
           }
           tmem_st_wait();
         }
@@ -408,7 +472,7 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
       // P = 2^(s - m_used) in bf16, the A operand of the PV MMA
       const float mref = m_used == -INFINITY ? 0.0f : m_used;
       float ls[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-      uint8_t* pbuf = sp + sb * kPBytes;
+      uint8_t* pbuf = sp + (j * kNP + pbi) * kPBytes;
 #pragma unroll
       for (int c = 0; c < kBK / 8; ++c) {    // 8 keys = one 16-byte chunk
         uint32_t w[4];
@@ -420,32 +484,30 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
           const __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
           w[h] = *reinterpret_cast<const uint32_t*>(&pb);
         }
-        *reinterpret_cast<uint4*>(pbuf + t * 128 + ((c ^ (t & 7)) << 4)) =
+        *reinterpret_cast<uint4*>(pbuf + (c >> 3) * kPSub + t * 128 + (((c & 7) ^ (t & 7)) << 4)) =
             make_uint4(w[0], w[1], w[2], w[3]);
       }
       l_sum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
       tc_fence_before_sync();
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&T->p_full[sb]);
+      if (lane == 0) mbar_arrive(&T->p_full[j][pbi]);
     }
-    // every PV product has finished: those of the last two blocks, one on
-    // each P buffer (earlier ones are known complete)
-    if (ok && nblk >= 2 && !wwait(&T->p_empty[(nblk - 2) & 1], ((nblk - 2) >> 1) & 1))
-      ok = false;
-    if (ok && nblk >= 1 && !wwait(&T->p_empty[(nblk - 1) & 1], ((nblk - 1) >> 1) & 1))
-      ok = false;
+    // every PV product of the tile has finished: the last one on each P
+    // buffer (earlier ones are known complete)
+    for (int bb = nblk - kNP > 0 ? nblk - kNP : 0; ok && bb < nblk; ++bb)
+      if (!wwait(&T->p_empty[j][bb % kNP], (bb / kNP) & 1)) ok = false;
     if (!ok) {
       *abort_v = 1;
       report(a.status, PCTREE_ERR_TIMEOUT);
     }
-    // one decision for all four softmax warps (they meet at named barriers
-    // below, which must see every one of them)
-    named_barrier(1, 128);
-    if (t == 0) T->last = *abort_v;
-    named_barrier(1, 128);
-    ok = T->last == 0;
-    named_barrier(1, 128);
+    // one decision for the tile's four softmax warps (they meet at named
+    // barriers below, which must see every one of them)
+    named_barrier(1 + j, 128);
+    if (t == 0) T->last[j] = *abort_v;
+    named_barrier(1 + j, 128);
+    ok = T->last[j] == 0;
+    named_barrier(1 + j, 128);
     tc_fence_after_sync();
     // ---------------- output ----------------
     // O is read from TMEM in four 32-column chunks; tcgen05.ld is
@@ -469,13 +531,13 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     auto load_chunk = [&](int c, float (&v)[32]) {
       if (nblk > 0) {
         uint32_t y[32];
-        tmem_ld_32x32b_x32(lane_base + kOCol + c * 32, y);
+        tmem_ld_32x32b_x32(o_col + c * 32, y);
         tmem_ld_wait();
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(y[j]);
+        for (int k2 = 0; k2 < 32; ++k2) v[k2] = __uint_as_float(y[k2]);
       } else {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+        for (int k2 = 0; k2 < 32; ++k2) v[k2] = 0.0f;
       }
     };
     if (a.n_split == 1) {
@@ -510,7 +572,7 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
   tc_fence_after_sync();
   if (warp == 1) {
     __syncwarp();
-    tmem_dealloc(tmem, 256);
+    tmem_dealloc(tmem, C::kTmemCols);
   }
 }
 // Merges the key splits of every (request, KV head, tile) unit: one thread
@@ -604,8 +666,8 @@ namespace {
 // (request, KV head, tile) units; they depend only on the configuration, so
 // the workspace size does too.
 struct AttnGeom {
-  int G, npt, R, nqt, nb_max, n_split, bps;
-  long long units;
+  int G, npt, R, nqt, tpc, npair, nb_max, n_split, bps;
+  long long units;                    // (request, KV head, query tile) triples
 };
 
 AttnGeom attn_geom(const pctree_attn_config& c) {
@@ -614,9 +676,16 @@ AttnGeom attn_geom(const pctree_attn_config& c) {
   g.npt = 128 / g.G < c.N ? 128 / g.G : c.N;
   g.R = g.G * g.npt;
   g.nqt = (c.N + g.npt - 1) / g.npt;
+  // two tiles per CTA once such CTAs still fill every SM: the set-up is then
+  // paid once per two tiles and their softmax waits overlap; otherwise one
+  // tile per CTA keeps more SMs busy
+  const long long pairs = static_cast<long long>(c.batch) * c.Hkv * ((g.nqt + 1) / 2);
+  g.tpc = (g.nqt >= 2 && pairs >= 152) ? 2 : 1;
+  g.npair = (g.nqt + g.tpc - 1) / g.tpc;
   g.units = static_cast<long long>(c.batch) * c.Hkv * g.nqt;
   g.nb_max = (c.max_slots + kBK - 1) / kBK;
-  long long want = (152 + g.units - 1) / g.units;
+  const long long ctas = static_cast<long long>(c.batch) * c.Hkv * g.npair;
+  long long want = (152 + ctas - 1) / ctas;
   if (want > g.nb_max) want = g.nb_max;
   if (want < 1) want = 1;
   g.bps = static_cast<int>((g.nb_max + want - 1) / want);
@@ -634,7 +703,7 @@ pctree_status attn_check(const pctree_attn_config* c) {
       c->batch > 65535 || c->Hkv > 65535)
     return PCTREE_ERR_UNSUPPORTED;
   const AttnGeom g = attn_geom(*c);
-  if (static_cast<long long>(g.nqt) * g.n_split > 0x7fffffffll)
+  if (static_cast<long long>(g.npair) * g.n_split > 0x7fffffffll)
     return PCTREE_ERR_UNSUPPORTED;
   return PCTREE_OK;
 }
@@ -726,6 +795,8 @@ pctree_status pctree_tree_attention(const pctree_attn_config* cfg, const void* q
   a.npt = g.npt;
   a.R = g.R;
   a.nqt = g.nqt;
+  a.tpc = g.tpc;
+  a.npair = g.npair;
   a.max_slots = c.max_slots;
   a.n_split = g.n_split;
   a.bps = g.bps;
@@ -740,14 +811,19 @@ pctree_status pctree_tree_attention(const pctree_attn_config* cfg, const void* q
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return PCTREE_ERR_CUDA;
   if (!attr_set[dev]) {
-    if (cudaFuncSetAttribute(tree_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(kAttnSmem)) != cudaSuccess)
+    if (cudaFuncSetAttribute(tree_attn_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(attn_smem<1>())) != cudaSuccess ||
+        cudaFuncSetAttribute(tree_attn_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(attn_smem<2>())) != cudaSuccess)
       return PCTREE_ERR_CUDA;
     attr_set[dev] = true;
   }
-  const dim3 grid(static_cast<unsigned>(g.nqt * g.n_split), static_cast<unsigned>(c.Hkv),
+  const dim3 grid(static_cast<unsigned>(g.npair * g.n_split), static_cast<unsigned>(c.Hkv),
                   static_cast<unsigned>(c.batch));
-  tree_attn_kernel<<<grid, kAttnThreads, kAttnSmem, stream>>>(tm_q, tm_k, tm_v, a);
+  if (g.tpc == 2)
+    tree_attn_kernel<2><<<grid, AttnCfg<2>::kThreads, attn_smem<2>(), stream>>>(tm_q, tm_k, tm_v, a);
+  else
+    tree_attn_kernel<1><<<grid, AttnCfg<1>::kThreads, attn_smem<1>(), stream>>>(tm_q, tm_k, tm_v, a);
   if (cudaGetLastError() != cudaSuccess) return PCTREE_ERR_CUDA;
   if (g.n_split > 1) {
     const dim3 mgrid(static_cast<unsigned>(g.units), (g.R + kMergeRows - 1) / kMergeRows);
