@@ -112,6 +112,15 @@ struct AttnArgs {
   float scale_log2;       // softmax scale * log2(e)
 };
 
+// 32 lanes x 8 columns of 32-bit TMEM words from registers: thread t of the
+// warp writes lane (taddr.lane + t), columns taddr.col .. +7.
+__device__ __forceinline__ void tmem_st_32x32b_x8(uint32_t taddr, const uint32_t (&r)[8]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+      : "memory");
+}
+
 // Records the first error in the optional status word.
 __device__ __forceinline__ void report(int32_t* status, int code) {
   if (status != nullptr) atomicCAS(status, 0, code);
@@ -452,15 +461,16 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
             break;
           }
           tc_fence_after_sync();
-#pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            uint32_t y[32];
-            tmem_ld_32x32b_x32(o_col + c * 32, y);
+          // eight columns at a time: the block's scores stay live meanwhile
+#pragma unroll 4
+          for (int c = 0; c < 16; ++c) {
+            uint32_t y[8];
+            tmem_ld_32x32b_x8(o_col + c * 8, y);
             tmem_ld_wait();
 #pragma unroll
-            for (int k2 = 0; k2 < 32; ++k2)
+            for (int k2 = 0; k2 < 8; ++k2)
               y[k2] = __float_as_uint(__uint_as_float(y[k2]) * alpha);
-            tmem_st_32x32b_x32(o_col + c * 32, y);
+            tmem_st_32x32b_x8(o_col + c * 8, y);
           }
           tmem_st_wait();
         }
