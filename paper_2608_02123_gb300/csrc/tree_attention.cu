@@ -3,42 +3,48 @@
 // every drafted node attends to the verified prefix, itself and its
 // root-to-node ancestors.
 //
-// Work unit (one CTA): request r, KV head h, one or two query tiles
-// (TILES) and a range of 64-key blocks.  A tile's rows are (node, query head
-// of the group) pairs, node-major: row t = node_local * G + g, R = G *
-// nodes_per_tile <= 128.  The G query heads sharing KV head h, and the
-// CTA's tiles, read each K/V block once.
+// Work items: request r, KV head h, one or two query tiles (TILES) and a
+// range of 64-key blocks.  A tile's rows are (node, query head of the group)
+// pairs, node-major: row t = node_local * G + g, R = G * nodes_per_tile <=
+// 128.  The G query heads sharing KV head h, and an item's tiles, read each
+// K/V block once.  The kernel is persistent: one CTA per SM takes items in
+// rounds of gridDim.x, forwards and backwards in turn, over a list ordered by
+// decreasing request length (longest first keeps the last round short), so
+// its set-up (barriers, TMEM) is paid once and the next item's loads and S
+// products overlap the current item's last blocks and output.
 //
-//   warp 0      TMA producer: the Q tiles, then K and V blocks (64 keys x 128
-//               dims, two 64-dim halves each, 128-byte swizzle) into a ring
-//               (four stages for one tile, three for two); Q and the first
-//               blocks are issued before the rest of the set-up
-//   warp 1      S issuer: S_b = Q K_b^T for each tile (tcgen05.mma, M=128,
-//               N=64 keys, K=128 dims) into one of the tile's two TMEM
+//   warp 0      TMA producer: K and V blocks (64 keys x 128 dims, two 64-dim
+//               halves each, 128-byte swizzle) into a ring (four stages for
+//               one tile, three for two) that runs on across items
+//   warp 1      S issuer: each item's Q tiles (once the previous item's S
+//               products are done), then S_b = Q K_b^T per tile (tcgen05.mma,
+//               M=128, N=64 keys, K=128 dims) into one of the tile's two TMEM
 //               buffers, up to two blocks ahead of its softmax
-//   warps 2..5  softmax of tile 0 (warps 6..9: tile 1): one thread per TMEM
-//               lane = tile row; each S row is read from TMEM once, masked
-//               and scaled; P = 2^(s - m_used) rounded to bf16 into a
+//   warps 2..5  softmax and output of tile 0 (warps 6..9: tile 1): one thread
+//               per TMEM lane = tile row; each S row is read from TMEM once,
+//               masked and scaled; P = 2^(s - m_used) rounded to bf16 into a
 //               shared-memory P buffer (the K-major A operand of the second
-//               MMA).  O accumulates in TMEM across blocks; the reference
-//               m_used rises (O and the row sum rescaled in place, tcgen05.ld
-//               / st) only when a block's maximum exceeds it by more than 8
-//               in log2 units, so P stays below 2^8.
-//   last warp   PV issuer: O += P_b V_b per tile (M=128, N=128 dims, K=64
+//               MMA).  O accumulates in TMEM across an item's blocks; the
+//               reference m_used rises (O and the row sum rescaled in place,
+//               tcgen05.ld / st) only when a block's maximum exceeds it by
+//               more than 8 in log2 units, so P stays below 2^8.  After the
+//               item's last block the same warps normalise O and store it.
+//   next warp   PV issuer: O += P_b V_b per tile (M=128, N=128 dims, K=64
 //               keys; V is the MN-major operand, dims contiguous) as soon as
-//               the tile's P_b is written; after the CTA's tiles it frees the
+//               the tile's P_b is written; after the item's tiles it frees the
 //               K/V stage (S_b, the other reader, finished before P_b existed)
+//   last warp   ancestor bits: the next item's ancestor-or-self masks (from
+//               the packed parents) into the second of two buffers
 //
 // With two tiles each SM sub-partition runs one softmax warp of each, so one
 // tile's waits (TMEM loads, the PV product before its single P buffer is
-// rewritten) overlap the other's arithmetic, and the CTA set-up is paid once
-// per two tiles; TMEM then holds 2 x (two 64-column S buffers + a 128-column
-// O) = 512 columns.  One tile per CTA (chosen when two-tile CTAs would leave
-// SMs idle) double-buffers P instead.  Key blocks of a request may be split
-// over several CTAs (few requests, long prefixes); each then writes (max,
-// sum, unnormalised O) of its rows and a second kernel merges the splits,
-// spread over all SMs.  All waits are bounded (1 s) and end in
-// PCTREE_ERR_TIMEOUT.
+// rewritten) overlap the other's arithmetic; TMEM then holds 2 x (two
+// 64-column S buffers + a 128-column O) = 512 columns.  One tile per item
+// (chosen when two-tile items would leave SMs idle) double-buffers P
+// instead.  Key blocks of a request may be split over several items (few
+// requests, long prefixes); each then writes (max, sum, unnormalised O) of
+// its rows and a second kernel merges the splits, spread over all SMs.  All
+// waits are bounded (1 s) and end in PCTREE_ERR_TIMEOUT.
 #include <cuda_bf16.h>
 
 #include "pctree_common.cuh"
@@ -57,14 +63,17 @@ constexpr int kPBytes = kPSub * (kBK / 64);
 constexpr int kMaskWords = PCTREE_ATTN_MAX_N / 32;
 constexpr uint64_t kAttnLimitNs = 1000000000ull;
 
+constexpr int kMaxOrder = 256;            // requests ordered by length in shared memory
+
 // Layout of a CTA with TILES query tiles (1 or 2).  One tile: a four-stage
 // K/V ring and two P buffers, so P_b is written while the PV product of
 // block b-1 still runs.  Two tiles: a three-stage ring and one P buffer per
 // tile (the other tile's softmax covers that wait).
 template <int TILES>
 struct AttnCfg {
-  static constexpr int kThreads = 32 * (3 + 4 * TILES);   // roles above
+  static constexpr int kThreads = 32 * (4 + 4 * TILES);   // roles above
   static constexpr int kPVWarp = 2 + 4 * TILES;
+  static constexpr int kAncWarp = 3 + 4 * TILES;
   static constexpr int kStages = TILES == 1 ? 4 : 3;
   static constexpr int kNP = TILES == 1 ? 2 : 1;          // P buffers per tile
   static constexpr int kQOff = 0;
@@ -78,19 +87,25 @@ struct AttnCfg {
   static_assert(kOCol + 128 * TILES <= 512, "TMEM columns");
 };
 
+// Barriers count blocks over the CTA's whole item sequence: K/V stage g %
+// kStages of the g-th block, S buffer g_j & 1 and P buffer g_j % kNP of the
+// g_j-th block of tile j, ancestor buffer k & 1 of the k-th item.
 template <int TILES>
 struct AttnTail {
   static constexpr int kStages = AttnCfg<TILES>::kStages, kNP = AttnCfg<TILES>::kNP;
-  uint64_t q_full;
+  uint64_t q_full, q_empty;
   uint64_t kv_full[kStages], kv_empty[kStages];
   uint64_t s_full[TILES][2], s_empty[TILES][2];
-  uint64_t p_full[TILES][kNP], p_empty[TILES][kNP];   // P / PV of blocks pb, pb + kNP, ...
+  uint64_t p_full[TILES][kNP], p_empty[TILES][kNP];
+  uint64_t anc_full[2], anc_empty[2];
   uint64_t done;
   uint32_t tmem_base;
   int abort;
   int last[TILES];
-  uint32_t anc[TILES][128][kMaskWords];   // ancestor-or-self bits per node
-  int32_t par[PCTREE_ATTN_MAX_N];         // the request's packed parents
+  uint32_t anc[2][TILES][128][kMaskWords];   // ancestor-or-self bits per node
+  int32_t par[PCTREE_ATTN_MAX_N];            // packed parents being walked
+  int32_t pre[kMaxOrder], nn[kMaxOrder];     // validated prefix / node counts
+  int32_t order[kMaxOrder];                  // requests by decreasing key count
 };
 
 template <int TILES>
@@ -109,8 +124,59 @@ struct AttnArgs {
   float2* part_ml;        // [unit][split][128]  (max in log2 units, sum)
   int32_t* status;
   int batch, N, Hq, Hkv, G, npt, R, nqt, tpc, npair, max_slots, n_split, bps;
+  int items;              // batch * Hkv * npair * n_split
   float scale_log2;       // softmax scale * log2(e)
 };
+
+// One work item: request r, KV head kvh, query tiles qt0 .. qt0+ntile-1 and
+// key blocks kb0 .. kb0+nblk-1 of the request's n_keys = Tp + n keys.
+struct AttnItem {
+  int r, kvh, qt0, ntile, split, Tp, n, n_keys, kb0, nblk;
+};
+
+// A request with an impossible prefix or tree size attends to nothing (its
+// rows are written as 0 and the launch reports PCTREE_ERR_INVALID_ARG).
+__device__ __forceinline__ bool request_ok(const AttnArgs& a, int Tp, int n) {
+  return Tp >= 0 && n >= 0 && n <= a.N && static_cast<long long>(Tp) + n <= a.max_slots;
+}
+
+// Item `idx` of the item list: the items of request idx / per_req (of that
+// rank in the longest-first order when `ranked`), as (split, KV head, tile
+// pair) triples.  `staged`: the validated request sizes are in shared
+// memory.
+template <typename Tail>
+__device__ __forceinline__ AttnItem item_facts(const AttnArgs& a, const Tail* T, int idx,
+                                               bool ranked, bool staged) {
+  AttnItem it;
+  const int per_req = a.Hkv * a.npair * a.n_split;
+  const int ri = idx / per_req, rest = idx - ri * per_req;
+  it.r = ranked ? T->order[ri] : ri;
+  it.split = rest / (a.Hkv * a.npair);
+  it.kvh = (rest / a.npair) % a.Hkv;
+  it.qt0 = (rest % a.npair) * a.tpc;
+  it.ntile = min(a.tpc, a.nqt - it.qt0);
+  if (staged) {
+    it.Tp = T->pre[it.r];
+    it.n = T->nn[it.r];
+  } else {
+    it.Tp = a.prefix[it.r];
+    it.n = a.n_nodes[it.r];
+    if (!request_ok(a, it.Tp, it.n)) it.Tp = it.n = 0;
+  }
+  it.n_keys = it.n > 0 ? it.Tp + it.n : 0;       // no queries: nothing to do
+  const int nb_r = (it.n_keys + kBK - 1) / kBK;
+  it.kb0 = it.split * a.bps;
+  it.nblk = max(0, min(it.kb0 + a.bps, nb_r) - it.kb0);
+  return it;
+}
+
+// Position in the longest-first list of this CTA's k-th item: rounds of
+// gridDim.x items, taken forwards and backwards in turn, so every CTA gets a
+// mix of long and short items.
+__device__ __forceinline__ long long item_pos(int k) {
+  const long long base = static_cast<long long>(k) * gridDim.x;
+  return (k & 1) ? base + gridDim.x - 1 - blockIdx.x : base + blockIdx.x;
+}
 
 // 32 lanes x 8 columns of 32-bit TMEM words from registers: thread t of the
 // warp writes lane (taddr.lane + t), columns taddr.col .. +7.
@@ -164,37 +230,44 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
   auto kv_k = [&](int s) { return sm + C::kKVOff + s * kStageBytes; };
   auto kv_v = [&](int s) { return sm + C::kKVOff + s * kStageBytes + 2 * kKVHalf; };
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int pair = blockIdx.x % a.npair, split = blockIdx.x / a.npair;
-  const int kvh = blockIdx.y, r = blockIdx.z;
-  const int qt0 = pair * a.tpc;                        // the CTA's first query tile
-  const int ntile = min(TILES, a.nqt - qt0);
-
-  // request facts; a request with an impossible prefix or tree size is
-  // reported and produces zero rows
-  int Tp = a.prefix[r], n = a.n_nodes[r];
-  if (Tp < 0 || n < 0 || n > a.N || static_cast<long long>(Tp) + n > a.max_slots) {
-    if (threadIdx.x == 0 && split == 0 && pair == 0 && kvh == 0)
-      report(a.status, PCTREE_ERR_INVALID_ARG);
-    Tp = 0;
-    n = 0;
-  }
-  const int n_keys = n > 0 ? Tp + n : 0;        // no queries: nothing to do
-  const int nb_r = (n_keys + kBK - 1) / kBK;
-  const int kb0 = split * a.bps;
-  const int nblk = max(0, min(kb0 + a.bps, nb_r) - kb0);
-
-  // K and V block b into ring stage b % kStages (producer thread only)
-  int issued = 0;
-  auto issue_kv = [&](int b) {
-    const int s = b % kStages, key0 = (kb0 + b) * kBK;
-    mbar_arrive_expect_tx(&T->kv_full[s], static_cast<uint32_t>(kStageBytes));
-    tma_load_4d(kv_k(s), &tm_k, &T->kv_full[s], 0, kvh, key0, r);
-    tma_load_4d(kv_k(s) + kKVHalf, &tm_k, &T->kv_full[s], 64, kvh, key0, r);
-    tma_load_4d(kv_v(s), &tm_v, &T->kv_full[s], 0, kvh, key0, r);
-    tma_load_4d(kv_v(s) + kKVHalf, &tm_v, &T->kv_full[s], 64, kvh, key0, r);
+  const long long n_items = a.items;
+  // ancestor-or-self bits of an item's tile nodes into buffer ab (one warp:
+  // stage the request's packed parents, then walk up from each node)
+  auto ancestor_bits = [&](const AttnItem& it, int ab) {
+    for (int i = lane; i < it.n; i += 32)
+      T->par[i] = a.parent[static_cast<size_t>(it.r) * a.N + i];
+    __syncwarp();
+    for (int i = lane; i < it.ntile * a.npt; i += 32) {
+      const int j = i / a.npt, nl = i - j * a.npt;
+      uint32_t bits[kMaskWords];
+#pragma unroll
+      for (int w = 0; w < kMaskWords; ++w) bits[w] = 0u;
+      int x = (it.qt0 + j) * a.npt + nl;
+      for (int steps = 0; steps <= it.n && x >= 0 && x < it.n; ++steps) {
+#pragma unroll
+        for (int w = 0; w < kMaskWords; ++w)
+          if ((x >> 5) == w) bits[w] |= 1u << (x & 31);
+        const int px = T->par[x];
+        x = px < x ? px : -1;          // parents precede children
+      }
+#pragma unroll
+      for (int w = 0; w < kMaskWords; ++w) T->anc[ab][j][nl][w] = bits[w];
+    }
+    __syncwarp();                      // all lanes done with par and anc
   };
+  // the longest-first order only matters when CTAs take several items; the
+  // request sizes are then staged in shared memory too
+  const bool ranked = a.batch <= kMaxOrder && n_items > static_cast<long long>(gridDim.x);
+  const bool staged = ranked;
+  // with one item per CTA its copies start right after the barrier set-up
+  // (thread 0, the producer, issues Q and the first K/V blocks)
+  int g_pre = 0;
+  bool q_pre = false;
+
+  // ---------------- set-up (once per CTA) ----------------
   if (threadIdx.x == 0) {
     mbar_init(&T->q_full, 1);
+    mbar_init(&T->q_empty, 1);
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&T->kv_full[s], 1);
       mbar_init(&T->kv_empty[s], 1);
@@ -209,55 +282,73 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
         mbar_init(&T->p_empty[j][pb], 1);
       }
     }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&T->anc_full[s], 1);
+      mbar_init(&T->anc_empty[s], 4 * TILES);   // every softmax warp
+    }
     mbar_init(&T->done, 2);              // one commit from each MMA issuer
     T->abort = 0;
     fence_barrier_init();
-    if (nblk > 0) {
-      // the producer's first copies start now and overlap the rest of the
-      // set-up (ancestor bits, TMEM allocation)
+  }
+  if (!ranked && (threadIdx.x == 0 || threadIdx.x == 32)) {
+    const AttnItem it = item_facts(a, T, static_cast<int>(blockIdx.x), false, false);
+    q_pre = it.nblk > 0;                 // known to the S issuer (thread 32) too
+    if (threadIdx.x == 0 && it.nblk > 0) {
       tma_prefetch_desc(&tm_q);
       tma_prefetch_desc(&tm_k);
       tma_prefetch_desc(&tm_v);
-      mbar_arrive_expect_tx(&T->q_full,
-                            static_cast<uint32_t>(ntile) * 2u * static_cast<uint32_t>(a.R) * 128u);
-      for (int j = 0; j < ntile; ++j) {
-        const int node0 = (qt0 + j) * a.npt;
-        tma_load_4d(sq + j * kQBytes, &tm_q, &T->q_full, 0, kvh * a.G, node0, r);
-        tma_load_4d(sq + j * kQBytes + kHalfBytes, &tm_q, &T->q_full, 64, kvh * a.G, node0, r);
+      mbar_arrive_expect_tx(&T->q_full, static_cast<uint32_t>(it.ntile) * 2u *
+                                            static_cast<uint32_t>(a.R) * 128u);
+      for (int j = 0; j < it.ntile; ++j) {
+        const int node0 = (it.qt0 + j) * a.npt;
+        tma_load_4d(sq + j * kQBytes, &tm_q, &T->q_full, 0, it.kvh * a.G, node0, it.r);
+        tma_load_4d(sq + j * kQBytes + kHalfBytes, &tm_q, &T->q_full, 64, it.kvh * a.G, node0,
+                    it.r);
       }
-      for (; issued < min(kStages, nblk); ++issued) issue_kv(issued);
+      for (; g_pre < min(kStages, it.nblk); ++g_pre) {
+        const int s = g_pre, key0 = (it.kb0 + g_pre) * kBK;
+        mbar_arrive_expect_tx(&T->kv_full[s], static_cast<uint32_t>(kStageBytes));
+        tma_load_4d(kv_k(s), &tm_k, &T->kv_full[s], 0, it.kvh, key0, it.r);
+        tma_load_4d(kv_k(s) + kKVHalf, &tm_k, &T->kv_full[s], 64, it.kvh, key0, it.r);
+        tma_load_4d(kv_v(s), &tm_v, &T->kv_full[s], 0, it.kvh, key0, it.r);
+        tma_load_4d(kv_v(s) + kKVHalf, &tm_v, &T->kv_full[s], 64, it.kvh, key0, it.r);
+      }
     }
   }
-  // rows R..127 of each Q tile are not loaded: zero them (read by the MMA)
+  // requests: validated sizes (reported once) and, when ranked, staged and
+  // ordered by key count
+  if (staged || blockIdx.x == 0) {
+    for (int u = threadIdx.x; u < a.batch; u += blockDim.x) {
+      int Tp = a.prefix[u], n = a.n_nodes[u];
+      if (!request_ok(a, Tp, n)) {
+        if (blockIdx.x == 0) report(a.status, PCTREE_ERR_INVALID_ARG);
+        Tp = n = 0;
+      }
+      if (staged) {
+        T->pre[u] = Tp;
+        T->nn[u] = n;
+      }
+    }
+  }
+  if (ranked) {
+    __syncthreads();
+    for (int u = threadIdx.x; u < a.batch; u += blockDim.x) {
+      const int ku = T->nn[u] > 0 ? T->pre[u] + T->nn[u] : 0;
+      int rank = 0;
+      for (int v = 0; v < a.batch; ++v) {
+        const int kv = T->nn[v] > 0 ? T->pre[v] + T->nn[v] : 0;
+        rank += (kv > ku || (kv == ku && v < u)) ? 1 : 0;
+      }
+      T->order[rank] = u;
+    }
+  }
+  // rows R..127 of each Q tile are never loaded: zero them once (read by
+  // the MMA)
   const int zq = (128 - a.R) * 8;                  // 16-byte chunks per half
-  for (int i = threadIdx.x; i < ntile * 2 * zq; i += blockDim.x) {
+  for (int i = threadIdx.x; i < TILES * 2 * zq; i += blockDim.x) {
     const int j = i / (2 * zq), half = (i / zq) & 1, rem = i % zq;
     *reinterpret_cast<uint4*>(sq + j * kQBytes + half * kHalfBytes + (a.R + rem / 8) * 128 +
                               (rem % 8) * 16) = make_uint4(0, 0, 0, 0);
-  }
-  // ancestor-or-self bits of the tiles' nodes (walk up the packed parents,
-  // staged in shared memory)
-  for (int i = threadIdx.x; i < n; i += blockDim.x)
-    T->par[i] = a.parent[static_cast<size_t>(r) * a.N + i];
-  __syncthreads();
-  for (int i = threadIdx.x; i < ntile * a.npt; i += blockDim.x) {
-    const int j = i / a.npt, nl = i - j * a.npt;
-    uint32_t bits[kMaskWords];
-#pragma unroll
-    for (int w = 0; w < kMaskWords; ++w) bits[w] = 0u;
-    int x = (qt0 + j) * a.npt + nl;
-    if (x < n) {
-      const int32_t* par = T->par;
-      for (int steps = 0; steps <= n && x >= 0 && x < n; ++steps) {
-#pragma unroll
-        for (int w = 0; w < kMaskWords; ++w)
-          if ((x >> 5) == w) bits[w] |= 1u << (x & 31);
-        const int px = par[x];
-        x = px < x ? px : -1;          // parents precede children
-      }
-    }
-#pragma unroll
-    for (int w = 0; w < kMaskWords; ++w) T->anc[j][nl][w] = bits[w];
   }
   fence_proxy_async_smem();
   if (warp == 1) tmem_alloc(&T->tmem_base, C::kTmemCols);
@@ -267,291 +358,399 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
   const uint32_t tmem = T->tmem_base;
   volatile int* abort_v = &T->abort;
 
-  if (warp == 0 && lane == 0 && nblk > 0) {
-    // ---------------- TMA producer (thread 0; Q and the first kStages
-    // blocks were issued during the set-up) ----------------
-    for (int b = issued; b < nblk; ++b) {
-      if (!mbar_wait_bounded(&T->kv_empty[b % kStages], ((b / kStages) - 1) & 1, abort_v,
-                             kAttnLimitNs)) {
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer: K and V blocks ----------------
+      tma_prefetch_desc(&tm_k);
+      tma_prefetch_desc(&tm_v);
+      int g = 0;                                   // blocks issued
+      bool ok = true;
+      for (int k = 0; ok; ++k) {
+        const long long pos = item_pos(k);
+        if (pos >= n_items) break;
+        const AttnItem it = item_facts(a, T, static_cast<int>(pos), ranked, staged);
+        // blocks issued during the set-up (first item only)
+        const int b0 = k == 0 ? g_pre : 0;
+        g += b0;
+        for (int b = b0; b < it.nblk; ++b, ++g) {
+          const int s = g % kStages, key0 = (it.kb0 + b) * kBK;
+          if (g >= kStages && !mbar_wait_bounded(&T->kv_empty[s], ((g / kStages) - 1) & 1,
+                                                 abort_v, kAttnLimitNs)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&T->kv_full[s], static_cast<uint32_t>(kStageBytes));
+          tma_load_4d(kv_k(s), &tm_k, &T->kv_full[s], 0, it.kvh, key0, it.r);
+          tma_load_4d(kv_k(s) + kKVHalf, &tm_k, &T->kv_full[s], 64, it.kvh, key0, it.r);
+          tma_load_4d(kv_v(s), &tm_v, &T->kv_full[s], 0, it.kvh, key0, it.r);
+          tma_load_4d(kv_v(s) + kKVHalf, &tm_v, &T->kv_full[s], 64, it.kvh, key0, it.r);
+        }
+      }
+      if (!ok) {
         *abort_v = 1;
+        report(a.status, PCTREE_ERR_TIMEOUT);
+      }
+      // copies still in flight land before the CTA may exit
+      for (int b = g - kStages > 0 ? g - kStages : 0; b < g; ++b)
+        (void)mbar_wait_bounded(&T->kv_full[b % kStages], (b / kStages) & 1, abort_v,
+                                kAttnLimitNs);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- S issuer (and the Q tiles of each item) ----------------
+      constexpr uint32_t idS = idesc_bf16_f32(128, kBK);
+      tma_prefetch_desc(&tm_q);
+      int g = 0, gj[TILES], q = 0;                 // blocks, per tile, Q loads
+      for (int j = 0; j < TILES; ++j) gj[j] = 0;
+      bool ok = true;
+      for (int k = 0; ok; ++k) {
+        const long long pos = item_pos(k);
+        if (pos >= n_items) break;
+        const AttnItem it = item_facts(a, T, static_cast<int>(pos), ranked, staged);
+        if (it.nblk == 0) continue;
+        // the Q buffers are free once the previous item's S products are done
+        if (q > 0 && !mbar_wait_bounded(&T->q_empty, (q - 1) & 1, abort_v, kAttnLimitNs)) {
+          ok = false;
+          break;
+        }
+        if (!(q == 0 && q_pre)) {          // else issued during the set-up
+          mbar_arrive_expect_tx(&T->q_full, static_cast<uint32_t>(it.ntile) * 2u *
+                                                static_cast<uint32_t>(a.R) * 128u);
+          for (int j = 0; j < it.ntile; ++j) {
+            const int node0 = (it.qt0 + j) * a.npt;
+            tma_load_4d(sq + j * kQBytes, &tm_q, &T->q_full, 0, it.kvh * a.G, node0, it.r);
+            tma_load_4d(sq + j * kQBytes + kHalfBytes, &tm_q, &T->q_full, 64, it.kvh * a.G,
+                        node0, it.r);
+          }
+        }
+        if (!mbar_wait_bounded(&T->q_full, q & 1, abort_v, kAttnLimitNs)) {
+          ok = false;
+          break;
+        }
+        ++q;
+        const uint32_t q0 = smem_u32(sq);
+        for (int b = 0; ok && b < it.nblk; ++b, ++g) {
+          const int s = g % kStages;
+          ok = mbar_wait_bounded(&T->kv_full[s], (g / kStages) & 1, abort_v, kAttnLimitNs);
+          const uint32_t k0 = smem_u32(kv_k(s));
+          for (int j = 0; ok && j < it.ntile; ++j) {
+            const int sb = gj[j] & 1;
+            // tile j's S buffer sb was last read by its softmax two blocks ago
+            if (gj[j] >= 2 && !mbar_wait_bounded(&T->s_empty[j][sb], ((gj[j] >> 1) - 1) & 1,
+                                                 abort_v, kAttnLimitNs)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after_sync();
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {      // 128 dims in steps of 16
+              tc_mma_bf16(tmem + (2 * j + sb) * kBK,
+                          desc_kmajor_sw128(q0 + j * kQBytes + (kk >> 2) * kHalfBytes +
+                                            (kk & 3) * 32),
+                          desc_kmajor_sw128(k0 + (kk >> 2) * kKVHalf + (kk & 3) * 32), idS,
+                          kk > 0 ? 1u : 0u);
+            }
+            tc_commit(&T->s_full[j][sb]);
+            ++gj[j];
+          }
+        }
+        tc_commit(&T->q_empty);          // arrives once the item's S products are done
+      }
+      if (!ok) {
+        *abort_v = 1;
+        report(a.status, PCTREE_ERR_TIMEOUT);
+      }
+      tc_commit(&T->done);               // every MMA this thread issued has finished
+      (void)mbar_wait_bounded(&T->done, 0, abort_v, kAttnLimitNs);
+    }
+  } else if (warp == C::kPVWarp) {
+    if (lane == 0) {
+      // ---------------- PV issuer ----------------
+      constexpr uint32_t idO = idesc_bf16_f32_bmn(128, 128);
+      int g = 0, gj[TILES];
+      for (int j = 0; j < TILES; ++j) gj[j] = 0;
+      bool ok = true;
+      for (int k = 0; ok; ++k) {
+        const long long pos = item_pos(k);
+        if (pos >= n_items) break;
+        const AttnItem it = item_facts(a, T, static_cast<int>(pos), ranked, staged);
+        for (int b = 0; ok && b < it.nblk; ++b, ++g) {
+          const int s = g % kStages;
+          const uint32_t v0 = smem_u32(kv_v(s));
+          for (int j = 0; j < it.ntile; ++j) {
+            const int pb = gj[j] % kNP;
+            // P_b of tile j, and with it S_b, is complete
+            if (!mbar_wait_bounded(&T->p_full[j][pb], (gj[j] / kNP) & 1, abort_v,
+                                   kAttnLimitNs)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after_sync();
+            const uint32_t pa = smem_u32(sp + (j * kNP + pb) * kPBytes);
+#pragma unroll
+            for (int kk = 0; kk < kBK / 16; ++kk) {
+              // A: P rows of 64 keys (128 B); B: 16 keys = 16 rows of 128 B,
+              // the dims 64..127 half kKVHalf further on
+              tc_mma_bf16(tmem + C::kOCol + j * 128,
+                          desc_kmajor_sw128(pa + (kk >> 2) * kPSub + (kk & 3) * 32),
+                          desc_mnmajor_sw128(v0 + kk * 16 * 128, kKVHalf, 1024), idO,
+                          (b > 0 || kk > 0) ? 1u : 0u);   // O accumulates over the item
+            }
+            tc_commit(&T->p_empty[j][pb]);
+            ++gj[j];
+          }
+          // the item's S and PV products of this block have read the stage
+          if (ok) tc_commit(&T->kv_empty[s]);
+        }
+      }
+      if (!ok) {
+        *abort_v = 1;
+        report(a.status, PCTREE_ERR_TIMEOUT);
+      }
+      tc_commit(&T->done);
+      (void)mbar_wait_bounded(&T->done, 0, abort_v, kAttnLimitNs);
+    }
+  } else if (warp == C::kAncWarp) {
+    // ---------------- ancestor bits of each item, one item ahead ----------------
+    for (int k = 0;; ++k) {
+      const long long pos = item_pos(k);
+      if (pos >= n_items) break;
+      const AttnItem it = item_facts(a, T, static_cast<int>(pos), ranked, staged);
+      const int ab = k & 1;
+      // buffer ab was last read by the softmax warps for item k - 2
+      const bool got = k < 2 || mbar_wait_bounded(&T->anc_empty[ab], ((k >> 1) - 1) & 1,
+                                                   abort_v, kAttnLimitNs);
+      if (!__all_sync(kFull, got)) {
+        if (lane == 0) {
+          *abort_v = 1;
+          report(a.status, PCTREE_ERR_TIMEOUT);
+        }
         break;
       }
-      issue_kv(b);
-      ++issued;
+      ancestor_bits(it, ab);
+      if (lane == 0) mbar_arrive(&T->anc_full[ab]);
     }
-    // copies still in flight land before the CTA may exit
-    (void)mbar_wait_bounded(&T->q_full, 0, abort_v, kAttnLimitNs);
-    for (int b = issued - kStages > 0 ? issued - kStages : 0; b < issued; ++b)
-      (void)mbar_wait_bounded(&T->kv_full[b % kStages], (b / kStages) & 1, abort_v,
-                              kAttnLimitNs);
-  } else if (warp == 1 && lane == 0 && nblk > 0) {
-    // ---------------- S issuer ----------------
-    constexpr uint32_t idS = idesc_bf16_f32(128, kBK);
-    bool ok = mbar_wait_bounded(&T->q_full, 0, abort_v, kAttnLimitNs);
-    for (int b = 0; ok && b < nblk; ++b) {
-      const int s = b % kStages, sb = b & 1;
-      ok = mbar_wait_bounded(&T->kv_full[s], (b / kStages) & 1, abort_v, kAttnLimitNs);
-      const uint32_t k0 = smem_u32(kv_k(s));
-      for (int j = 0; ok && j < ntile; ++j) {
-        // tile j's S buffer sb was last read by its softmax at block b - 2
-        if (b >= 2 && !mbar_wait_bounded(&T->s_empty[j][sb], ((b >> 1) - 1) & 1, abort_v,
-                                         kAttnLimitNs)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after_sync();
-        const uint32_t q0 = smem_u32(sq + j * kQBytes);
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {      // 128 dims in steps of 16
-          tc_mma_bf16(tmem + (2 * j + sb) * kBK,
-                      desc_kmajor_sw128(q0 + (kk >> 2) * kHalfBytes + (kk & 3) * 32),
-                      desc_kmajor_sw128(k0 + (kk >> 2) * kKVHalf + (kk & 3) * 32), idS,
-                      kk > 0 ? 1u : 0u);
-        }
-        tc_commit(&T->s_full[j][sb]);
-      }
-    }
-    if (!ok) {
-      *abort_v = 1;
-      report(a.status, PCTREE_ERR_TIMEOUT);
-    }
-    tc_commit(&T->done);               // every MMA this thread issued has finished
-    (void)mbar_wait_bounded(&T->done, 0, abort_v, kAttnLimitNs);
-  } else if (warp == C::kPVWarp && lane == 0 && nblk > 0) {
-    // ---------------- PV issuer ----------------
-    constexpr uint32_t idO = idesc_bf16_f32_bmn(128, 128);
-    bool ok = true;
-    for (int b = 0; ok && b < nblk; ++b) {
-      const int s = b % kStages;
-      const uint32_t v0 = smem_u32(kv_v(s));
-      const int pb = b % kNP;
-      for (int j = 0; j < ntile; ++j) {
-        // P_b of tile j, and with it S_b, is complete
-        if (!mbar_wait_bounded(&T->p_full[j][pb], (b / kNP) & 1, abort_v, kAttnLimitNs)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after_sync();
-        const uint32_t pa = smem_u32(sp + (j * kNP + pb) * kPBytes);
-#pragma unroll
-        for (int kk = 0; kk < kBK / 16; ++kk) {
-          // A: P rows of 64 keys (128 B); B: 16 keys = 16 rows of 128 B, the
-          // dims 64..127 half kKVHalf further on
-          tc_mma_bf16(tmem + C::kOCol + j * 128,
-                      desc_kmajor_sw128(pa + (kk >> 2) * kPSub + (kk & 3) * 32),
-                      desc_mnmajor_sw128(v0 + kk * 16 * 128, kKVHalf, 1024), idO,
-                      (b > 0 || kk > 0) ? 1u : 0u);   // O accumulates over blocks
-        }
-        tc_commit(&T->p_empty[j][pb]);
-      }
-      // both tiles' S and PV products of block b have read the stage
-      if (ok) tc_commit(&T->kv_empty[s]);
-    }
-    if (!ok) {
-      *abort_v = 1;
-      report(a.status, PCTREE_ERR_TIMEOUT);
-    }
-    tc_commit(&T->done);
-    (void)mbar_wait_bounded(&T->done, 0, abort_v, kAttnLimitNs);
   }
-  else if (warp >= 2 && warp < 2 + 4 * TILES && (warp - 2) / 4 < ntile) {
-    // ---------------- softmax, one thread per tile row ----------------
+  else if (warp >= 2 && warp < 2 + 4 * TILES) {
+    // ---------------- softmax and output, one thread per tile row ----------------
     // O accumulates in TMEM through the PV MMA with P = 2^(s - m_used); the
     // reference m_used moves (and O and l are rescaled in place) only when
     // a block's maximum exceeds it by more than 2^8, so P stays <= 256.
     const int j = (warp - 2) / 4;            // the tile of this warp
-    const int qt = qt0 + j;
     const int quad = warp & 3;               // TMEM lanes quad*32 .. +31
     const int t = quad * 32 + lane;          // tile row
     const int nl = t / a.G, g = t - nl * a.G;
-    const int node = qt * a.npt + nl;
-    const bool row_ok = t < a.R && node < n;
-    const uint32_t* anc = T->anc[j][nl < a.npt ? nl : 0];
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(quad * 32) << 16);
     const uint32_t s_col = lane_base + 2 * j * kBK, o_col = lane_base + C::kOCol + j * 128;
     const float sc = a.scale_log2;
-    float m_used = -INFINITY, l_sum = 0.0f;  // O and l_sum are relative to m_used
-    bool ok = true;
     // the warp continues only if all its lanes saw the phase complete, so
     // the warp-collective tcgen05 loads that follow never diverge
     auto wwait = [&](uint64_t* bar, uint32_t parity) -> bool {
       const bool got = mbar_wait_bounded(bar, parity, abort_v, kAttnLimitNs);
       return __all_sync(kFull, got);
     };
-    for (int b = 0; b < nblk; ++b) {
-      const int sb = b & 1, st = b % kStages;
-      const int key0 = (kb0 + b) * kBK;
-      if (!wwait(&T->s_full[j][sb], (b >> 1) & 1)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after_sync();
-      float x[kBK];
-      {
-        uint32_t* xu = reinterpret_cast<uint32_t*>(x);
-#pragma unroll
-        for (int c = 0; c < kBK / 32; ++c)
-          tmem_ld_32x32b_x32(s_col + sb * kBK + c * 32,
-                             *reinterpret_cast<uint32_t(*)[32]>(xu + c * 32));
-        tmem_ld_wait();
-      }
-      tc_fence_before_sync();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&T->s_empty[j][sb]);   // S buffer free
-      // scaled scores; keys the row may not see become -inf (eight
-      // independent running maxima keep the dependency chains short)
-      float m8[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) m8[u] = -INFINITY;
-      if (row_ok && key0 + kBK <= Tp) {      // a block of prefix keys only
-#pragma unroll
-        for (int k2 = 0; k2 < kBK; ++k2) {
-          x[k2] *= sc;
-          m8[k2 & 7] = fmaxf(m8[k2 & 7], x[k2]);
-        }
-      } else {
-#pragma unroll
-        for (int c = 0; c < kBK / 32; ++c) {
-          const uint32_t al = row_ok ? allowed_bits(key0 + c * 32, Tp, anc) : 0u;
-#pragma unroll
-          for (int k2 = 0; k2 < 32; ++k2) {
-            const float v = ((al >> k2) & 1u) ? x[c * 32 + k2] * sc : -INFINITY;
-            x[c * 32 + k2] = v;
-            m8[k2 & 7] = fmaxf(m8[k2 & 7], v);
-          }
-        }
-      }
-      const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
-                             fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
-      // the last block of the request: V rows past the tree hold whatever the
-      // cache held there; zero them so that 0 * (non-finite) cannot reach O.
-      // Both tiles' warps do it: each tile's PV product then reads rows its
-      // own warps zeroed and fenced, and the other tile only ever writes the
-      // same zero bytes there.
-      const int valid = n_keys - key0;
-      if (valid < kBK) {
-        if (!wwait(&T->kv_full[st], (b / kStages) & 1)) {
+    int gr = 0, gj = 0;                      // blocks of the ring, of tile j
+    for (int k = 0;; ++k) {
+      const long long pos = item_pos(k);
+      if (pos >= n_items) break;
+      const AttnItem it = item_facts(a, T, static_cast<int>(pos), ranked, staged);
+      const int ab = k & 1;
+      // the item's ancestor bits; both tiles' warps take part in the buffer
+      // hand-off, also for an item without a tile j
+      bool ok = wwait(&T->anc_full[ab], (k >> 1) & 1);
+      const bool active = j < it.ntile;
+      const int node = (it.qt0 + j) * a.npt + nl;
+      const bool row_ok = active && t < a.R && node < it.n;
+      const uint32_t* anc = T->anc[ab][j][nl < a.npt ? nl : 0];
+      const int Tp = it.Tp, n_keys = it.n_keys, nblk = active ? it.nblk : 0;
+      const int g0 = gj;                     // the item's first block of tile j
+      float m_used = -INFINITY, l_sum = 0.0f;  // O and l_sum are relative to m_used
+      for (int b = 0; ok && b < nblk; ++b) {
+        const int gb = g0 + b, sb = gb & 1, st = (gr + b) % kStages;
+        const int key0 = (it.kb0 + b) * kBK;
+        if (!wwait(&T->s_full[j][sb], (gb >> 1) & 1)) {
           ok = false;
           break;
         }
-        uint8_t* v = kv_v(st);
-        for (int i = t; i < 2 * (kBK - valid) * 8; i += 128) {
-          const int half = i / ((kBK - valid) * 8), rem = i % ((kBK - valid) * 8);
-          *reinterpret_cast<uint4*>(v + half * kKVHalf + (valid + rem / 8) * 128 +
-                                    (rem % 8) * 16) = make_uint4(0, 0, 0, 0);
+        tc_fence_after_sync();
+        float x[kBK];
+        {
+          uint32_t* xu = reinterpret_cast<uint32_t*>(x);
+#pragma unroll
+          for (int c = 0; c < kBK / 32; ++c)
+            tmem_ld_32x32b_x32(s_col + sb * kBK + c * 32,
+                               *reinterpret_cast<uint32_t(*)[32]>(xu + c * 32));
+          tmem_ld_wait();
         }
-      }
-      // P buffer pbi was last read by the PV product of block b - kNP
-      const int pbi = b % kNP;
-      if (b >= kNP && !wwait(&T->p_empty[j][pbi], ((b / kNP) - 1) & 1)) {
-        ok = false;
-        break;
-      }
-      // move the reference up where a row needs it; tcgen05.ld / st are
-      // warp-collective, so the warp rescales together (alpha = 1 for rows
-      // that keep their reference)
-      const bool mine = mx > m_used + 8.0f;
-      const float alpha = mine ? ex2_approx(m_used - mx) : 1.0f;   // 0 from -inf
-      if (__any_sync(kFull, mine)) {
-        if (b >= 1) {
-          // O must hold every block before b: the PV product of block b - 1
-          // has finished (with one P buffer, the wait above saw to that)
-          if (kNP > 1 && !wwait(&T->p_empty[j][(b - 1) % kNP], ((b - 1) / kNP) & 1)) {
+        tc_fence_before_sync();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&T->s_empty[j][sb]);   // S buffer free
+        // scaled scores; keys the row may not see become -inf (eight
+        // independent running maxima keep the dependency chains short)
+        float m8[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) m8[u] = -INFINITY;
+        if (row_ok && key0 + kBK <= Tp) {      // a block of prefix keys only
+#pragma unroll
+          for (int k2 = 0; k2 < kBK; ++k2) {
+            x[k2] *= sc;
+            m8[k2 & 7] = fmaxf(m8[k2 & 7], x[k2]);
+          }
+        } else {
+#pragma unroll
+          for (int c = 0; c < kBK / 32; ++c) {
+            const uint32_t al = row_ok ? allowed_bits(key0 + c * 32, Tp, anc) : 0u;
+#pragma unroll
+            for (int k2 = 0; k2 < 32; ++k2) {
+              const float v = ((al >> k2) & 1u) ? x[c * 32 + k2] * sc : -INFINITY;
+              x[c * 32 + k2] = v;
+              m8[k2 & 7] = fmaxf(m8[k2 & 7], v);
+            }
+          }
+        }
+        const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+                               fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
+        // the last block of the request: V rows past the tree hold whatever
+        // the cache held there; zero them so that 0 * (non-finite) cannot
+        // reach O.  Both tiles' warps do it: each tile's PV product then reads
+        // rows its own warps zeroed and fenced, and the other tile only ever
+        // writes the same zero bytes there.
+        const int valid = n_keys - key0;
+        if (valid < kBK) {
+          if (!wwait(&T->kv_full[st], ((gr + b) / kStages) & 1)) {
             ok = false;
             break;
           }
-          tc_fence_after_sync();
-          // eight columns at a time: the block's scores stay live meanwhile
-#pragma unroll 4
-          for (int c = 0; c < 16; ++c) {
-            uint32_t y[8];
-            tmem_ld_32x32b_x8(o_col + c * 8, y);
-            tmem_ld_wait();
-#pragma unroll
-            for (int k2 = 0; k2 < 8; ++k2)
-              y[k2] = __float_as_uint(__uint_as_float(y[k2]) * alpha);
-            tmem_st_32x32b_x8(o_col + c * 8, y);
+          uint8_t* v = kv_v(st);
+          for (int i = t; i < 2 * (kBK - valid) * 8; i += 128) {
+            const int half = i / ((kBK - valid) * 8), rem = i % ((kBK - valid) * 8);
+            *reinterpret_cast<uint4*>(v + half * kKVHalf + (valid + rem / 8) * 128 +
+                                      (rem % 8) * 16) = make_uint4(0, 0, 0, 0);
           }
-          tmem_st_wait();
         }
-        if (mine) {
-          l_sum *= alpha;
-          m_used = mx;
+        // P buffer pbi was last read by the PV product kNP blocks ago (maybe
+        // of the previous item)
+        const int pbi = gb % kNP;
+        if (gb >= kNP && !wwait(&T->p_empty[j][pbi], ((gb / kNP) - 1) & 1)) {
+          ok = false;
+          break;
         }
-      }
-      // P = 2^(s - m_used) in bf16, the A operand of the PV MMA
-      const float mref = m_used == -INFINITY ? 0.0f : m_used;
-      float ls[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-      uint8_t* pbuf = sp + (j * kNP + pbi) * kPBytes;
+        // move the reference up where a row needs it; tcgen05.ld / st are
+        // warp-collective, so the warp rescales together (alpha = 1 for rows
+        // that keep their reference)
+        const bool mine = mx > m_used + 8.0f;
+        const float alpha = mine ? ex2_approx(m_used - mx) : 1.0f;   // 0 from -inf
+        if (__any_sync(kFull, mine)) {
+          if (b >= 1) {
+            // O must hold every block before b: the PV product of block b - 1
+            // has finished (with one P buffer, the wait above saw to that)
+            if (kNP > 1 && !wwait(&T->p_empty[j][(gb - 1) % kNP], ((gb - 1) / kNP) & 1)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after_sync();
+            // eight columns at a time: the block's scores stay live meanwhile
+#pragma unroll 4
+            for (int c = 0; c < 16; ++c) {
+              uint32_t y[8];
+              tmem_ld_32x32b_x8(o_col + c * 8, y);
+              tmem_ld_wait();
 #pragma unroll
-      for (int c = 0; c < kBK / 8; ++c) {    // 8 keys = one 16-byte chunk
-        uint32_t w[4];
-#pragma unroll
-        for (int h = 0; h < 4; ++h) {
-          const float p0 = ex2_approx(x[c * 8 + 2 * h] - mref);
-          const float p1 = ex2_approx(x[c * 8 + 2 * h + 1] - mref);
-          ls[h] += p0 + p1;
-          const __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
-          w[h] = *reinterpret_cast<const uint32_t*>(&pb);
+              for (int k2 = 0; k2 < 8; ++k2)
+                y[k2] = __float_as_uint(__uint_as_float(y[k2]) * alpha);
+              tmem_st_32x32b_x8(o_col + c * 8, y);
+            }
+            tmem_st_wait();
+          }
+          if (mine) {
+            l_sum *= alpha;
+            m_used = mx;
+          }
         }
-        *reinterpret_cast<uint4*>(pbuf + (c >> 3) * kPSub + t * 128 + (((c & 7) ^ (t & 7)) << 4)) =
-            make_uint4(w[0], w[1], w[2], w[3]);
+        // P = 2^(s - m_used) in bf16, the A operand of the PV MMA
+        const float mref = m_used == -INFINITY ? 0.0f : m_used;
+        float ls[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        uint8_t* pbuf = sp + (j * kNP + pbi) * kPBytes;
+#pragma unroll
+        for (int c = 0; c < kBK / 8; ++c) {    // 8 keys = one 16-byte chunk
+          uint32_t w[4];
+#pragma unroll
+          for (int h = 0; h < 4; ++h) {
+            const float p0 = ex2_approx(x[c * 8 + 2 * h] - mref);
+            const float p1 = ex2_approx(x[c * 8 + 2 * h + 1] - mref);
+            ls[h] += p0 + p1;
+            const __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
+            w[h] = *reinterpret_cast<const uint32_t*>(&pb);
+          }
+          *reinterpret_cast<uint4*>(pbuf + (c >> 3) * kPSub + t * 128 +
+                                    (((c & 7) ^ (t & 7)) << 4)) =
+              make_uint4(w[0], w[1], w[2], w[3]);
+        }
+        l_sum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+        tc_fence_before_sync();
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&T->p_full[j][pbi]);
       }
-      l_sum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
-      tc_fence_before_sync();
-      fence_proxy_async_smem();
+      // the ancestor bits of this item are no longer needed
       __syncwarp();
-      if (lane == 0) mbar_arrive(&T->p_full[j][pbi]);
-    }
-    // every PV product of the tile has finished: the last one on each P
-    // buffer (earlier ones are known complete)
-    for (int bb = nblk - kNP > 0 ? nblk - kNP : 0; ok && bb < nblk; ++bb)
-      if (!wwait(&T->p_empty[j][bb % kNP], (bb / kNP) & 1)) ok = false;
-    if (!ok) {
-      *abort_v = 1;
-      report(a.status, PCTREE_ERR_TIMEOUT);
-    }
-    // one decision for the tile's four softmax warps (they meet at named
-    // barriers below, which must see every one of them)
-    named_barrier(1 + j, 128);
-    if (t == 0) T->last[j] = *abort_v;
-    named_barrier(1 + j, 128);
-    ok = T->last[j] == 0;
-    named_barrier(1 + j, 128);
-    tc_fence_after_sync();
-    // ---------------- output ----------------
-    // O is read from TMEM in four 32-column chunks; tcgen05.ld is
-    // warp-collective, so every lane loads and only valid rows store.
-    const int unit = (r * a.Hkv + kvh) * a.nqt + qt;
-    const bool store_row = t < a.R && node < a.N;
-    uint16_t* orow = a.out + ((static_cast<size_t>(r) * a.N + node) * a.Hq + kvh * a.G + g) * 128;
-    auto store_chunk = [&](int c, const float (&v)[32], float inv) {
+      if (lane == 0) mbar_arrive(&T->anc_empty[ab]);
+      // every PV product of the item has finished: the last one on each P
+      // buffer (earlier ones are known complete)
+      for (int gb = g0 + nblk - kNP > g0 ? g0 + nblk - kNP : g0; ok && gb < g0 + nblk; ++gb)
+        if (!wwait(&T->p_empty[j][gb % kNP], (gb / kNP) & 1)) ok = false;
+      gr += it.nblk;
+      gj += nblk;
+      if (!ok) {
+        *abort_v = 1;
+        report(a.status, PCTREE_ERR_TIMEOUT);
+      }
+      // one decision for the tile's four softmax warps (they meet at named
+      // barriers, which must see every one of them)
+      named_barrier(1 + j, 128);
+      if (t == 0) T->last[j] = *abort_v;
+      named_barrier(1 + j, 128);
+      ok = T->last[j] == 0;
+      named_barrier(1 + j, 128);
+      if (!ok) break;
+      if (!active) continue;
+      tc_fence_after_sync();
+      // ---------------- output ----------------
+      // O is read from TMEM in four 32-column chunks; tcgen05.ld is
+      // warp-collective, so every lane loads and only valid rows store.  The
+      // loads finish (tcgen05.wait::ld) before this warp's next P is
+      // published, so the next item's first PV product cannot overwrite O
+      // early.
+      const int unit = (it.r * a.Hkv + it.kvh) * a.nqt + it.qt0 + j;
+      const bool store_row = t < a.R && node < a.N;
+      uint16_t* orow =
+          a.out + ((static_cast<size_t>(it.r) * a.N + node) * a.Hq + it.kvh * a.G + g) * 128;
+      auto store_chunk = [&](int c, const float (&v)[32], float inv) {
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        uint32_t w[4];
+        for (int q = 0; q < 4; ++q) {
+          uint32_t w[4];
 #pragma unroll
-        for (int h = 0; h < 4; ++h) {
-          const __nv_bfloat162 b2 =
-              __floats2bfloat162_rn(v[q * 8 + 2 * h] * inv, v[q * 8 + 2 * h + 1] * inv);
-          w[h] = *reinterpret_cast<const uint32_t*>(&b2);
+          for (int h = 0; h < 4; ++h) {
+            const __nv_bfloat162 b2 =
+                __floats2bfloat162_rn(v[q * 8 + 2 * h] * inv, v[q * 8 + 2 * h + 1] * inv);
+            w[h] = *reinterpret_cast<const uint32_t*>(&b2);
+          }
+          *reinterpret_cast<uint4*>(orow + c * 32 + q * 8) = make_uint4(w[0], w[1], w[2], w[3]);
         }
-        *reinterpret_cast<uint4*>(orow + c * 32 + q * 8) = make_uint4(w[0], w[1], w[2], w[3]);
-      }
-    };
-    auto load_chunk = [&](int c, float (&v)[32]) {
-      if (nblk > 0) {
-        uint32_t y[32];
-        tmem_ld_32x32b_x32(o_col + c * 32, y);
-        tmem_ld_wait();
+      };
+      auto load_chunk = [&](int c, float (&v)[32]) {
+        if (nblk > 0) {
+          uint32_t y[32];
+          tmem_ld_32x32b_x32(o_col + c * 32, y);
+          tmem_ld_wait();
 #pragma unroll
-        for (int k2 = 0; k2 < 32; ++k2) v[k2] = __uint_as_float(y[k2]);
-      } else {
+          for (int k2 = 0; k2 < 32; ++k2) v[k2] = __uint_as_float(y[k2]);
+        } else {
 #pragma unroll
-        for (int k2 = 0; k2 < 32; ++k2) v[k2] = 0.0f;
-      }
-    };
-    if (a.n_split == 1) {
-      if (ok) {
+          for (int k2 = 0; k2 < 32; ++k2) v[k2] = 0.0f;
+        }
+      };
+      if (a.n_split == 1) {
         const float inv = l_sum > 0.0f ? 1.0f / l_sum : 0.0f;
 #pragma unroll 1
         for (int c = 0; c < 4; ++c) {
@@ -559,21 +758,22 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
           load_chunk(c, v);
           if (store_row) store_chunk(c, v, inv);
         }
-      }
-    } else if (ok) {
-      const size_t slot = static_cast<size_t>(unit) * a.n_split + split;
-      a.part_ml[slot * 128 + t] = make_float2(l_sum > 0.0f ? m_used : -INFINITY, l_sum);
-      float4* po = reinterpret_cast<float4*>(a.part_o + (slot * 128 + t) * 128);
+      } else {
+        const size_t slot = static_cast<size_t>(unit) * a.n_split + it.split;
+        a.part_ml[slot * 128 + t] = make_float2(l_sum > 0.0f ? m_used : -INFINITY, l_sum);
+        float4* po = reinterpret_cast<float4*>(a.part_o + (slot * 128 + t) * 128);
 #pragma unroll 1
-      for (int c = 0; c < 4; ++c) {
-        float v[32];
-        load_chunk(c, v);
-        if (l_sum > 0.0f) {
+        for (int c = 0; c < 4; ++c) {
+          float v[32];
+          load_chunk(c, v);
+          if (l_sum > 0.0f) {
 #pragma unroll
-          for (int q = 0; q < 8; ++q)
-            po[c * 8 + q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            for (int q = 0; q < 8; ++q)
+              po[c * 8 + q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+          }
         }
       }
+      tc_fence_before_sync();
     }
   }
   // ---------------- teardown ----------------
@@ -670,11 +870,11 @@ tree_attn_merge_kernel(AttnArgs a) {
 namespace pct {
 namespace {
 
-// Tiling of a configuration: query tiles per (request, KV head) and the split
-// of each request's key blocks over CTAs.  Splits are chosen so that the
-// grid has about one CTA per SM of a 152-SM GB300 when there are few
-// (request, KV head, tile) units; they depend only on the configuration, so
-// the workspace size does too.
+// Tiling of a configuration: query tiles per (request, KV head), tiles per
+// item and the split of each request's key blocks over items.  Splits are
+// chosen so that there are about as many items as the 152 SMs of a GB300
+// when there are few (request, KV head, tile) units; they depend only on the
+// configuration, so the workspace size does too.
 struct AttnGeom {
   int G, npt, R, nqt, tpc, npair, nb_max, n_split, bps;
   long long units;                    // (request, KV head, query tile) triples
@@ -686,9 +886,8 @@ AttnGeom attn_geom(const pctree_attn_config& c) {
   g.npt = 128 / g.G < c.N ? 128 / g.G : c.N;
   g.R = g.G * g.npt;
   g.nqt = (c.N + g.npt - 1) / g.npt;
-  // two tiles per CTA once such CTAs still fill every SM: the set-up is then
-  // paid once per two tiles and their softmax waits overlap; otherwise one
-  // tile per CTA keeps more SMs busy
+  // two tiles per item once such items still fill every SM (their softmax
+  // waits overlap); otherwise one tile per item keeps more SMs busy
   const long long pairs = static_cast<long long>(c.batch) * c.Hkv * ((g.nqt + 1) / 2);
   g.tpc = (g.nqt >= 2 && pairs >= 152) ? 2 : 1;
   g.npair = (g.nqt + g.tpc - 1) / g.tpc;
@@ -713,7 +912,7 @@ pctree_status attn_check(const pctree_attn_config* c) {
       c->batch > 65535 || c->Hkv > 65535)
     return PCTREE_ERR_UNSUPPORTED;
   const AttnGeom g = attn_geom(*c);
-  if (static_cast<long long>(g.npair) * g.n_split > 0x7fffffffll)
+  if (static_cast<long long>(c->batch) * c->Hkv * g.npair * g.n_split > 0x7fffffffll)
     return PCTREE_ERR_UNSUPPORTED;
   return PCTREE_OK;
 }
@@ -807,6 +1006,7 @@ pctree_status pctree_tree_attention(const pctree_attn_config* cfg, const void* q
   a.nqt = g.nqt;
   a.tpc = g.tpc;
   a.npair = g.npair;
+  a.items = static_cast<int>(static_cast<long long>(c.batch) * c.Hkv * g.npair * g.n_split);
   a.max_slots = c.max_slots;
   a.n_split = g.n_split;
   a.bps = g.bps;
@@ -828,8 +1028,8 @@ pctree_status pctree_tree_attention(const pctree_attn_config* cfg, const void* q
       return PCTREE_ERR_CUDA;
     attr_set[dev] = true;
   }
-  const dim3 grid(static_cast<unsigned>(g.npair * g.n_split), static_cast<unsigned>(c.Hkv),
-                  static_cast<unsigned>(c.batch));
+  // persistent: one CTA per SM walks its share of the items
+  const dim3 grid(static_cast<unsigned>(a.items < num_sms ? a.items : num_sms));
   if (g.tpc == 2)
     tree_attn_kernel<2><<<grid, AttnCfg<2>::kThreads, attn_smem<2>(), stream>>>(tm_q, tm_k, tm_v, a);
   else
