@@ -333,7 +333,7 @@ typedef struct {
 } pctree_attn_config;
 
 /* Workspace bytes pctree_tree_attention needs (0 when a request's keys are
- * never split over several CTAs); 256-byte aligned, any prior content. */
+ * never split over several work items); 256-byte aligned, any prior content. */
 PCTREE_API size_t pctree_tree_attention_workspace_bytes(const pctree_attn_config* cfg);
 
 /*
