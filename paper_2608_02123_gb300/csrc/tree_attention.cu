@@ -14,34 +14,34 @@
 // products overlap the current item's last blocks and output.
 //
 //   warp 0      TMA producer: K and V blocks (64 keys x 128 dims, two 64-dim
-//               halves each, 128-byte swizzle) into a ring (four stages for
-//               one tile, three for two) that runs on across items
+//               halves each, 128-byte swizzle) into a ring (five stages for
+//               one tile, four for two) that runs on across items
 //   warp 1      S issuer: each item's Q tiles (once the previous item's S
 //               products are done), then S_b = Q K_b^T per tile (tcgen05.mma,
 //               M=128, N=64 keys, K=128 dims) into one of the tile's two TMEM
 //               buffers, up to two blocks ahead of its softmax
 //   warps 2..5  softmax and output of tile 0 (warps 6..9: tile 1): one thread
 //               per TMEM lane = tile row; each S row is read from TMEM once,
-//               masked and scaled; P = 2^(s - m_used) rounded to bf16 into a
-//               shared-memory P buffer (the K-major A operand of the second
-//               MMA).  O accumulates in TMEM across an item's blocks; the
+//               masked and scaled; P = 2^(s - m_used) rounded to bf16 pairs is
+//               written back over the first 32 columns of the S buffer (the
+//               TMEM A operand of the second MMA).  O accumulates in TMEM
+//               across an item's blocks; the
 //               reference m_used rises (O and the row sum rescaled in place,
 //               tcgen05.ld / st) only when a block's maximum exceeds it by
 //               more than 8 in log2 units, so P stays below 2^8.  After the
 //               item's last block the same warps normalise O and store it.
 //   next warp   PV issuer: O += P_b V_b per tile (M=128, N=128 dims, K=64
-//               keys; V is the MN-major operand, dims contiguous) as soon as
-//               the tile's P_b is written; after the item's tiles it frees the
-//               K/V stage (S_b, the other reader, finished before P_b existed)
+//               keys; P read from TMEM, V the MN-major shared-memory operand,
+//               dims contiguous) as soon as the tile's P_b is written; its
+//               commit frees the S buffer and, after the item's tiles, the K/V
+//               stage (S_b, the other reader, finished before P_b existed)
 //   last warp   ancestor bits: the next item's ancestor-or-self masks (from
 //               the packed parents) into the second of two buffers
 //
 // With two tiles each SM sub-partition runs one softmax warp of each, so one
-// tile's waits (TMEM loads, the PV product before its single P buffer is
-// rewritten) overlap the other's arithmetic; TMEM then holds 2 x (two
-// 64-column S buffers + a 128-column O) = 512 columns.  One tile per item
-// (chosen when two-tile items would leave SMs idle) double-buffers P
-// instead.  Key blocks of a request may be split over several items (few
+// tile's waits overlap the other's arithmetic; TMEM then holds 2 x (two
+// 64-column S buffers + a 128-column O) = 512 columns.  One tile per item is
+// chosen when two-tile items would leave SMs idle.  Key blocks of a request may be split over several items (few
 // requests, long prefixes); each then writes (max, sum, unnormalised O) of
 // its rows and a second kernel merges the splits, spread over all SMs.  All
 // waits are bounded (1 s) and end in PCTREE_ERR_TIMEOUT.
@@ -58,29 +58,26 @@ constexpr int kHalfBytes = 128 * 128;     // Q: 128 rows x 64 bf16 (one dim half
 constexpr int kQBytes = 2 * kHalfBytes;   // one Q tile
 constexpr int kKVHalf = kBK * 128;        // K or V: 64 keys x 64 bf16 (one dim half)
 constexpr int kStageBytes = 4 * kKVHalf;  // K (two halves) then V (two halves)
-constexpr int kPSub = 128 * 128;          // P: 128 rows x 64 keys bf16 (SW128)
-constexpr int kPBytes = kPSub * (kBK / 64);
 constexpr int kMaskWords = PCTREE_ATTN_MAX_N / 32;
 constexpr uint64_t kAttnLimitNs = 1000000000ull;
 
 constexpr int kMaxOrder = 256;            // requests ordered by length in shared memory
 
-// Layout of a CTA with TILES query tiles (1 or 2).  One tile: a four-stage
-// K/V ring and two P buffers, so P_b is written while the PV product of
-// block b-1 still runs.  Two tiles: a three-stage ring and one P buffer per
-// tile (the other tile's softmax covers that wait).
+// Layout of a CTA with TILES query tiles (1 or 2): the Q tiles and a K/V
+// ring in shared memory (five stages for one tile, four for two); per tile,
+// two S buffers of 64 fp32 columns in TMEM (P, packed bf16 pairs, overwrites
+// the first 32 columns of its S buffer and is the TMEM A operand of the PV
+// product) and a 128-column O.
 template <int TILES>
 struct AttnCfg {
   static constexpr int kThreads = 32 * (4 + 4 * TILES);   // roles above
   static constexpr int kPVWarp = 2 + 4 * TILES;
   static constexpr int kAncWarp = 3 + 4 * TILES;
-  static constexpr int kStages = TILES == 1 ? 4 : 3;
-  static constexpr int kNP = TILES == 1 ? 2 : 1;          // P buffers per tile
+  static constexpr int kStages = TILES == 1 ? 5 : 4;
   static constexpr int kQOff = 0;
   static constexpr int kKVOff = TILES * kQBytes;
-  static constexpr int kPOff = kKVOff + kStages * kStageBytes;
-  static constexpr int kTailOff = kPOff + TILES * kNP * kPBytes;
-  // TMEM: tile j's two S buffers at columns (2j + sb) * kBK, its O (128
+  static constexpr int kTailOff = kKVOff + kStages * kStageBytes;
+  // TMEM: tile j's S buffer sb at columns (2j + sb) * kBK, its O (128
   // columns) at kOCol + 128 j
   static constexpr uint32_t kOCol = 2 * TILES * kBK;
   static constexpr uint32_t kTmemCols = kOCol + 128 * TILES <= 256 ? 256 : 512;
@@ -88,15 +85,16 @@ struct AttnCfg {
 };
 
 // Barriers count blocks over the CTA's whole item sequence: K/V stage g %
-// kStages of the g-th block, S buffer g_j & 1 and P buffer g_j % kNP of the
-// g_j-th block of tile j, ancestor buffer k & 1 of the k-th item.
+// kStages of the g-th block, S/P buffer g_j & 1 of the g_j-th block of tile
+// j, ancestor buffer k & 1 of the k-th item.
 template <int TILES>
 struct AttnTail {
-  static constexpr int kStages = AttnCfg<TILES>::kStages, kNP = AttnCfg<TILES>::kNP;
+  static constexpr int kStages = AttnCfg<TILES>::kStages;
   uint64_t q_full, q_empty;
   uint64_t kv_full[kStages], kv_empty[kStages];
-  uint64_t s_full[TILES][2], s_empty[TILES][2];
-  uint64_t p_full[TILES][kNP], p_empty[TILES][kNP];
+  uint64_t s_full[TILES][2];               // S written
+  uint64_t p_full[TILES][2];               // P written over it
+  uint64_t p_empty[TILES][2];              // PV product done: buffer free
   uint64_t anc_full[2], anc_empty[2];
   uint64_t done;
   uint32_t tmem_base;
@@ -187,6 +185,31 @@ __device__ __forceinline__ void tmem_st_32x32b_x8(uint32_t taddr, const uint32_t
       : "memory");
 }
 
+// 32 lanes x 16 columns of 32-bit TMEM words from registers (see
+// tmem_st_32x32b_x8).
+__device__ __forceinline__ void tmem_st_32x32b_x16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15])
+      : "memory");
+}
+
+// D[tmem] (+)= A[tmem] * B[smem]: the A operand (M = 128 rows on the TMEM
+// lanes, 16 K elements as 8 columns of bf16 pairs, the lower half holding the
+// even element) is read from tensor memory.  Issued by one thread.
+__device__ __forceinline__ void tc_mma_bf16_tmem_a(uint32_t d_tmem, uint32_t a_tmem,
+                                                   uint64_t b_desc, uint32_t idesc,
+                                                   uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 // Records the first error in the optional status word.
 __device__ __forceinline__ void report(int32_t* status, int code) {
   if (status != nullptr) atomicCAS(status, 0, code);
@@ -219,13 +242,12 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
                  const __grid_constant__ CUtensorMap tm_k,
                  const __grid_constant__ CUtensorMap tm_v, AttnArgs a) {
   using C = AttnCfg<TILES>;
-  constexpr int kStages = C::kStages, kNP = C::kNP;
+  constexpr int kStages = C::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   AttnTail<TILES>* T = reinterpret_cast<AttnTail<TILES>*>(sm + C::kTailOff);
   uint8_t* sq = sm + C::kQOff;
-  uint8_t* sp = sm + C::kPOff;
   // ring stage s: K (two dim halves) then V (two dim halves)
   auto kv_k = [&](int s) { return sm + C::kKVOff + s * kStageBytes; };
   auto kv_v = [&](int s) { return sm + C::kKVOff + s * kStageBytes + 2 * kKVHalf; };
@@ -273,13 +295,10 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
       mbar_init(&T->kv_empty[s], 1);
     }
     for (int j = 0; j < TILES; ++j) {
-      for (int s = 0; s < 2; ++s) {
-        mbar_init(&T->s_full[j][s], 1);
-        mbar_init(&T->s_empty[j][s], 4);
-      }
-      for (int pb = 0; pb < kNP; ++pb) {
-        mbar_init(&T->p_full[j][pb], 4);
-        mbar_init(&T->p_empty[j][pb], 1);
+      for (int sb = 0; sb < 2; ++sb) {
+        mbar_init(&T->s_full[j][sb], 1);
+        mbar_init(&T->p_full[j][sb], 4);
+        mbar_init(&T->p_empty[j][sb], 1);
       }
     }
     for (int s = 0; s < 2; ++s) {
@@ -435,8 +454,9 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
           const uint32_t k0 = smem_u32(kv_k(s));
           for (int j = 0; ok && j < it.ntile; ++j) {
             const int sb = gj[j] & 1;
-            // tile j's S buffer sb was last read by its softmax two blocks ago
-            if (gj[j] >= 2 && !mbar_wait_bounded(&T->s_empty[j][sb], ((gj[j] >> 1) - 1) & 1,
+            // tile j's S buffer sb holds the P of block gj - 2 until that
+            // block's PV product is done
+            if (gj[j] >= 2 && !mbar_wait_bounded(&T->p_empty[j][sb], ((gj[j] >> 1) - 1) & 1,
                                                  abort_v, kAttnLimitNs)) {
               ok = false;
               break;
@@ -478,25 +498,24 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
           const int s = g % kStages;
           const uint32_t v0 = smem_u32(kv_v(s));
           for (int j = 0; j < it.ntile; ++j) {
-            const int pb = gj[j] % kNP;
+            const int sb = gj[j] & 1;
             // P_b of tile j, and with it S_b, is complete
-            if (!mbar_wait_bounded(&T->p_full[j][pb], (gj[j] / kNP) & 1, abort_v,
+            if (!mbar_wait_bounded(&T->p_full[j][sb], (gj[j] >> 1) & 1, abort_v,
                                    kAttnLimitNs)) {
               ok = false;
               break;
             }
             tc_fence_after_sync();
-            const uint32_t pa = smem_u32(sp + (j * kNP + pb) * kPBytes);
+            const uint32_t pa = tmem + (2 * j + sb) * kBK;       // P: 32 columns
 #pragma unroll
             for (int kk = 0; kk < kBK / 16; ++kk) {
-              // A: P rows of 64 keys (128 B); B: 16 keys = 16 rows of 128 B,
-              // the dims 64..127 half kKVHalf further on
-              tc_mma_bf16(tmem + C::kOCol + j * 128,
-                          desc_kmajor_sw128(pa + (kk >> 2) * kPSub + (kk & 3) * 32),
-                          desc_mnmajor_sw128(v0 + kk * 16 * 128, kKVHalf, 1024), idO,
-                          (b > 0 || kk > 0) ? 1u : 0u);   // O accumulates over the item
+              // A: 16 keys of P = 8 TMEM columns; B: 16 keys = 16 rows of 128 B
+              // of V, the dims 64..127 half kKVHalf further on
+              tc_mma_bf16_tmem_a(tmem + C::kOCol + j * 128, pa + kk * 8,
+                                 desc_mnmajor_sw128(v0 + kk * 16 * 128, kKVHalf, 1024), idO,
+                                 (b > 0 || kk > 0) ? 1u : 0u);   // O accumulates over the item
             }
-            tc_commit(&T->p_empty[j][pb]);
+            tc_commit(&T->p_empty[j][sb]);
             ++gj[j];
           }
           // the item's S and PV products of this block have read the stage
@@ -582,9 +601,6 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
                                *reinterpret_cast<uint32_t(*)[32]>(xu + c * 32));
           tmem_ld_wait();
         }
-        tc_fence_before_sync();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&T->s_empty[j][sb]);   // S buffer free
         // scaled scores; keys the row may not see become -inf (eight
         // independent running maxima keep the dependency chains short)
         float m8[8];
@@ -628,13 +644,6 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
                                       (rem % 8) * 16) = make_uint4(0, 0, 0, 0);
           }
         }
-        // P buffer pbi was last read by the PV product kNP blocks ago (maybe
-        // of the previous item)
-        const int pbi = gb % kNP;
-        if (gb >= kNP && !wwait(&T->p_empty[j][pbi], ((gb / kNP) - 1) & 1)) {
-          ok = false;
-          break;
-        }
         // move the reference up where a row needs it; tcgen05.ld / st are
         // warp-collective, so the warp rescales together (alpha = 1 for rows
         // that keep their reference)
@@ -643,8 +652,8 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
         if (__any_sync(kFull, mine)) {
           if (b >= 1) {
             // O must hold every block before b: the PV product of block b - 1
-            // has finished (with one P buffer, the wait above saw to that)
-            if (kNP > 1 && !wwait(&T->p_empty[j][(gb - 1) % kNP], ((gb - 1) / kNP) & 1)) {
+            // has finished
+            if (!wwait(&T->p_empty[j][(gb - 1) & 1], ((gb - 1) >> 1) & 1)) {
               ok = false;
               break;
             }
@@ -667,38 +676,37 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
             m_used = mx;
           }
         }
-        // P = 2^(s - m_used) in bf16, the A operand of the PV MMA
+        // P = 2^(s - m_used) in bf16 pairs over the first 32 columns of the
+        // S buffer (all of S is in registers): the TMEM A operand of the PV
+        // MMA
         const float mref = m_used == -INFINITY ? 0.0f : m_used;
         float ls[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-        uint8_t* pbuf = sp + (j * kNP + pbi) * kPBytes;
 #pragma unroll
-        for (int c = 0; c < kBK / 8; ++c) {    // 8 keys = one 16-byte chunk
-          uint32_t w[4];
+        for (int c = 0; c < kBK / 32; ++c) {
+          uint32_t pk[16];
 #pragma unroll
-          for (int h = 0; h < 4; ++h) {
-            const float p0 = ex2_approx(x[c * 8 + 2 * h] - mref);
-            const float p1 = ex2_approx(x[c * 8 + 2 * h + 1] - mref);
-            ls[h] += p0 + p1;
+          for (int h = 0; h < 16; ++h) {
+            const float p0 = ex2_approx(x[c * 32 + 2 * h] - mref);
+            const float p1 = ex2_approx(x[c * 32 + 2 * h + 1] - mref);
+            ls[h & 3] += p0 + p1;
             const __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
-            w[h] = *reinterpret_cast<const uint32_t*>(&pb);
+            pk[h] = *reinterpret_cast<const uint32_t*>(&pb);
           }
-          *reinterpret_cast<uint4*>(pbuf + (c >> 3) * kPSub + t * 128 +
-                                    (((c & 7) ^ (t & 7)) << 4)) =
-              make_uint4(w[0], w[1], w[2], w[3]);
+          tmem_st_32x32b_x16(s_col + sb * kBK + c * 16, pk);
         }
+        tmem_st_wait();
         l_sum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
         tc_fence_before_sync();
-        fence_proxy_async_smem();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&T->p_full[j][pbi]);
+        if (lane == 0) mbar_arrive(&T->p_full[j][sb]);
       }
       // the ancestor bits of this item are no longer needed
       __syncwarp();
       if (lane == 0) mbar_arrive(&T->anc_empty[ab]);
-      // every PV product of the item has finished: the last one on each P
+      // every PV product of the item has finished: the last one on each S/P
       // buffer (earlier ones are known complete)
-      for (int gb = g0 + nblk - kNP > g0 ? g0 + nblk - kNP : g0; ok && gb < g0 + nblk; ++gb)
-        if (!wwait(&T->p_empty[j][gb % kNP], (gb / kNP) & 1)) ok = false;
+      for (int gb = g0 + nblk - 2 > g0 ? g0 + nblk - 2 : g0; ok && gb < g0 + nblk; ++gb)
+        if (!wwait(&T->p_empty[j][gb & 1], (gb >> 1) & 1)) ok = false;
       gr += it.nblk;
       gj += nblk;
       if (!ok) {
