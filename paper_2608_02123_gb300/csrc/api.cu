@@ -69,7 +69,9 @@ Layout make_layout(const pctree_config& c) {
   l.off_pool_par = take(static_cast<size_t>(c.batch) * l.P * sizeof(int32_t));
   l.off_pool_s = take(static_cast<size_t>(c.batch) * l.P * sizeof(float2));
   l.off_front = take(static_cast<size_t>(c.batch) * c.k * sizeof(int32_t));
-  l.sync_bytes = 2 * static_cast<size_t>(c.B) * sizeof(int);   // tickets, flags
+  // stage tickets and release flags, then one flag per (CTA boundary,
+  // TMEM lane quadrant) for the tiles two CTAs share
+  l.sync_bytes = (2 * static_cast<size_t>(c.B) + 4 * kFusedMaxGrid) * sizeof(int);
   l.off_sync = take(l.sync_bytes);
   const size_t fparts = static_cast<size_t>(kFusedRows) * kFusedMaxGrid;
   l.off_fpm = take(fparts * sizeof(float));
@@ -77,6 +79,10 @@ Layout make_layout(const pctree_config& c) {
   l.off_fcz = take(fparts * c.k * sizeof(float));
   l.off_fct = take(fparts * c.k * sizeof(int32_t));
   l.off_xtok = take(static_cast<size_t>(c.batch) * c.k * sizeof(int32_t));
+  // partial accumulators of shared tiles, [stage parity][boundary][row][128]
+  l.off_fxch = l.rows_max <= kFusedRows
+                   ? take(2 * fparts * kFusedTileRows * sizeof(float))
+                   : l.off_xtok;
   l.total = off;
   return l;
 }
@@ -240,6 +246,8 @@ pctree_status draft_fused(const pctree_config& c, const Layout& lay,
   a.part_s = reinterpret_cast<float*>(ws + lay.off_fps);
   a.cand_z = reinterpret_cast<float*>(ws + lay.off_fcz);
   a.cand_t = reinterpret_cast<int32_t*>(ws + lay.off_fct);
+  a.xflag = sync + 2 * c.B;
+  a.xch = reinterpret_cast<float*>(ws + lay.off_fxch);
   a.status = out.status;
   a.limit_ns = g_wait_limit_ns;
   a.stall_stage = g_stall_stage;

@@ -32,6 +32,7 @@ struct Layout {
   size_t off_pool_tok, off_pool_par, off_pool_s, off_front;
   // fused-round path: cross-CTA flags, per-CTA partials, parent tokens
   size_t off_sync, sync_bytes, off_fpm, off_fps, off_fcz, off_fct, off_xtok;
+  size_t off_fxch;  // fused-round path: partial accumulators of shared tiles
   size_t total;
 };
 
@@ -40,6 +41,7 @@ struct Layout {
 constexpr int kFusedRows = 16;
 constexpr int kFusedMaxK = 16;
 constexpr int kFusedMaxGrid = 256;
+constexpr int kFusedTileRows = 128;   // vocabulary rows per W_out tile (MMA M)
 
 struct FusedArgs {
   const float* L;        // [batch][B][V] base logits
@@ -58,6 +60,8 @@ struct FusedArgs {
   float* part_s;         // [kFusedRows][grid] per-CTA sum of exp
   float* cand_z;         // [kFusedRows][grid][k] per-CTA top-k logits
   int32_t* cand_t;       // [kFusedRows][grid][k] per-CTA top-k tokens
+  int* xflag;            // [grid][4] stage + 1 once a shared tile's partial is out
+  float* xch;            // [2][kFusedMaxGrid][kFusedRows][128] those partials
   int32_t* status;
   unsigned long long limit_ns;   // bound of every wait (1 s)
   int stall_stage;       // test hook: stage whose release is withheld, or -1

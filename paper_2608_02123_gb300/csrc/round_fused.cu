@@ -64,9 +64,8 @@ struct FusedSmem {
       float m[R][kEpiThreads];
       float s[R][kEpiThreads];
     } part;
-    struct {                               // merge: first entries of 32 CTAs
-      float z[kEpiWarps][kG][32];
-      int t[kEpiWarps][kG][32];
+    struct {                               // merge: CTAs whose best entry
+      int cta[kEpiWarps][kG * 32];         // reaches the k-th best of them
     } stage;
   } u;
   unsigned long long keys[R * kMaxKF];     // new layer: (score, id) keys
@@ -82,20 +81,43 @@ constexpr size_t smem_bytes() {
 
 __device__ __forceinline__ void epi_barrier() { named_barrier(1, kEpiThreads); }
 
-// i-th tile (0-based) of this CTA in stage d, and the kc-th K chunk of a
-// tile: even stages walk forward, odd stages backward, so each stage visits
-// (tile, chunk) in the exact reverse of the previous stage's order.
-__device__ __forceinline__ int tile_at(int d, int i, int n_my) {
-  const int j = (d & 1) ? n_my - 1 - i : i;
-  return blockIdx.x + j * gridDim.x;
-}
+// This CTA's share of a stage: the contiguous range [lo, hi) of the stage's
+// n_tiles * n_k (tile, K chunk) pairs numbered tile-major, lo = b * W / G for
+// CTA b of G.  Every CTA gets floor(W / G) or ceil(W / G) pairs, so all of
+// them stream the same number of bytes per stage.  A tile cut by a range
+// boundary is shared by the two CTAs beside it (the grid never exceeds the
+// tile count, so a range spans at least n_k pairs and no tile is cut twice):
+// the CTA that reaches it first exports its partial accumulator, the other
+// adds that partial to its own and runs the epilogue of the whole tile.
+struct Share {
+  int lo, hi;   // pair range
+  int t0, n;    // first tile, number of (whole or partial) tiles
+  __device__ __forceinline__ Share(int n_tiles, int n_k) {
+    const long long W = static_cast<long long>(n_tiles) * n_k;
+    lo = static_cast<int>(W * blockIdx.x / gridDim.x);
+    hi = static_cast<int>(W * (blockIdx.x + 1) / gridDim.x);
+    t0 = lo / n_k;
+    n = (hi - 1) / n_k - t0 + 1;
+  }
+  // Unit i (0-based) of stage d: even stages walk the units forward, odd
+  // stages backward, so each stage visits (tile, chunk) pairs in the exact
+  // reverse of the previous stage's order.  [c0, c1) is the chunk range.
+  __device__ __forceinline__ void unit(int d, int i, int n_k, int& tile, int& c0,
+                                       int& c1) const {
+    tile = t0 + ((d & 1) ? n - 1 - i : i);
+    c0 = max(lo - tile * n_k, 0);
+    c1 = min(hi - tile * n_k, n_k);
+  }
+  // CTA boundary of a cut tile: b - 1 when it begins this CTA's range,
+  // b when it ends it.
+  __device__ __forceinline__ int boundary(int c0) const {
+    return c0 > 0 ? static_cast<int>(blockIdx.x) - 1 : static_cast<int>(blockIdx.x);
+  }
+};
 
-__device__ __forceinline__ int chunk_at(int d, int kc, int n_k) {
-  return (d & 1) ? n_k - 1 - kc : kc;
-}
-
-__device__ __forceinline__ int my_tiles(int n_tiles) {
-  return (n_tiles - static_cast<int>(blockIdx.x) + gridDim.x - 1) / gridDim.x;
+// K chunk of the kc-th step through the range [c0, c1) in stage d.
+__device__ __forceinline__ int chunk_at(int d, int kc, int c0, int c1) {
+  return (d & 1) ? c1 - 1 - kc : c0 + kc;
 }
 
 // --------------------------------------------------------------------------
@@ -106,7 +128,7 @@ template <int R>
 __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
                         const FusedArgs& a, unsigned char* ring,
                         FusedSmem<R>* S, volatile int* abort_v) {
-  const int n_my = my_tiles(a.n_tiles);
+  const Share sh(a.n_tiles, a.n_k);
   const uint64_t stream_policy = l2_policy_evict_first();
   constexpr uint32_t tx = kABytes + kBBytes;
   int stage = 0;
@@ -126,9 +148,10 @@ __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
   for (int d = 0; d < a.B && ok; ++d) {
     bool have = d == 0;   // stage 0 rows were written before the launch
     n_pend = 0;
-    for (int i = 0; i < n_my && ok; ++i) {
-      const int tile = tile_at(d, i, n_my);
-      for (int kc = 0; kc < a.n_k; ++kc) {
+    for (int i = 0; i < sh.n && ok; ++i) {
+      int tile, c0, c1;
+      sh.unit(d, i, a.n_k, tile, c0, c1);
+      for (int kc = 0; kc < c1 - c0; ++kc) {
         if (!have) {
           bool rdy = poll_flag(&a.ready[d]);
           if (!rdy && n_pend == kStages) {
@@ -150,7 +173,7 @@ __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
           ok = false;
           break;
         }
-        const int kx = chunk_at(d, kc, a.n_k);
+        const int kx = chunk_at(d, kc, c0, c1);
         mbar_arrive_expect_tx(&S->full[stage], tx);
         tma_load_2d_hint(ring + stage * kStageBytes, tmap_w, &S->full[stage],
                          kx * kBK, tile * kBM, stream_policy);
@@ -201,21 +224,23 @@ template <int R>
 __device__ void mma(const FusedArgs& a, unsigned char* ring, FusedSmem<R>* S,
                     uint32_t tmem_base, volatile int* abort_v) {
   constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN);
-  const int n_my = my_tiles(a.n_tiles);
+  const Share sh(a.n_tiles, a.n_k);
   int stage = 0;
   uint32_t phase = 0;
   int acc = 0;
   uint32_t acc_phase = 0;
   bool ok = true;
   for (int d = 0; d < a.B && ok; ++d) {
-    for (int i = 0; i < n_my && ok; ++i) {
+    for (int i = 0; i < sh.n && ok; ++i) {
+      int tile, c0, c1;
+      sh.unit(d, i, a.n_k, tile, c0, c1);
       if (!mbar_wait_bounded(&S->acc_empty[acc], acc_phase ^ 1u, abort_v, a.limit_ns)) {
         ok = false;
         break;
       }
       tc_fence_after_sync();
       const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * kBN);
-      for (int kc = 0; kc < a.n_k; ++kc) {
+      for (int kc = 0; kc < c1 - c0; ++kc) {
         if (!mbar_wait_bounded(&S->full[stage], phase, abort_v, a.limit_ns)) {
           ok = false;
           break;
@@ -270,84 +295,93 @@ __device__ void merge_stage(const CUtensorMap* tmap_w, const FusedArgs& a,
   if (d > 0) (void)ld_acquire_gpu(&a.ready[d]);   // pool of earlier stages
 #pragma unroll 1
   for (int c = ew; c < rows; c += kEpiWarps) {
+    const int req = c / rpq, j0 = c - req * rpq;
+    // PCTree: this row's children belong to frontier slot j0.  Shared-Markov:
+    // the chain row's children go to every slot of the request.
+    const int j_lo = a.shared ? 0 : j0, j_hi = a.shared ? b_d : j0 + 1;
+    int32_t* tok = a.pool_tok + static_cast<size_t>(req) * a.P;
+    int32_t* par = a.pool_par + static_cast<size_t>(req) * a.P;
+    float2* sc = a.pool_s + static_cast<size_t>(req) * a.P;
+    const float* cz = a.cand_z + static_cast<size_t>(c) * grid * k;
+    const int32_t* ct = a.cand_t + static_cast<size_t>(c) * grid * k;
+    // Loads that do not depend on one another go out together: the parent's
+    // pool id, the first (best) entry of every CTA's list and the
+    // normaliser partials.  Other CTAs wrote all of these during this
+    // launch: L2 loads (__ldcg), as for every cross-CTA read below -- this
+    // SM's L1 may still hold the same addresses from an earlier stage.
+    const int pid0 = __ldcg(a.front + req * k + j_lo);
+    float fz[kG];
+    int ft[kG];
+#pragma unroll
+    for (int u = 0; u < kG; ++u) {
+      const int g = u * 32 + lane;
+      fz[u] = g < grid ? __ldcg(cz + static_cast<size_t>(g) * k) : kNegInf;
+      ft[u] = g < grid ? __ldcg(ct + static_cast<size_t>(g) * k) : 0x7fffffff;
+    }
     // log-softmax normaliser of parent row c over all CTAs' partials (Eq. 2)
     const float lse = warp_lse_from_partials<8>(
         a.part_m + static_cast<size_t>(c) * grid,
         a.part_s + static_cast<size_t>(c) * grid, grid);
+    const float2 sp0 = __ldcg(sc + pid0);
     if (lse == kNegInf && lane == 0) set_status(a.status, PCTREE_ERR_NONFINITE);
     // Every CTA list is sorted best first.  Pass 1: the top-k of the CTAs'
     // first entries; its k-th value T is a lower bound of the row's k-th
     // value (k distinct CTAs hold an entry >= T).  Pass 2: only CTAs whose
     // first entry is >= T can hold further children; their lower ranks are
-    // offered.  Loops stay rolled: this code runs once per stage.
-    const float* cz = a.cand_z + static_cast<size_t>(c) * grid * k;
-    const int32_t* ct = a.cand_t + static_cast<size_t>(c) * grid * k;
-    float(*sz)[32] = S->u.stage.z[ew];
-    int(*st)[32] = S->u.stage.t[ew];
+    // gathered into one list and loaded in warp-wide batches.
+    WarpList lst;
+    lst.seed(fz[0], ft[0], k);
+#pragma unroll 1
+    for (int u = 1; u < kG; ++u) lst.offer(fz[u], ft[u], k);
+    const float T = __shfl_sync(kFull, lst.v, k - 1);
+    int* qlist = S->u.stage.cta[ew];   // CTAs that reach T
+    int nq = 0;
 #pragma unroll
     for (int u = 0; u < kG; ++u) {
-      const int g = u * 32 + lane;
-      // other CTAs wrote these during this launch: L2 loads (__ldcg), as
-      // for every cross-CTA read below -- this SM's L1 may still hold the
-      // same addresses from an earlier stage
-      const float v = g < grid ? __ldcg(cz + static_cast<size_t>(g) * k) : kNegInf;
-      const int t = g < grid ? __ldcg(ct + static_cast<size_t>(g) * k) : 0x7fffffff;
-      sz[u][lane] = v;
-      st[u][lane] = t;
+      const bool qual = u * 32 + lane < grid && fz[u] >= T && ft[u] != 0x7fffffff;
+      const unsigned q = __ballot_sync(kFull, qual);
+      if (qual) qlist[nq + __popc(q & ((1u << lane) - 1u))] = u * 32 + lane;
+      nq += __popc(q);
     }
     __syncwarp();
-    WarpList lst;
-    lst.seed(sz[0][lane], st[0][lane], k);
+    const int km1 = k - 1;
+    const int n_low = nq * km1;              // ranks 1..k-1 of those CTAs
+    constexpr int kJ = 4;
 #pragma unroll 1
-    for (int u = 1; u < kG; ++u) lst.offer(sz[u][lane], st[u][lane], k);
-    const float T = __shfl_sync(kFull, lst.v, k - 1);
-#pragma unroll 1
-    for (int u = 0; u < kG; ++u) {
-      unsigned q = __ballot_sync(kFull, u * 32 + lane < grid && sz[u][lane] >= T &&
-                                            st[u][lane] != 0x7fffffff);
-      // ranks 1..k-1 of up to 32/(k-1) qualifying CTAs per warp-wide load
-      while (q) {
-        const int per = 32 / (k - 1 > 0 ? k - 1 : 1);
-        int g_lane = -1, r_lane = 0;
-        unsigned take = q;
-        for (int n = 0; n < per && take; ++n) {
-          const int src = __ffs(take) - 1;
-          take &= take - 1;
-          if (k > 1 && lane >= n * (k - 1) && lane < (n + 1) * (k - 1)) {
-            g_lane = u * 32 + src;
-            r_lane = 1 + lane - n * (k - 1);
-          }
+    for (int f0 = 0; f0 < n_low; f0 += 32 * kJ) {
+      float v[kJ];
+      int t[kJ];
+#pragma unroll
+      for (int j = 0; j < kJ; ++j) {
+        const int f = f0 + j * 32 + lane;
+        v[j] = kNegInf;
+        t[j] = 0x7fffffff;
+        if (f < n_low) {
+          const int g = qlist[f / km1];
+          const int r = 1 + f - (f / km1) * km1;
+          v[j] = __ldcg(cz + static_cast<size_t>(g) * k + r);
+          t[j] = __ldcg(ct + static_cast<size_t>(g) * k + r);
         }
-        q = take;
-        float v = kNegInf;
-        int t = 0x7fffffff;
-        if (g_lane >= 0) {
-          v = __ldcg(cz + static_cast<size_t>(g_lane) * k + r_lane);
-          t = __ldcg(ct + static_cast<size_t>(g_lane) * k + r_lane);
-        }
-        const bool ok = g_lane >= 0 && v >= T && t != 0x7fffffff;
-        lst.offer(ok ? v : kNegInf, ok ? t : 0x7fffffff, k);
+      }
+#pragma unroll
+      for (int j = 0; j < kJ; ++j) {
+        const bool ok = v[j] >= T && t[j] != 0x7fffffff;
+        lst.offer(ok ? v[j] : kNegInf, ok ? t[j] : 0x7fffffff, k);
       }
     }
     __syncwarp();
-    const int req = c / rpq, j0 = c - req * rpq;
-    int32_t* tok = a.pool_tok + static_cast<size_t>(req) * a.P;
-    int32_t* par = a.pool_par + static_cast<size_t>(req) * a.P;
-    float2* sc = a.pool_s + static_cast<size_t>(req) * a.P;
     int t = lst.t;
     float logpi = lst.v - lse;
     if (t < 0 || t >= a.V) {
       t = 0;
       logpi = kNegInf;
     }
-    // PCTree: this row's children belong to frontier slot j0.  Shared-Markov:
-    // the chain row's children go to every slot of the request.
-    const int j_lo = a.shared ? 0 : j0, j_hi = a.shared ? b_d : j0 + 1;
     for (int j = j_lo; j < j_hi; ++j) {
-      const int pid = __ldcg(a.front + req * k + j);
+      const int pid = j == j_lo ? pid0 : __ldcg(a.front + req * k + j);
+      const float2 sp = j == j_lo ? sp0 : __ldcg(sc + pid);
       if (lane < k) {
         const int id = base + j * k + lane;
-        const float2 sn = ff_add(__ldcg(sc + pid), logpi);   // Eq. 4
+        const float2 sn = ff_add(sp, logpi);   // Eq. 4
         tok[id] = t;
         par[id] = pid;
         sc[id] = sn;
@@ -444,9 +478,9 @@ __device__ void epilogue(const CUtensorMap* tmap_w, const FusedArgs& a,
   const int tid = ew * 32 + lane;
   const int grid = gridDim.x;
   const int k = a.k;
-  const int n_my = my_tiles(a.n_tiles);
+  const Share sh(a.n_tiles, a.n_k);
   uint32_t acc_phase = 0;
-  int g_tile = 0;                          // tiles issued by the MMA so far
+  int g_tile = 0;                          // units issued by the MMA so far
   bool bad = false;
   for (int d = 0; d < a.B; ++d) {
     const int rpq = a.shared ? 1 : (d == 0 ? 1 : k);   // rows per request
@@ -461,9 +495,11 @@ __device__ void epilogue(const CUtensorMap* tmap_w, const FusedArgs& a,
     }
     bool ok = true;
     bool first = true;                     // first tile of this stage
-    for (int i = 0; i < n_my; ++i, ++g_tile) {
+    for (int i = 0; i < sh.n; ++i, ++g_tile) {
       if ((g_tile & 1) != grp) continue;
-      const int tile = tile_at(d, i, n_my);
+      int tile, c0, c1;
+      sh.unit(d, i, a.n_k, tile, c0, c1);
+      const bool cut = c1 - c0 < a.n_k;    // a tile shared with a neighbour
       // the lanes agree before the warp-collective TMEM load
       if (!__all_sync(kFull, mbar_wait_bounded(&S->acc_full[grp], acc_phase, abort_v,
                                                a.limit_ns))) {
@@ -479,6 +515,33 @@ __device__ void epilogue(const CUtensorMap* tmap_w, const FusedArgs& a,
       tc_fence_before_sync();
       __syncwarp();
       if (lane == 0) mbar_arrive(&S->acc_empty[grp]);
+      if (cut) {
+        const int bnd = sh.boundary(c0);
+        float* xp = a.xch +
+                    (static_cast<size_t>(d & 1) * kFusedMaxGrid + bnd) * (kBN * kBM) +
+                    quad * 32 + lane;
+        int* flag = a.xflag + bnd * 4 + quad;
+        if (i == 0) {
+          // first unit of the walk: hand the partial sums to the neighbour,
+          // which reaches this tile as its last unit
+#pragma unroll
+          for (int c = 0; c < R; ++c)
+            if (c < rows) __stcg(xp + c * kBM, acc[c]);
+          __threadfence();
+          __syncwarp();
+          if (lane == 0) st_release_gpu(flag, d + 1);
+          continue;
+        }
+        // last unit of the walk: the neighbour exported its part of this
+        // tile when it began the stage
+        if (!__all_sync(kFull, wait_at_least_bounded(flag, d + 1, abort_v, a.limit_ns))) {
+          ok = false;
+          break;
+        }
+#pragma unroll
+        for (int c = 0; c < R; ++c)
+          if (c < rows) acc[c] += __ldcg(xp + c * kBM);
+      }
       const int v = tile * kBM + quad * 32 + lane;
       const bool inb = v < a.V;
       const float* Lrow = a.L + static_cast<size_t>(d) * a.V + (inb ? v : 0);
@@ -545,27 +608,44 @@ __device__ void epilogue(const CUtensorMap* tmap_w, const FusedArgs& a,
     // per-CTA partials, one row per warp (rolled: runs once per stage)
 #pragma unroll 1
     for (int c = ew; c < rows; c += kEpiWarps) {
-      float mm = kNegInf, ss = 0.0f;
+      // this CTA's normaliser partial of row c: the max over its 256
+      // threads first, then one exponential per thread partial
+      float mv[kEpiWarps], sv[kEpiWarps];
+      float mm = kNegInf;
 #pragma unroll
-      for (int q = 0; q < kEpiWarps; ++q)
-        lse_merge(mm, ss, S->u.part.m[c][q * 32 + lane], S->u.part.s[c][q * 32 + lane]);
-#pragma unroll 1
-      for (int o = 16; o > 0; o >>= 1) {
-        const float m2 = __shfl_xor_sync(kFull, mm, o);
-        const float s2 = __shfl_xor_sync(kFull, ss, o);
-        lse_merge(mm, ss, m2, s2);
+      for (int q = 0; q < kEpiWarps; ++q) {
+        mv[q] = S->u.part.m[c][q * 32 + lane];
+        sv[q] = S->u.part.s[c][q * 32 + lane];
+        mm = fmaxf(mm, mv[q]);
       }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) mm = fmaxf(mm, __shfl_xor_sync(kFull, mm, o));
+      float ss = 0.0f;
+      if (mm > kNegInf) {
+#pragma unroll
+        for (int q = 0; q < kEpiWarps; ++q) ss += sv[q] * expf(mv[q] - mm);
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(kFull, ss, o);
       if (lane == 0) {
         a.part_m[static_cast<size_t>(c) * grid + blockIdx.x] = mm;
         a.part_s[static_cast<size_t>(c) * grid + blockIdx.x] = ss;
       }
+      // the eight warp lists, 32 / k of them per warp-wide batch: the first
+      // batch is sorted in one go, the others offered
+      const int per = 32 / k;
       WarpList cl;
-      cl.seed(lane < k ? S->lv[0][c][lane] : kNegInf,
-              lane < k ? S->lt[0][c][lane] : 0x7fffffff, k);
+      {
+        const int w = lane / k, e = lane - w * k;
+        const bool has = w < per && w < kEpiWarps;
+        cl.seed(has ? S->lv[w][c][e] : kNegInf, has ? S->lt[w][c][e] : 0x7fffffff, k);
+      }
 #pragma unroll 1
-      for (int w = 1; w < kEpiWarps; ++w)
-        cl.offer(lane < k ? S->lv[w][c][lane] : kNegInf,
-                 lane < k ? S->lt[w][c][lane] : 0x7fffffff, k);
+      for (int w0 = per; w0 < kEpiWarps; w0 += per) {
+        const int w = w0 + lane / k, e = lane - (lane / k) * k;
+        const bool has = lane < per * k && w < kEpiWarps;
+        cl.offer(has ? S->lv[w][c][e] : kNegInf, has ? S->lt[w][c][e] : 0x7fffffff, k);
+      }
       if (lane < k) {   // this CTA's top-k of row c, best first
         const size_t o = (static_cast<size_t>(c) * grid + blockIdx.x) * k + lane;
         a.cand_z[o] = cl.v;

@@ -393,6 +393,29 @@ __device__ __forceinline__ bool wait_flag_bounded(const int* flag,
   }
 }
 
+// Spins until *flag >= v (a counter another CTA raises with a release
+// store); gives up after `limit_ns` or once `*abort` is set.
+__device__ __forceinline__ bool wait_at_least_bounded(const int* flag, int v,
+                                                      volatile int* abort,
+                                                      uint64_t limit_ns) {
+  if (ld_relaxed_gpu(flag) >= v) {
+    fence_acq_rel_gpu();
+    return true;
+  }
+  const uint64_t t0 = global_timer_ns();
+  for (uint32_t it = 1;; ++it) {
+    __nanosleep(64);
+    if (ld_relaxed_gpu(flag) >= v) {
+      fence_acq_rel_gpu();
+      return true;
+    }
+    if ((it & 15) == 0) {
+      if (*abort) return false;
+      if (global_timer_ns() - t0 > limit_ns) return false;
+    }
+  }
+}
+
 // Orders this thread's generic-proxy global accesses against async-proxy
 // (TMA) accesses: used between writing data that another CTA will read with
 // TMA and publishing it, and between observing such a flag and the TMA load.
