@@ -33,6 +33,7 @@ constexpr int kBK = 64;           // K elements per ring stage (128 B of bf16)
 constexpr int kUmmaK = 16;        // K per tcgen05.mma kind::f16
 constexpr int kThreads = 192;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per bounded wait
+constexpr int kLGroup = 16;       // requests whose base logits load together
 
 template <int BN>
 struct TcCfg {
@@ -44,9 +45,10 @@ struct TcCfg {
   static constexpr int kTmemCols =
       (2 * BN) <= 32 ? 32 : (2 * BN) <= 64 ? 64 : (2 * BN) <= 128 ? 128
                         : (2 * BN) <= 256 ? 256 : 512;
+  static constexpr size_t kLBytes = kLGroup * kBM * sizeof(float);
   static constexpr size_t kSmemBytes =
       1024 /*alignment slack*/ + static_cast<size_t>(kStages) * kStageBytes +
-      256 /*barriers*/;
+      kLBytes + 256 /*barriers*/;
 };
 
 template <int BN>
@@ -61,7 +63,11 @@ markov_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   unsigned char* ring = smem;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(ring + C::kStages * C::kStageBytes);
+  // base logits of up to kLGroup requests at each epilogue thread's
+  // vocabulary entry ([request][row of tile]; each thread owns its column)
+  float(*sl)[kBM] = reinterpret_cast<float(*)[kBM]>(ring + C::kStages * C::kStageBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ring + C::kStages * C::kStageBytes +
+                                               C::kLBytes);
   uint64_t* full = bars;                      // [kStages]
   uint64_t* empty = bars + C::kStages;        // [kStages]
   uint64_t* acc_full = bars + 2 * C::kStages; // [2]
@@ -197,41 +203,64 @@ markov_tc_kernel(const __grid_constant__ CUtensorMap tmap_w,
     int acc = 0;
     uint32_t acc_phase = 0;
     bool bad = false;
-    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
-      // the lanes agree before the warp-collective TMEM loads
-      if (!__all_sync(0xffffffffu, mbar_wait_bounded(&acc_full[acc], acc_phase, abort_v,
-                                                     kWaitLimitNs))) {
-        *abort_v = 1;
-        set_status(status, PCTREE_ERR_TIMEOUT);
-        break;
-      }
-      tc_fence_after_sync();
+    const int req_lo = col0 / rows_per_req;
+    const int req_hi = (col0 + cols - 1) / rows_per_req;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
       const int v = tile * kBM + r_in_tile;
+      const bool inb = v < V;
       const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
                              static_cast<uint32_t>(acc * BN);
-      int cur_req = -1;
-      float lval = 0.0f;
-      for (int c0 = 0; c0 < cols; c0 += 16) {
-        uint32_t r[16];
-        tmem_ld_32x32b_x16(t_row + c0, r);
-        tmem_ld_wait();
-        if (v < V) {
+      for (int g0 = req_lo; g0 <= req_hi; g0 += kLGroup) {
+        // the group's base logits, as independent loads issued together
+        // (for the first group: before the accumulator wait)
+        float lv[kLGroup];
+#pragma unroll
+        for (int q = 0; q < kLGroup; ++q)
+          lv[q] = inb && g0 + q <= req_hi
+                      ? __ldg(L + static_cast<long long>(g0 + q) * l_req_stride + v)
+                      : 0.0f;
+        if (g0 == req_lo) {
+          // the lanes agree before the warp-collective TMEM loads
+          if (!__all_sync(0xffffffffu, mbar_wait_bounded(&acc_full[acc], acc_phase,
+                                                         abort_v, kWaitLimitNs))) {
+            *abort_v = 1;
+            set_status(status, PCTREE_ERR_TIMEOUT);
+            ok = false;
+            break;
+          }
+          tc_fence_after_sync();
+        }
+#pragma unroll
+        for (int q = 0; q < kLGroup; ++q) sl[q][r_in_tile] = lv[q];
+        // pass-relative columns of the group's requests
+        const int c_lo = max(col0, g0 * rows_per_req) - col0;
+        const int c_hi = min(col0 + cols, (g0 + kLGroup) * rows_per_req) - col0;
+        int q = (col0 + c_lo) / rows_per_req - g0;      // request of column c_lo
+        int next = (g0 + q + 1) * rows_per_req - col0;  // its first column after
+        for (int c0 = c_lo & ~15; c0 < c_hi; c0 += 16) {
+          uint32_t r[16];
+          tmem_ld_32x32b_x16(t_row + c0, r);
+          tmem_ld_wait();
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
-            const int col = col0 + c0 + j;
-            if (c0 + j < cols) {
-              const int req = col / rows_per_req;
-              if (req != cur_req) {
-                cur_req = req;
-                lval = L[static_cast<long long>(req) * l_req_stride + v];
+            const int c = c0 + j;
+            if (c >= c_lo && c < c_hi) {
+              if (c == next) {
+                ++q;
+                next += rows_per_req;
               }
-              const float z = lval + __uint_as_float(r[j]);
-              bad |= isnan(z) || (isinf(z) && !(isinf(lval) && lval < 0.0f)) ;
-              Z[static_cast<size_t>(col) * ldz + v] = z;
+              if (inb) {
+                const float lval = sl[q][r_in_tile];
+                const float z = lval + __uint_as_float(r[j]);
+                bad |= isnan(z) || (isinf(z) && !(isinf(lval) && lval < 0.0f));
+                Z[static_cast<size_t>(col0 + c) * ldz + v] = z;
+              }
             }
           }
         }
       }
+      if (!ok) break;
       tc_fence_before_sync();
       __syncwarp();
       if (lane == 0) mbar_arrive(&acc_empty[acc]);
