@@ -63,148 +63,134 @@ __global__ void init_kernel(const int32_t* __restrict__ root, const void* E_in,
 }
 
 // ---------------------------------------------------------------------------
-// partials: one CTA per (chunk of kChunk logits, row)
+// partials: one warp per (row, chunk of kChunk logits)
 // ---------------------------------------------------------------------------
 
-constexpr int kCandCap = 256;      // candidates a chunk may hold in shared memory
+constexpr int kPartWarps = 8;      // warps (work items) per CTA
+constexpr int kPartVec = 4;        // float4 loads per lane and step
+constexpr int kPartVals = 4 * kPartVec;        // logits per lane and step
+constexpr int kPartStep = 32 * kPartVals;      // logits per warp and step
 
-__global__ void __launch_bounds__(kChunkThreads, 3)
+// Per (row, chunk): the chunk's (max, sum of exp) and its k best logits with
+// their tokens, best first (padding (-inf, INT_MAX) when the chunk holds
+// fewer than k).  The warp streams the chunk in steps of 512 logits (16 per
+// lane, float4 loads, all in flight before use).  Each lane keeps an online
+// max / sum of exp with one rescale per step.  The warp keeps a sorted top-k
+// list; each lane marks its logits that beat the list's k-th entry and the
+// warp offers one marked logit per lane at a time, so a step costs as many
+// offers as its busiest lane has marks (usually none or one).
+__global__ void __launch_bounds__(32 * kPartWarps, 3)
 partials_kernel(const float* __restrict__ Z, int ldz, int V, int k,
-                int n_chunks, float* __restrict__ part_m,
+                int n_chunks, int rows, float* __restrict__ part_m,
                 float* __restrict__ part_s, float* __restrict__ part_z,
                 int32_t* __restrict__ part_t, int32_t* status) {
-  const int chunk = blockIdx.x;
-  const int row = blockIdx.y;
   const int lane = threadIdx.x & 31;
-  const int warp = threadIdx.x >> 5;
-  constexpr int kWarps = kChunkThreads / 32;
-  __shared__ float sm_m[kWarps], sm_s[kWarps], sm_kth[kWarps];
-  __shared__ float sm_v[kCandCap];
-  __shared__ int sm_t[kCandCap];
-  __shared__ int sm_count;
-
-  const float* z_row = Z + static_cast<size_t>(row) * ldz;
+  const int item = blockIdx.x * kPartWarps + (threadIdx.x >> 5);
+  if (item >= rows * n_chunks) return;
+  const int row = item / n_chunks;
+  const int chunk = item - row * n_chunks;
   const int v0 = chunk * kChunk;
-  constexpr int kPer = kChunk / kChunkThreads;
-  float zs[kPer];
-  // every load of the chunk in flight at once; selection work afterwards
-#pragma unroll
-  for (int i = 0; i < kPer; ++i) {
-    const int v = v0 + i * kChunkThreads + threadIdx.x;
-    zs[i] = v < V ? z_row[v] : kNegInf;
-  }
-  if (threadIdx.x == 0) sm_count = 0;
-  // this thread's max, then its sum of exp relative to it (no branches)
-  float tmax = kNegInf;
+  const int len = min(kChunk, V - v0);
+  const float* z_row = Z + static_cast<size_t>(row) * ldz + v0;
+  float m = kNegInf, s = 0.0f;
   bool bad = false;
+  WarpList lst;
+  lst.reset();
+  // value i of this lane in the step at b is logit b + (i / 4) * 128 +
+  // lane * 4 + i % 4; slots past the chunk hold -inf
+  auto load_step = [&](int b, float (&z)[kPartVals]) {
 #pragma unroll
-  for (int i = 0; i < kPer; ++i) {
-    bad |= is_nonfinite_logit(zs[i]);
-    tmax = fmaxf(tmax, zs[i]);
-  }
-  float tsum = 0.0f;
-  if (tmax != kNegInf) {
+    for (int j = 0; j < kPartVec; ++j) {
+      const int o = b + j * 128 + lane * 4;
+      if (o + 3 < len) {
+        const float4 q = __ldcs(reinterpret_cast<const float4*>(z_row + o));
+        z[4 * j] = q.x;
+        z[4 * j + 1] = q.y;
+        z[4 * j + 2] = q.z;
+        z[4 * j + 3] = q.w;
+      } else {
 #pragma unroll
-    for (int i = 0; i < kPer; ++i) tsum += __expf(zs[i] - tmax);
+        for (int e = 0; e < 4; ++e) z[4 * j + e] = o + e < len ? z_row[o + e] : kNegInf;
+      }
+    }
+  };
+  float zn[kPartVals];
+  load_step(0, zn);
+#pragma unroll 1
+  for (int b = 0; b < len; b += kPartStep) {
+    float z[kPartVals];
+#pragma unroll
+    for (int i = 0; i < kPartVals; ++i) z[i] = zn[i];
+    if (b + kPartStep < len) load_step(b + kPartStep, zn);   // next step in flight
+    float lm = kNegInf;
+    int li = 0;
+#pragma unroll
+    for (int i = 0; i < kPartVals; ++i) {
+      bad |= is_nonfinite_logit(z[i]);
+      if (z[i] > lm) {
+        lm = z[i];
+        li = i;
+      }
+    }
+    if (lm > m) {
+      s = m == kNegInf ? 0.0f : s * __expf(m - lm);
+      m = lm;
+    }
+    if (m != kNegInf) {
+#pragma unroll
+      for (int i = 0; i < kPartVals; ++i) s += __expf(z[i] - m);
+    }
+    const int tbase = v0 + b + lane * 4;
+    unsigned skip = 0;
+    if (b == 0) {
+      // first step: the list starts from the 32 lanes' best logits (a sort
+      // instead of serial inserts into an empty list)
+      const int lt = lm > kNegInf ? tbase + (li >> 2) * 128 + (li & 3) : 0x7fffffff;
+      lst.seed(lm > kNegInf ? lm : kNegInf, lt, k);
+      if (lm > kNegInf) skip = 1u << li;
+    }
+    // logits that beat the list's k-th entry (out-of-range slots hold -inf
+    // and the sentinel token, which beats nothing)
+    const float tv = __shfl_sync(kFull, lst.v, k - 1);
+    const int tt = __shfl_sync(kFull, lst.t, k - 1);
+    unsigned marks = 0;
+#pragma unroll
+    for (int i = 0; i < kPartVals; ++i) {
+      const int o = b + (i >> 2) * 128 + lane * 4 + (i & 3);
+      const int tok = o < len ? tbase + (i >> 2) * 128 + (i & 3) : 0x7fffffff;
+      if (cand_better(z[i], tok, tv, tt)) marks |= 1u << i;
+    }
+    marks &= ~skip;
+    while (__any_sync(kFull, marks != 0)) {
+      const int sel = marks != 0 ? __ffs(marks) - 1 : -1;
+      marks &= marks - 1;
+      float cv = kNegInf;
+      int ct = 0x7fffffff;
+#pragma unroll
+      for (int i = 0; i < kPartVals; ++i) {
+        if (i == sel) {
+          cv = z[i];
+          ct = tbase + (i >> 2) * 128 + (i & 3);
+        }
+      }
+      lst.offer(cv, ct, k);
+    }
   }
   if (bad) set_status(status, PCTREE_ERR_NONFINITE);
-  float m = tmax, s = tsum;
+#pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     const float m2 = __shfl_xor_sync(kFull, m, o);
     const float s2 = __shfl_xor_sync(kFull, s, o);
     lse_merge(m, s, m2, s2);
   }
-  // a warp's k-th largest thread maximum bounds the chunk's k-th largest
-  // logit from below (k distinct threads hold a logit >= it), and so does
-  // the largest such value over the warps: only logits >= that floor can
-  // enter the chunk's top-k
-  WarpList lst;
-  lst.seed(tmax, threadIdx.x, k);
-  const float warp_kth = __shfl_sync(kFull, lst.v, k - 1);
-  if (lane == 0) {
-    sm_m[warp] = m;
-    sm_s[warp] = s;
-    sm_kth[warp] = warp_kth;
-  }
-  __syncthreads();
-  float floor_z = sm_kth[0];
-#pragma unroll
-  for (int w = 1; w < kWarps; ++w) floor_z = fmaxf(floor_z, sm_kth[w]);
   const size_t p = static_cast<size_t>(row) * n_chunks + chunk;
-  if (warp == 0) {
-    float mm = lane < kWarps ? sm_m[lane] : kNegInf;
-    float ss = lane < kWarps ? sm_s[lane] : 0.0f;
-    for (int o = 16; o > 0; o >>= 1) {
-      const float m2 = __shfl_xor_sync(kFull, mm, o);
-      const float s2 = __shfl_xor_sync(kFull, ss, o);
-      lse_merge(mm, ss, m2, s2);
-    }
-    if (lane == 0) {
-      part_m[p] = mm;
-      part_s[p] = ss;
-    }
+  if (lane == 0) {
+    part_m[p] = m;
+    part_s[p] = s;
   }
-  // candidates (logits >= the floor) appended to shared memory, one atomic
-  // per warp and round
-#pragma unroll
-  for (int i = 0; i < kPer; ++i) {
-    const int v = v0 + i * kChunkThreads + threadIdx.x;
-    const bool pass = v < V && zs[i] >= floor_z;
-    const unsigned mask = __ballot_sync(kFull, pass);
-    if (mask) {
-      int base = 0;
-      if (lane == 0) base = atomicAdd(&sm_count, __popc(mask));
-      base = __shfl_sync(kFull, base, 0);
-      const int slot = base + __popc(mask & ((1u << lane) - 1u));
-      if (pass && slot < kCandCap) {
-        sm_v[slot] = zs[i];
-        sm_t[slot] = v;
-      }
-    }
-  }
-  __syncthreads();
-  const int count = sm_count;
-  if (count <= kCandCap) {
-    // rank of each candidate among the others (tokens are distinct)
-    for (int i = threadIdx.x; i < count; i += blockDim.x) {
-      const float cv = sm_v[i];
-      const int ct = sm_t[i];
-      int rank = 0;
-      for (int j = 0; j < count; ++j) rank += cand_better(sm_v[j], sm_t[j], cv, ct);
-      if (rank < k) {
-        part_z[p * k + rank] = cv;
-        part_t[p * k + rank] = ct;
-      }
-    }
-    // fewer candidates than k (a short last chunk): padding entries
-    for (int i = count + threadIdx.x; i < k; i += blockDim.x) {
-      part_z[p * k + i] = kNegInf;
-      part_t[p * k + i] = 0x7fffffff;
-    }
-    return;
-  }
-  // many logits at the floor (ties): every warp keeps a list of its
-  // candidates, warp 0 merges them
-  __syncthreads();
-  lst.reset();
-#pragma unroll
-  for (int i = 0; i < kPer; ++i) {
-    const int v = v0 + i * kChunkThreads + threadIdx.x;
-    const bool pass = v < V && zs[i] >= floor_z;
-    if (__any_sync(kFull, pass))
-      lst.offer(pass ? zs[i] : kNegInf, pass ? v : 0x7fffffff, k);
-  }
-  sm_v[warp * 32 + lane] = lst.v;
-  sm_t[warp * 32 + lane] = lst.t;
-  __syncthreads();
-  if (warp == 0) {
-    for (int w = 1; w < kWarps; ++w)
-      lst.offer(lane < k ? sm_v[w * 32 + lane] : kNegInf,
-                lane < k ? sm_t[w * 32 + lane] : 0x7fffffff, k);
-    if (lane < k) {
-      part_z[p * k + lane] = lst.v;
-      part_t[p * k + lane] = lst.t;
-    }
+  if (lane < k) {
+    part_z[p * k + lane] = lst.v;
+    part_t[p * k + lane] = lst.t;
   }
 }
 
@@ -658,10 +644,11 @@ cudaError_t launch_init(const pctree_config& c, const Layout& lay,
 cudaError_t launch_partials(const Layout& lay, int k, int V, int rows,
                             unsigned char* ws, int32_t* status,
                             cudaStream_t stream) {
-  dim3 grid(lay.n_chunks, rows);
-  partials_kernel<<<grid, kChunkThreads, 0, stream>>>(
+  const int items = rows * lay.n_chunks;
+  const int grid = (items + kPartWarps - 1) / kPartWarps;
+  partials_kernel<<<grid, 32 * kPartWarps, 0, stream>>>(
       reinterpret_cast<const float*>(ws + lay.off_z), lay.ldz, V, k,
-      lay.n_chunks, reinterpret_cast<float*>(ws + lay.off_pm),
+      lay.n_chunks, rows, reinterpret_cast<float*>(ws + lay.off_pm),
       reinterpret_cast<float*>(ws + lay.off_ps),
       reinterpret_cast<float*>(ws + lay.off_pz),
       reinterpret_cast<int32_t*>(ws + lay.off_pt), status);
