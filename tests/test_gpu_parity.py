@@ -36,6 +36,9 @@ SMALL = {
     "k32_bf16": strong(BASE, V=4096, H=64, B=3, k=32, N=200, batch=1, seed=17),
     "B1_bf16": strong(BASE, V=999, H=64, B=1, k=5, N=4, batch=2, seed=18),
     "weak_head_bf16": BASE.with_(V=20000, H=512, B=6, k=8, N=32, batch=2, seed=19),
+    # more W_out tiles than SMs and a ragged K chunk (64 + 64 + 8): the fused
+    # round's equal shares cut tiles between neighbouring CTAs
+    "cut_tiles_bf16": strong(BASE, V=40000, H=136, B=5, k=8, N=32, batch=1, seed=26),
     "mixed_temp_bf16": strong(WORKLOADS["14b_b16_bs32"], V=6000, H=128, B=6,
                               k=6, N=24, batch=4, seed=20),
     "f32_pos_offset": WORKLOADS["tiny"].with_(V=3001, H=37, B=5, k=3, N=20,
