@@ -463,46 +463,46 @@ pack_kernel(int B, int k, int N, int P, int pos_offset,
   // breadth-first packing: level by level, (parent's index, token) order
   int* pidx = reinterpret_cast<int*>(sm_key);  // pool id -> packed index
   for (int i = tid; i < P; i += blockDim.x) pidx[i] = -1;
-  __syncthreads();
-  int my_id = tid < n ? sm_sel[tid] : -1;
+  const int my_id = tid < n ? sm_sel[tid] : -1;
   const int my_lvl = my_id >= 0 ? level_of(my_id, k) : -1;
+  // parent and token of this thread's node, loaded once: the level loop
+  // below touches shared memory only
+  const int my_pid = my_id >= 0 ? par[my_id] : -1;
+  const int my_tok = my_id >= 0 ? tok[my_id] : 0;
+  __shared__ unsigned long long sm_k2[PCTREE_MAX_N];
+  __shared__ int sm_kid[PCTREE_MAX_N];
+  __shared__ int sm_lvl_cnt[2];   // nodes of the current level, by parity
+  if (tid == 0) sm_lvl_cnt[0] = 0;
   __syncthreads();
   int placed = 0;
   for (int t = 0; t <= B; ++t) {
+    // the level's nodes take slots; the counter of the next level (last
+    // read before the previous barrier) is cleared meanwhile
     const bool at = my_lvl == t;
     unsigned long long key2 = 0ull;
     if (at) {
-      const int pid = par[my_id];
-      const int pp = (t == 0 || pid < 0 || pid >= P) ? -1 : pidx[pid];
+      const int pp = (t == 0 || my_pid < 0 || my_pid >= P) ? -1 : pidx[my_pid];
       key2 = (static_cast<unsigned long long>(static_cast<unsigned int>(pp + 1)) << 32) |
-             static_cast<unsigned int>(tok[my_id]);
+             static_cast<unsigned int>(my_tok);
+      const int slot = atomicAdd(&sm_lvl_cnt[t & 1], 1);
+      sm_k2[slot] = key2;
+      sm_kid[slot] = my_id;
     }
-    int n_t;
-    block_excl_scan(at ? 1 : 0, sm_warp, &n_t);
-    if (n_t == 0) break;
+    if (tid == 0) sm_lvl_cnt[(t + 1) & 1] = 0;
+    __syncthreads();
+    const int n_t = sm_lvl_cnt[t & 1];
+    if (n_t == 0) break;   // the selection is ancestor-closed: no deeper level
     // rank among the nodes of this level (<= n of them).  Siblings carry
     // distinct tokens, so (parent, token) is unique; the pool id breaks ties
     // anyway so that every packed slot is written exactly once whatever the
     // pool holds (e.g. after a round already flagged non-finite).
-    __shared__ unsigned long long sm_k2[PCTREE_MAX_N];
-    __shared__ int sm_kid[PCTREE_MAX_N];
-    __shared__ int sm_lvl_slot;
-    if (tid == 0) sm_lvl_slot = 0;
-    __syncthreads();
-    int slot = -1;
-    if (at) {
-      slot = atomicAdd(&sm_lvl_slot, 1);
-      sm_k2[slot] = key2;
-      sm_kid[slot] = my_id;
-    }
-    __syncthreads();
     if (at) {
       int rank = 0;
       for (int j = 0; j < n_t; ++j)
         rank += sm_k2[j] < key2 || (sm_k2[j] == key2 && sm_kid[j] < my_id);
       const int a = placed + rank;
       pidx[my_id] = a;
-      sm_sel[a] = my_id;  // safe: slots of this level are read via my_id only
+      sm_sel[a] = my_id;  // safe: sm_sel is not read inside this loop
     }
     placed += n_t;
     __syncthreads();
