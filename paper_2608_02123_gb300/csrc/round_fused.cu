@@ -3,10 +3,12 @@
 // stage (batch * k <= 16, k <= 16) -- the batch-1 drafting of Sec. 5 -- with
 // either child scoring (PCTree, or the Shared-Markov control of Sec. 5.3).
 //
-// Per stage d, every CTA (one per SM) streams its share of W_out tiles with
-// TMA and multiplies them on the tensor cores (tcgen05, bf16 -> f32 in TMEM)
-// against the stage's parent rows X = E_in[parent tokens] (Eq. 3), a 16-row
-// buffer in global memory loaded with one TMA box per ring slot.  The
+// Per stage d, every CTA (one per SM) streams an equal share of the stage's
+// (W_out tile, K chunk) pairs with TMA and multiplies them on the tensor
+// cores (tcgen05, bf16 -> f32 in TMEM) against the stage's parent rows
+// X = E_in[parent tokens] (Eq. 3), a 16-row buffer in global memory loaded
+// with one TMA box per ring slot; a tile cut by a share boundary is finished
+// by one of the two CTAs that share it (see Share below).  The
 // epilogue adds the shared base logits L_d and keeps, per parent row, a
 // running log-sum-exp (Eq. 2) and a warp-resident top-k list -- the stage
 // logits never reach HBM.  When a CTA has finished its tiles it publishes
@@ -17,10 +19,10 @@
 // prefetching the next stage's W_out tiles while that merge runs and only
 // hold back the parent-row loads until the flag is set.
 //
-// Consecutive stages walk the vocabulary tiles in opposite directions, so a
-// stage begins with the tiles the previous stage read last; W_out is read
-// with an L2 evict_first policy, so those are the tiles most likely to still
-// sit in L2.
+// Consecutive stages walk a CTA's (tile, chunk) pairs in opposite
+// directions, so a stage begins with the data the previous stage read last;
+// W_out is read with an L2 evict_first policy, so that data is the most
+// likely to still sit in L2.
 //
 // Warp roles (320 threads): warp 0 TMA producer, warp 1 TMEM allocator + MMA
 // issuer, warps 2..9 epilogue in two groups of four, group h reading TMEM
