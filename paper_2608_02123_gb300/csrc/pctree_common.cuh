@@ -13,8 +13,7 @@
 namespace pct {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kChunk = 8192;          // vocabulary entries per partials CTA
-constexpr int kChunkThreads = 256;
+constexpr int kChunk = 8192;          // vocabulary entries per partials work item
 
 // ---------------------------------------------------------------------------
 // workspace layout (host and device agree through this struct)
