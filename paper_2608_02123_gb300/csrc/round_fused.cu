@@ -331,10 +331,44 @@ __device__ void merge_stage(const CUtensorMap* tmap_w, const FusedArgs& a,
     // value (k distinct CTAs hold an entry >= T).  Pass 2: only CTAs whose
     // first entry is >= T can hold further children; their lower ranks are
     // gathered into one list and loaded in warp-wide batches.
+    // The list starts from each lane's best first entry (one sort); the
+    // lane's other entries are offered only where they beat the k-th of
+    // those, one marked entry per lane at a time.
+    float bz = fz[0];
+    int bt = ft[0], bu = 0;
+#pragma unroll
+    for (int u = 1; u < kG; ++u) {
+      if (cand_better(fz[u], ft[u], bz, bt)) {
+        bz = fz[u];
+        bt = ft[u];
+        bu = u;
+      }
+    }
     WarpList lst;
-    lst.seed(fz[0], ft[0], k);
+    lst.seed(bz, bt, k);
+    {
+      const float tz = __shfl_sync(kFull, lst.v, k - 1);
+      const int tt = __shfl_sync(kFull, lst.t, k - 1);
+      unsigned marks = 0;
+#pragma unroll
+      for (int u = 0; u < kG; ++u)
+        if (u != bu && cand_better(fz[u], ft[u], tz, tt)) marks |= 1u << u;
 #pragma unroll 1
-    for (int u = 1; u < kG; ++u) lst.offer(fz[u], ft[u], k);
+      while (__any_sync(kFull, marks != 0)) {
+        const int sel = marks != 0 ? __ffs(marks) - 1 : -1;
+        marks &= marks - 1;
+        float cv = kNegInf;
+        int cti = 0x7fffffff;
+#pragma unroll
+        for (int u = 0; u < kG; ++u) {
+          if (u == sel) {
+            cv = fz[u];
+            cti = ft[u];
+          }
+        }
+        lst.offer(cv, cti, k);
+      }
+    }
     const float T = __shfl_sync(kFull, lst.v, k - 1);
     int* qlist = S->u.stage.cta[ew];   // CTAs that reach T
     int nq = 0;
