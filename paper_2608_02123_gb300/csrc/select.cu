@@ -12,16 +12,15 @@
 #include <cuda_bf16.h>
 
 #include "pctree_common.cuh"
+#include "sm103_ptx.cuh"
 
 namespace pct {
 
 namespace {
 
 constexpr float kNegInf = -INFINITY;
-
-__device__ __forceinline__ bool is_nonfinite_logit(float z) {
-  return isnan(z) || z == __int_as_float(0x7f800000);
-}
+constexpr float kPosInf = INFINITY;
+constexpr float kLog2e = 1.4426950408889634f;
 
 // Copies one Markov input row E_in[token] into X[row] (bf16: 16-byte words).
 __device__ void copy_row(const void* E_in, void* X, int token, int row, int H,
@@ -122,37 +121,45 @@ partials_kernel(const float* __restrict__ Z, int ldz, int V, int k,
 #pragma unroll
     for (int i = 0; i < kPartVals; ++i) z[i] = zn[i];
     if (b + kPartStep < len) load_step(b + kPartStep, zn);   // next step in flight
+    // non-finite check (NaN or +inf: not below +inf) and the step maximum
     float lm = kNegInf;
-    int li = 0;
+    bool nf = false;
 #pragma unroll
     for (int i = 0; i < kPartVals; ++i) {
-      bad |= is_nonfinite_logit(z[i]);
-      if (z[i] > lm) {
-        lm = z[i];
-        li = i;
-      }
+      nf |= !(z[i] < kPosInf);
+      lm = fmaxf(lm, z[i]);
     }
+    bad |= nf;
     if (lm > m) {
-      s = m == kNegInf ? 0.0f : s * __expf(m - lm);
+      s = m == kNegInf ? 0.0f : s * ex2_approx((m - lm) * kLog2e);
       m = lm;
     }
     if (m != kNegInf) {
+      // exp(z - m) = 2^(z log2 e - m log2 e): one FMA and one ex2 per logit
+      const float mb = m * kLog2e;
 #pragma unroll
-      for (int i = 0; i < kPartVals; ++i) s += __expf(z[i] - m);
+      for (int i = 0; i < kPartVals; ++i) s += ex2_approx(fmaf(z[i], kLog2e, -mb));
     }
     const int tbase = v0 + b + lane * 4;
     unsigned skip = 0;
     if (b == 0) {
       // first step: the list starts from the 32 lanes' best logits (a sort
-      // instead of serial inserts into an empty list)
+      // instead of serial inserts into an empty list); the lowest index
+      // holding the lane's maximum has the lowest token among equal logits
+      int li = 0;
+#pragma unroll
+      for (int i = kPartVals - 1; i >= 0; --i)
+        if (z[i] == lm) li = i;
       const int lt = lm > kNegInf ? tbase + (li >> 2) * 128 + (li & 3) : 0x7fffffff;
       lst.seed(lm > kNegInf ? lm : kNegInf, lt, k);
       if (lm > kNegInf) skip = 1u << li;
     }
     // logits that beat the list's k-th entry (out-of-range slots hold -inf
-    // and the sentinel token, which beats nothing)
+    // and the sentinel token, which beats nothing); a lane whose maximum is
+    // below the k-th value holds none, and most steps have no such lane
     const float tv = __shfl_sync(kFull, lst.v, k - 1);
     const int tt = __shfl_sync(kFull, lst.t, k - 1);
+    if (!__any_sync(kFull, lm >= tv)) continue;
     unsigned marks = 0;
 #pragma unroll
     for (int i = 0; i < kPartVals; ++i) {
