@@ -295,13 +295,44 @@ merge_kernel(int d, int B, int k, int b_d, int rpq, int shared, int V, int H,
         cv[u] = c < n_cand ? cz[c] : kNegInf;
         ci[u] = c < n_cand ? ct[c] : 0x7fffffff;
       }
+      // The first batch seeds the list with each lane's best candidate (one
+      // sort); then every lane offers, one at a time, only its candidates
+      // that beat the list's k-th entry.
+      unsigned skip = 0;
+      if (c0 == 0) {
+        float bv = cv[0];
+        int bi = ci[0], bu = 0;
 #pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
-        if (c0 == 0 && u == 0) {
-          lst.seed(cv[u], ci[u], k);
-        } else {
-          lst.offer(cv[u], ci[u], k);
+        for (int u = 1; u < kUnroll; ++u) {
+          if (cand_better(cv[u], ci[u], bv, bi)) {
+            bv = cv[u];
+            bi = ci[u];
+            bu = u;
+          }
         }
+        lst.seed(bv, bi, k);
+        skip = 1u << bu;
+      }
+      const float tv = __shfl_sync(kFull, lst.v, k - 1);
+      const int tt = __shfl_sync(kFull, lst.t, k - 1);
+      unsigned marks = 0;
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u)
+        if (cand_better(cv[u], ci[u], tv, tt)) marks |= 1u << u;
+      marks &= ~skip;
+      while (__any_sync(kFull, marks != 0)) {
+        const int sel = marks != 0 ? __ffs(marks) - 1 : -1;
+        marks &= marks - 1;
+        float ov = kNegInf;
+        int ot = 0x7fffffff;
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+          if (u == sel) {
+            ov = cv[u];
+            ot = ci[u];
+          }
+        }
+        lst.offer(ov, ot, k);
       }
     }
     int t = lst.t;
