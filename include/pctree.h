@@ -176,7 +176,10 @@ PCTREE_API size_t pctree_workspace_bytes(const pctree_config* cfg);
  *                call.
  * Ranking rules: children of a parent by (log pi desc, token asc); the
  * frontier by (score desc, id asc); the global budget by (score desc, depth
- * asc, id asc), all on float32 scores accumulated along paths in float64.
+ * asc, id asc).  Scores are ranked as float32; along a path they are
+ * accumulated exactly as an unevaluated float pair (hi + lo, each step added
+ * with Knuth's TwoSum), so the only rounding is that of each stage's float32
+ * log-probability.  No float64 arithmetic runs on the device.
  * Errors: PCTREE_ERR_INVALID_ARG / _WORKSPACE / _UNSUPPORTED before any work;
  * PCTREE_ERR_CUDA if a launch fails.
  */
@@ -197,7 +200,8 @@ PCTREE_API pctree_status pctree_draft(const pctree_config* cfg, const float* bas
  * Scratch: a fixed 16 MiB array inside the library, reserved on every GPU
  * that loads it until the process exits; a round whose
  * pctree_workspace_bytes exceeds 16 MiB returns PCTREE_ERR_WORKSPACE before
- * any work (batch-1 Qwen3-shaped rounds need about 5 MB).  The first call on
+ * any work (batch-1 Qwen3-shaped rounds fit: V=151936 with H=2560, B=16,
+ * k=8, N=64 needs 9.47 MB; with H=5120, B=16, k=16, N=128, 14.7 MB).  The first call on
  * a device, with that device current, looks up the array's address; make
  * that first call before any stream capture begins.  Every call on a device
  * shares the array, which keeps the previous call's contents (the round
@@ -219,7 +223,8 @@ PCTREE_API pctree_status pctree_draft_noalloc(const pctree_config* cfg,
  * Starting at the root, repeatedly accept the child whose token equals the
  * target model's token at the current node, until no child matches.
  *   tree           the tokens, parent and n_nodes of a drafted tree (other
- *                  fields unused)
+ *                  fields unused); an n_nodes[r] outside [0, N] is clamped
+ *                  to that range, so the walk never leaves the request's rows
  *   target_tokens  [batch][N] int32: the target's greedy token at each node's
  *                  position, i.e. the token it wants as that node's child
  *   accepted_idx   [batch][B+1] out: node indices of the accepted path from

@@ -187,6 +187,15 @@ def _margin(sorted_vals: Sequence[float], m: int) -> float:
     return a - b
 
 
+def _order_margin(sorted_vals: Sequence[float], m: int) -> float:
+    """Smallest of the cut gap and the gaps between consecutive kept values:
+    how far this decision is from one whose kept set or order differs."""
+    gaps = [_margin(sorted_vals, m)]
+    top = list(sorted_vals[:m])
+    gaps += [0.0 if a == b else a - b for a, b in zip(top, top[1:])]
+    return min(gaps)
+
+
 def _check_choice(name: str, chosen: Sequence, candidates: Sequence,
                   val: Dict, delta: float, ordered: bool) -> None:
     """Raise unless ``chosen`` is a valid top-|chosen| of ``candidates``
@@ -293,6 +302,10 @@ class Round:
     n_ambiguous: int          # adopted hinted choices that differ from ours
     margins: Dict[str, float]  # smallest own margin per decision kind
     markov_calls: List[int]   # batch size b_d of each Markov call
+    # per adopted differing choice: (decision kind, our own margin there --
+    # the smaller of the cut gap and the gaps between consecutive kept values
+    # for ordered decisions, the cut gap for the unordered global selection)
+    adopted: List[Tuple[str, float]] = dataclasses.field(default_factory=list)
 
 
 def _check_logits(L: np.ndarray) -> None:
@@ -341,6 +354,7 @@ def draft(L: np.ndarray, E_in: np.ndarray, W_out: np.ndarray, root: int,
     chain = root                                      # greedy chain (shared)
     margins = {"children": math.inf, "frontier": math.inf, "global": math.inf}
     n_amb = 0
+    adopted: List[Tuple[str, float]] = []
     calls = []
     for d in range(B):                                # stage d builds level d+1
         if mode == "shared":
@@ -375,6 +389,7 @@ def draft(L: np.ndarray, E_in: np.ndarray, W_out: np.ndarray, root: int,
                     _check_choice(f"children of {pool.path[pid]}", theirs,
                                   cands, zval, delta, ordered=True)
                     n_amb += 1
+                    adopted.append(("children", _order_margin(zs, k)))
                     kids = list(theirs)
             if slot == 0:
                 first_kids = list(kids)
@@ -406,6 +421,7 @@ def draft(L: np.ndarray, E_in: np.ndarray, W_out: np.ndarray, root: int,
                                   {i: pool.s[i] for i in layer}, delta,
                                   ordered=True)
                     n_amb += 1
+                    adopted.append(("frontier", _order_margin(ranked, k)))
                     frontier = theirs
     n_pool = len(pool.token)
     mine = global_topn(pool.s, pool.depth, N)
@@ -422,9 +438,10 @@ def draft(L: np.ndarray, E_in: np.ndarray, W_out: np.ndarray, root: int,
                           {i: pool.s[i] for i in range(n_pool)}, delta,
                           ordered=False)
             n_amb += 1
+            adopted.append(("global", margins["global"]))
             chosen = theirs
     packed, tree = pack(pool, chosen, N, B, pos_offset)
-    return Round(pool, packed, tree, n_amb, margins, calls)
+    return Round(pool, packed, tree, n_amb, margins, calls, adopted)
 
 
 # ----------------------------------------------------------------------------

@@ -258,6 +258,7 @@ pctree_status draft_fused(const pctree_config& c, const Layout& lay,
                                stream));
   if (st != PCTREE_OK) return st;
   prof_record(0, stream);
+  NvtxRange range("round_fused (all stages)");
   const cudaError_t e = launch_round_fused(&tmap_w, &tmap_x, a, grid, stream);
   prof_record(1, stream);
   if (e != cudaSuccess) return PCTREE_ERR_CUDA;
@@ -305,6 +306,7 @@ pctree_status pctree_draft(const pctree_config* cfg, const float* base_logits,
                            const int32_t* root_token, const pctree_tree* out,
                            void* workspace, size_t workspace_bytes,
                            void* stream_ptr) {
+  NvtxRange range("pctree_draft");
   pctree_status st = check_config(cfg);
   if (st != PCTREE_OK) return st;
   const pctree_config c = *cfg;
@@ -351,7 +353,12 @@ pctree_status pctree_draft(const pctree_config* cfg, const float* base_logits,
   if (st != PCTREE_OK) return st;
   float* Z = reinterpret_cast<float*>(ws + lay.off_z);
   const long long l_req_stride = static_cast<long long>(c.B) * c.V;
+  static const char* const kStageNames[] = {
+      "stage 0",  "stage 1",  "stage 2",  "stage 3",  "stage 4",  "stage 5",
+      "stage 6",  "stage 7",  "stage 8",  "stage 9",  "stage 10", "stage 11",
+      "stage 12", "stage 13", "stage 14", "stage 15", "stage 16+"};
   for (int d = 0; d < c.B; ++d) {
+    NvtxRange stage_range(kStageNames[d < 16 ? d : 16]);
     const int rpq = rows_per_request(c, d);  // b_d (Sec. 4.1), or 1
     const int rows = c.batch * rpq;
     const float* L_d = base_logits + static_cast<size_t>(d) * c.V;
@@ -381,6 +388,7 @@ pctree_status pctree_accept(const pctree_config* cfg, const pctree_tree* tree,
                             const int32_t* target_tokens,
                             int32_t* accepted_idx, int32_t* accepted_len,
                             int32_t* bonus_token, void* stream_ptr) {
+  NvtxRange range("pctree_accept");
   pctree_status st = check_config(cfg);
   if (st != PCTREE_OK) return st;
   if (tree == nullptr || tree->n_nodes == nullptr || tree->tokens == nullptr ||

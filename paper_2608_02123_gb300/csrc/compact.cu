@@ -142,6 +142,7 @@ pctree_status pctree_compact(const pctree_compact_layout* layout,
                              const int32_t* prefix_len, void* cache,
                              const void* hidden_in, void* hidden_out,
                              int32_t* status, void* stream) {
+  pct::NvtxRange range("pctree_compact");
   using pct::aligned16;
   if (layout == nullptr || accepted_idx == nullptr || accepted_len == nullptr ||
       prefix_len == nullptr)

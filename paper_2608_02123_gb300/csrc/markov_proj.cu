@@ -282,13 +282,11 @@ cudaError_t launch_tc(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
                       int ldz, int V, int H, int rows, int rows_per_req,
                       int num_sms, int32_t* status, cudaStream_t stream) {
   using C = TcCfg<BN>;
-  static bool attr_done = false;  // the attribute is per function, per process
-  if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(markov_tc_kernel<BN>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(C::kSmemBytes));
+  static SmemLimit limit;
+  {
+    cudaError_t e = limit.ensure(reinterpret_cast<const void*>(markov_tc_kernel<BN>),
+                                 C::kSmemBytes);
     if (e != cudaSuccess) return e;
-    attr_done = true;
   }
   const int n_tiles = (V + kBM - 1) / kBM;
   const int grid = n_tiles < num_sms ? n_tiles : num_sms;

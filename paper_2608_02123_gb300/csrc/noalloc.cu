@@ -27,13 +27,13 @@
 namespace pct {
 namespace {
 
-// 16 MiB: enough for batch-1 Qwen3-shaped rounds (a B=16, k=8, N=64 round
-// over V=151936 needs about 5 MB); larger rounds are rejected.
+// 16 MiB: enough for batch-1 Qwen3-shaped rounds (pctree_workspace_bytes is
+// 9.47 MB for V=151936, H=2560, B=16, k=8, N=64 and 14.7 MB for V=151936,
+// H=5120, B=16, k=16, N=128); larger rounds are rejected.
 constexpr size_t kStaticScratchBytes = size_t(16) << 20;
 
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
-constexpr int kMaxDevices = 64;
 std::mutex g_scratch_mu;
 void* g_scratch_ptr[kMaxDevices] = {nullptr};
 

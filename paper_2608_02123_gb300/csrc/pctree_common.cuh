@@ -7,6 +7,8 @@
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_runtime.h>
+#include <mutex>
+#include <nvtx3/nvToolsExt.h>
 
 #include "pctree.h"
 
@@ -243,6 +245,44 @@ __device__ __forceinline__ void set_status(int32_t* status, int code) {
 // ---------------------------------------------------------------------------
 // launchers (return cudaGetLastError() of the launch)
 // ---------------------------------------------------------------------------
+
+constexpr int kMaxDevices = 64;
+
+// NVTX range over a host scope (the enqueue of a call or of one stage):
+// profilers that attach to NVTX (Nsight Systems, Nsight Compute's range
+// filters) attribute the kernels launched inside it to the range.  Without
+// an attached tool a push/pop costs a few nanoseconds.
+class NvtxRange {
+ public:
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+
+// Raises one kernel's dynamic shared-memory limit on the current device,
+// once per device: the attribute belongs to the function on one device, so a
+// process that drafts on several GPUs sets it on each.  Thread-safe; a call
+// that fails is retried by the next launch.
+class SmemLimit {
+ public:
+  cudaError_t ensure(const void* fn, size_t bytes) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(mu_);
+    if (done_[dev]) return cudaSuccess;
+    e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(bytes));
+    if (e == cudaSuccess) done_[dev] = true;
+    return e;
+  }
+
+ private:
+  std::mutex mu_;
+  bool done_[kMaxDevices] = {};
+};
 
 // Z[row][v] = L[req(row)][v] + sum_h W_out[v][h] X[row][h] for rows
 // [0, rows), req(row) = row / rows_per_req.  `L` points at depth d of

@@ -749,14 +749,10 @@ round_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
 template <int R>
 cudaError_t launch_r(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
                      const FusedArgs& args, int grid, cudaStream_t stream) {
-  static bool attr_done = false;
-  if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(round_fused_kernel<R>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem_bytes<R>()));
-    if (e != cudaSuccess) return e;
-    attr_done = true;
-  }
+  static SmemLimit limit;
+  cudaError_t e = limit.ensure(reinterpret_cast<const void*>(round_fused_kernel<R>),
+                               smem_bytes<R>());
+  if (e != cudaSuccess) return e;
   CUtensorMap w = *tmap_w, x = *tmap_x;
   FusedArgs a = args;
   void* params[] = {&w, &x, &a};

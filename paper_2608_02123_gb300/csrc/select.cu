@@ -630,7 +630,9 @@ __global__ void accept_kernel(int B, int N, const int32_t* __restrict__ n_nodes,
   const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (r >= batch) return;
   const int lane = threadIdx.x & 31;
-  const int n = n_nodes[r];
+  // a caller-built tree may claim more nodes than its rows hold: walk at most
+  // the N rows of the request
+  const int n = min(max(n_nodes[r], 0), N);
   const int32_t* tk = tokens + static_cast<size_t>(r) * N;
   const int32_t* pa = parent + static_cast<size_t>(r) * N;
   const int32_t* tg = target + static_cast<size_t>(r) * N;
@@ -719,12 +721,10 @@ cudaError_t launch_pack(const pctree_config& c, const Layout& lay,
                         unsigned char* ws, const pctree_tree& out,
                         cudaStream_t stream) {
   const size_t smem = static_cast<size_t>(lay.P) * sizeof(unsigned long long);
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaFuncSetAttribute(pack_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         PCTREE_MAX_POOL * static_cast<int>(sizeof(unsigned long long)));
-    attr_set = true;
-  }
+  static SmemLimit limit;
+  const cudaError_t e = limit.ensure(reinterpret_cast<const void*>(pack_kernel),
+                                     PCTREE_MAX_POOL * sizeof(unsigned long long));
+  if (e != cudaSuccess) return e;
   pack_kernel<<<c.batch, kPackThreads, smem, stream>>>(
       c.B, c.k, c.N, lay.P, c.pos_offset,
       reinterpret_cast<const int32_t*>(ws + lay.off_pool_tok),

@@ -960,6 +960,7 @@ pctree_status pctree_tree_attention(const pctree_attn_config* cfg, const void* q
                                     void* out, void* workspace,
                                     size_t workspace_bytes, int32_t* status,
                                     void* stream_ptr) {
+  pct::NvtxRange range("pctree_tree_attention");
   using namespace pct;
   pctree_status st = attn_check(cfg);
   if (st != PCTREE_OK) return st;
@@ -1025,17 +1026,12 @@ pctree_status pctree_tree_attention(const pctree_attn_config* cfg, const void* q
     a.part_ml = reinterpret_cast<float2*>(ws + w.part_ml);
   }
   // a dummy status word is not needed: kernels test for NULL
-  static bool attr_set[64] = {false};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return PCTREE_ERR_CUDA;
-  if (!attr_set[dev]) {
-    if (cudaFuncSetAttribute(tree_attn_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(attn_smem<1>())) != cudaSuccess ||
-        cudaFuncSetAttribute(tree_attn_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(attn_smem<2>())) != cudaSuccess)
-      return PCTREE_ERR_CUDA;
-    attr_set[dev] = true;
-  }
+  static SmemLimit limit1, limit2;
+  if (limit1.ensure(reinterpret_cast<const void*>(tree_attn_kernel<1>), attn_smem<1>()) !=
+          cudaSuccess ||
+      limit2.ensure(reinterpret_cast<const void*>(tree_attn_kernel<2>), attn_smem<2>()) !=
+          cudaSuccess)
+    return PCTREE_ERR_CUDA;
   // persistent: one CTA per SM walks its share of the items
   const dim3 grid(static_cast<unsigned>(a.items < num_sms ? a.items : num_sms));
   if (g.tpc == 2)

@@ -13,6 +13,14 @@ from workloads import RoundInputs, target_for_tree
 
 LOGP_TOL = 1e-4      # absolute, on cumulative log-probs
 
+# Largest own margin at which the CUDA path may legitimately decide otherwise
+# than the float64 oracle.  Children are ranked on float32 stage logits
+# z = L + bias (rounding of the sum and of the float32 dot product: a few
+# 1e-6 for |z| up to ~100); frontier and budget on float32 scores whose error
+# grows over up to 16 stages to at most ~5e-5 (twice that for a pair).  A
+# near-tie adopted at a wider margin is a regression, not float32 noise.
+FLOAT32_DECISION_BOUND = {"children": 5e-5, "frontier": 1e-4, "global": 1e-4}
+
 
 def device_inputs(inp: RoundInputs, device="cuda"):
     wl = inp.wl
@@ -27,16 +35,87 @@ def device_inputs(inp: RoundInputs, device="cuda"):
     return L, E, W, root
 
 
+# ---------------------------------------------------------------------------
+# canary padding: every output tensor and the workspace sit inside a larger
+# buffer whose margins hold a fixed bit pattern; a write past either end of
+# any of them changes the pattern
+# ---------------------------------------------------------------------------
+
+CANARY_PAD = 512          # elements before and after each tensor
+_CANARY = {torch.int32: 0x5A5A5A5A, torch.float32: 0x7FA5A5A5,
+           torch.uint8: 0xA5}
+
+
+class Canaries:
+    def __init__(self, device="cuda"):
+        self.device = device
+        self.bufs = []           # (name, padded buffer, inner element count)
+
+    def tensor(self, name, shape, dtype):
+        n = int(np.prod(shape))
+        bits = torch.int32 if dtype == torch.float32 else dtype
+        buf = torch.full((n + 2 * CANARY_PAD,), _CANARY[dtype], dtype=bits,
+                         device=self.device)
+        if dtype == torch.float32:
+            buf = buf.view(torch.float32)
+        self.bufs.append((name, buf, n))
+        return buf[CANARY_PAD:CANARY_PAD + n].view(*shape)
+
+    def check(self):
+        for name, buf, n in self.bufs:
+            raw = buf.view(torch.int32) if buf.dtype == torch.float32 else buf
+            want = _CANARY[buf.dtype]
+            head = raw[:CANARY_PAD].cpu().numpy()
+            tail = raw[CANARY_PAD + n:].cpu().numpy()
+            if buf.dtype == torch.uint8:
+                ok = (head == want).all() and (tail == want).all()
+            else:
+                ok = ((head.view(np.uint32) == np.uint32(want)).all() and
+                      (tail.view(np.uint32) == np.uint32(want)).all())
+            assert ok, f"canary around {name} overwritten"
+
+
+def canary_drafter(P, cfg, with_pool: bool):
+    """A Drafter whose tree, accept outputs and workspace are canary-padded."""
+    dr = P.Drafter(cfg, with_pool=with_pool)
+    cz = Canaries()
+    R, N, B = cfg.batch, cfg.N, cfg.B
+    Pn = P.pctree_pool_capacity(cfg)
+    i32, f32, u8 = torch.int32, torch.float32, torch.uint8
+    dr.tree = P.Tree(
+        n_nodes=cz.tensor("n_nodes", (R,), i32),
+        tokens=cz.tensor("tokens", (R, N), i32),
+        parent=cz.tensor("parent", (R, N), i32),
+        depth=cz.tensor("depth", (R, N), i32),
+        logp=cz.tensor("logp", (R, N), f32),
+        position_ids=cz.tensor("position_ids", (R, N), i32),
+        mask=cz.tensor("mask", (R, N, N), u8),
+        retrieve=cz.tensor("retrieve", (R, N, B + 1), i32),
+        n_leaves=cz.tensor("n_leaves", (R,), i32),
+        status=cz.tensor("status", (1,), i32),
+        pool_token=cz.tensor("pool_token", (R, Pn), i32) if with_pool else None,
+        pool_parent=cz.tensor("pool_parent", (R, Pn), i32) if with_pool else None,
+        pool_logp=cz.tensor("pool_logp", (R, Pn), f32) if with_pool else None)
+    # the workspace keeps its 256-byte alignment: the pad is 512 bytes
+    nbytes = dr.workspace.numel()
+    dr.workspace = cz.tensor("workspace", (nbytes,), u8)
+    dr.accepted_idx = cz.tensor("accepted_idx", (R, B + 1), i32)
+    dr.accepted_len = cz.tensor("accepted_len", (R,), i32)
+    dr.bonus = cz.tensor("bonus", (R,), i32)
+    return dr, cz
+
+
 def run_gpu(inp: RoundInputs, with_pool=True, accept=True,
             path: int = 0) -> Dict[str, np.ndarray]:
     """One round through the C ABI; ``path`` 0 = automatic (fused round
-    kernel where it applies), 1 = per-stage kernels."""
+    kernel where it applies), 1 = per-stage kernels.  Every output tensor
+    and the workspace are canary-padded and checked afterwards."""
     from paper_2608_02123_gb300 import pctree as P
     wl = inp.wl
     cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, inp.L.shape[0],
                         wl.pos_offset, wl.weight_dtype, wl.mode)
     L, E, W, root = device_inputs(inp)
-    dr = P.Drafter(cfg, with_pool=with_pool)
+    dr, canaries = canary_drafter(P, cfg, with_pool)
     P.pctree_set_path(path)
     try:
         tree = dr.draft(L, E, W, root)
@@ -52,6 +131,7 @@ def run_gpu(inp: RoundInputs, with_pool=True, accept=True,
         host["accepted_idx"] = acc.cpu().numpy()
         host["accepted_len"] = length.cpu().numpy()
         host["bonus"] = bonus.cpu().numpy()
+    canaries.check()
     return host
 
 
@@ -76,6 +156,15 @@ class Report:
     max_logp_err: float = 0.0
     requests: int = 0
     min_margin: float = np.inf
+    # smallest own margin per decision kind over the compared requests
+    margins: Dict[str, float] = dataclasses.field(default_factory=dict)
+    # (request, kind, own margin) of every adopted near-tie decision
+    adopted: List[tuple] = dataclasses.field(default_factory=list)
+
+    def summary(self) -> str:
+        m = " ".join(f"{k}={v:.1e}" for k, v in sorted(self.margins.items()))
+        return (f"requests={self.requests} ambiguous={self.ambiguous} "
+                f"max|dlogp|={self.max_logp_err:.2e} min margins: {m}")
 
 
 def _close(got: np.ndarray, want: np.ndarray, r: int) -> float:
@@ -114,6 +203,14 @@ def compare(inp: RoundInputs, host: Dict[str, np.ndarray],
         rep.requests += 1
         rep.ambiguous += rnd.n_ambiguous
         rep.min_margin = min(rep.min_margin, *rnd.margins.values())
+        for kind, m in rnd.margins.items():
+            rep.margins[kind] = min(rep.margins.get(kind, np.inf), m)
+        for kind, m in rnd.adopted:
+            rep.adopted.append((r, kind, m))
+            assert m <= FLOAT32_DECISION_BOUND[kind], (
+                f"request {r}: the CUDA path decided a {kind} choice "
+                f"otherwise than the oracle across a margin of {m:.2e}, "
+                f"wider than float32 noise ({FLOAT32_DECISION_BOUND[kind]:.0e})")
         assert int(host["n_nodes"][r]) == t.n_nodes
         for name in ("tokens", "parent", "depth", "position_ids"):
             np.testing.assert_array_equal(host[name][r], getattr(t, name),

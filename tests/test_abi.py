@@ -130,3 +130,13 @@ def test_stall_hook_argument_checks(P):
     assert lib.pctree_debug_stall_stage(1, 10) == -1
     assert lib.pctree_debug_stall_stage(1, 2 * 10**10) == -1
     assert lib.pctree_debug_stall_stage(-1, 10**9) == 0      # the default
+
+
+def test_batch1_qwen3_rounds_fit_the_noalloc_array(P):
+    """pctree_draft_noalloc serves batch-1 Qwen3-shaped rounds from its fixed
+    16 MiB array: a layout change that outgrows it fails here."""
+    limit = 16 << 20
+    for V, H, B, k, N in ((151936, 2560, 16, 8, 64), (151936, 2560, 7, 8, 32),
+                          (151936, 4096, 7, 8, 64), (151936, 5120, 16, 16, 128)):
+        ws = P.pctree_workspace_bytes(P.make_config(V, H, B, k, N, 1))
+        assert 0 < ws <= limit, (V, H, B, k, N, ws)

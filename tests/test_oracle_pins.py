@@ -137,6 +137,12 @@ def test_replay_adopts_only_near_ties():
     rep = O.draft(L2, E, W, root, B, k, N, hint=alt_hint)
     assert rep.n_ambiguous >= 1
     assert b in rep.pool.token[1:1 + k] and a not in rep.pool.token[1:1 + k]
+    # each adopted choice records our own margin there: the root's children
+    # were decided across a 1e-6 gap
+    assert len(rep.adopted) == rep.n_ambiguous
+    kinds = dict(rep.adopted)
+    assert kinds["children"] == pytest.approx(1e-6, rel=1e-3)
+    assert all(m <= 1e-6 * 1.001 for _, m in rep.adopted)
     # the same swap with a clear gap is refused
     L4 = L.copy()
     L4[0, b] = L4[0, a] - 0.5
