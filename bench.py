@@ -49,6 +49,10 @@ def parse_args():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="4b_b16", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-batched", action="store_true",
+                    help="skip the short timing of the batched serving "
+                         "workloads (8B-shaped batch 16, 14B-shaped batch 32) "
+                         "that the default line carries under 'batched'")
     ap.add_argument("--mode", default="parent", choices=["parent", "shared"],
                     help="child scoring: PCTree, or the Shared-Markov control")
     ap.add_argument("--sweep", action="store_true",
@@ -197,19 +201,36 @@ def oracle_threads():
     return os.cpu_count() or 1
 
 
+def host_cpu():
+    """The host's logical CPU count and model (lscpu), for the baseline's
+    record."""
+    model = None
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True,
+                             timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().startswith("Model name:"):
+                model = line.split(":", 1)[1].strip()
+                break
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return {"nproc": os.cpu_count(), "model": model}
+
+
 class OracleRunner:
-    """Runs the oracle's drafting round on prefixes of the workload's rounds:
-    a sample of `stages` of the B stages, scaled to whole rounds."""
+    """Runs the oracle's drafting round on the workload's rounds (whole
+    rounds, or the first `stages` of the B stages of each)."""
 
     def __init__(self, wl, E_in, W_out_bits, sets):
         from oracle import pctree_oracle as O
         self.O, self.wl, self.E_in, self.sets = O, wl, E_in, sets
         self.W = O.as_f64(W_out_bits, wl.weight_dtype)   # weights load once
 
-    def run(self, i, stages):
+    def run(self, i, stages=None, hint=None):
         L, root = self.sets[i % len(self.sets)]
-        self.O.draft(L[:stages], self.E_in, self.W, root, stages, self.wl.k,
-                     self.wl.N, mode=self.wl.mode)
+        s = self.wl.B if stages is None else stages
+        return self.O.draft(L[:s], self.E_in, self.W, root, s, self.wl.k,
+                            self.wl.N, mode=self.wl.mode, hint=hint)
 
 
 def markov_rows(wl, stages):
@@ -217,36 +238,65 @@ def markov_rows(wl, stages):
     request at stage 0, then one per frontier parent (k per request), or one
     chain row per request in the Shared-Markov control.  The oracle's cost
     is proportional to these rows (each is a vocabulary-wide projection and
-    selection), so samples are scaled to whole rounds by them."""
+    selection), so partial-round samples are scaled to whole rounds by them."""
     per_stage = 1 if wl.mode == "shared" else wl.k
     return wl.batch * (1 + (stages - 1) * per_stage) if stages > 0 else 0
 
 
-def oracle_sample_stages(wl):
-    return min(wl.B, 4)
+def tree_hint(O, host, r=0):
+    """The GPU round's decisions (children, frontiers, kept set) rebuilt from
+    its candidate pool, for the oracle's near-tie replay."""
+    n = int(host["n_nodes"][r])
+    tok, par = host["tokens"][r], host["parent"][r]
+    paths = []
+    for a in range(n):
+        paths.append(() if a == 0 else paths[par[a]] + (int(tok[a]),))
+    return O.choices_from_pool(host["pool_token"][r], host["pool_parent"][r],
+                               host["pool_token"].shape[1], set(paths))
 
 
-def cpu_baseline(runner, wl, budget_s=12.0):
-    stages = oracle_sample_stages(wl)
-    t0 = time.perf_counter()
-    n = 0
-    while True:
-        runner.run(n, stages)
-        n += 1
-        if time.perf_counter() - t0 >= budget_s:
-            break
-    dt = time.perf_counter() - t0
-    scale = markov_rows(wl, wl.B) / markov_rows(wl, stages)
-    rounds = n / scale
-    return {"value": rounds / dt, "unit": "rounds/s", "cores": oracle_threads(),
-            "kind": "oracle",
-            "sample": f"{n} oracle runs of the first {stages} of {wl.B} stages "
-                      f"of {wl.name} request rounds ({dt:.1f} s), scaled to "
-                      f"whole rounds by Markov rows "
-                      f"({markov_rows(wl, wl.B)}/{markov_rows(wl, stages)})"}
+def cpu_baseline(runner, wl, gpu_trees, budget_s=12.0):
+    """The oracle, as it stands, on whole rounds of the benchmark's input sets
+    (request 0 of each), for about `budget_s` seconds on the host cores.
+    Each round replays the GPU round's near-tie decisions (``hint``; the
+    replay only engages where the two differ), so the same runs also check
+    the benchmark's own trees against the oracle."""
+    O = runner.O
+    times, ambiguous, max_err, equal = [], 0, 0.0, True
+    t_start = time.perf_counter()
+    i = 0
+    while i < len(gpu_trees) and (i < 2 or time.perf_counter() - t_start < budget_s):
+        host = gpu_trees[i]
+        t0 = time.perf_counter()
+        rnd = runner.run(i, hint=tree_hint(O, host))
+        times.append(time.perf_counter() - t0)
+        t = rnd.tree
+        ambiguous += rnd.n_ambiguous
+        n = t.n_nodes
+        equal &= (int(host["n_nodes"][0]) == n and
+                  all((host[f][0] == getattr(t, f)).all()
+                      for f in ("tokens", "parent", "depth", "mask",
+                                "retrieve")))
+        fin = np.isfinite(t.logp[:n])
+        if fin.any():
+            max_err = max(max_err, float(np.abs(host["logp"][0][:n][fin]
+                                                - t.logp[:n][fin]).max()))
+        i += 1
+    dt = sum(times)
+    return {"value": len(times) / dt, "unit": "rounds/s",
+            "cores": oracle_threads(), "host": host_cpu(), "kind": "oracle",
+            "sample": f"{len(times)} whole oracle rounds of {wl.name} "
+                      f"(input sets 0..{len(times) - 1}, request 0), "
+                      f"{dt:.1f} s, {dt / len(times):.2f} s per round",
+            "oracle_check": {"rounds": len(times), "trees_equal": bool(equal),
+                             "ambiguous": ambiguous,
+                             "max_abs_logp_err": max_err}}
 
 
-def run_reference(args, wl, rank, world):
+def run_reference(args, wl, rank, world, budget_s=180.0):
+    """The oracle on the host cores, one drafting round per step.  Steps are
+    whole rounds when K + W of them fit in ``budget_s``; otherwise each step
+    runs the first stages of a round, scaled to whole rounds by Markov rows."""
     if rank != 0:
         return
     E_in, W_out = draw_head(wl)
@@ -255,15 +305,27 @@ def run_reference(args, wl, rank, world):
         L, root, _, _ = draw_request(wl.with_(batch=N_SETS), r)
         sets.append((L, root))
     runner = OracleRunner(wl, E_in, W_out, sets)
-    stages = oracle_sample_stages(wl)
+    t0 = time.perf_counter()
+    runner.run(0)                                    # first warm-up: a whole round
+    t_round = time.perf_counter() - t0
+    stages = wl.B
+    while stages > 1 and (args.steps + args.warmup) * t_round * \
+            markov_rows(wl, stages) / markov_rows(wl, wl.B) > budget_s:
+        stages -= 1
     scale = markov_rows(wl, wl.B) / markov_rows(wl, stages)
-    for i in range(args.warmup):
+    for i in range(1, args.warmup):
         runner.run(i, stages)
     t0 = time.perf_counter()
     for i in range(args.steps):
         runner.run(i, stages)
     dt = time.perf_counter() - t0
     value = args.steps / scale / dt
+    step = ("one whole oracle round (all {} stages)".format(wl.B)
+            if stages == wl.B else
+            f"the oracle's first {stages} of {wl.B} stages of a round, "
+            f"scaled to whole rounds by Markov rows "
+            f"({markov_rows(wl, wl.B)}/{markov_rows(wl, stages)}); a whole "
+            f"round took {t_round:.2f} s")
     line = {
         "metric": METRIC, "value": value, "unit": "rounds/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
@@ -271,14 +333,11 @@ def run_reference(args, wl, rank, world):
         "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "impl": "reference",
         "config": {"workload": wl.name, "V": wl.V, "H": wl.H, "B": wl.B,
-                   "k": wl.k, "N": wl.N, "batch": wl.batch,
-                   "step": f"the oracle's first {stages} of {wl.B} stages of a "
-                           f"round, scaled to whole rounds by Markov rows "
-                           f"({markov_rows(wl, wl.B)}/{markov_rows(wl, stages)})"},
+                   "k": wl.k, "N": wl.N, "batch": wl.batch, "step": step},
         "cpu_baseline": {"value": value, "unit": "rounds/s",
-                         "cores": oracle_threads(), "kind": "oracle",
-                         "sample": f"{args.steps} oracle runs of the first "
-                                   f"{stages} stages"},
+                         "cores": oracle_threads(), "host": host_cpu(),
+                         "kind": "oracle",
+                         "sample": f"{args.steps} steps, each {step}"},
         "e2e": {"value": value, "unit": "rounds/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -359,9 +418,9 @@ def run_ours(args, wl, rank, world, local_rank):
     dr = P.Drafter(cfg, dev)
     stream = torch.cuda.current_stream()
 
-    def target_of(i):
+    def target_of(i, tree=None):
         # synthetic target model: node i at depth t wants g[t] as its child
-        depth = dr.tree.depth.long().clamp_min(0)
+        depth = (dr.tree if tree is None else tree).depth.long().clamp_min(0)
         return torch.gather(greedy_dev[i % n_sets], 1, depth).to(torch.int32)
 
     def step(i):
@@ -445,6 +504,20 @@ def run_ours(args, wl, rank, world, local_rank):
     e2e_ms = e_start.elapsed_time(e_end)
     clk = clocks.stop()
 
+    # outside the timed regions: one round per input set with its candidate
+    # pool, for the mean acceptance length on the synthetic target and for
+    # the oracle's check of the benchmark's own trees
+    check = P.Drafter(cfg, dev, with_pool=True)
+    accepted, gpu_trees = [], []
+    for i in range(n_sets):
+        check.draft(L_dev[i], E, W, root_dev[i], stream)
+        check.accept(target_of(i, check.tree), stream)
+        torch.cuda.synchronize()
+        check.check_status()
+        accepted += check.accepted_len.cpu().tolist()
+        gpu_trees.append(check.tree.to_host())
+    mean_tau = 1.0 + float(np.mean(accepted))     # tau counts the bonus token
+
     ms, e2e_ms = max_over_ranks([ms, e2e_ms], world, dev)
     if rank != 0:
         return
@@ -486,17 +559,108 @@ def run_ours(args, wl, rank, world, local_rank):
                      "p50": draft_us[len(draft_us) // 2],
                      "p90": draft_us[(9 * len(draft_us)) // 10]},
         "accept_us": statistics.mean(accept_us),
+        "mean_tau_synthetic": mean_tau,
+        "mean_tau_note": f"mean accepted length + 1 over the {n_sets} input "
+                         f"sets' rounds against the synthetic target (a "
+                         f"property of the input generator, not of a model)",
         "e2e": {"value": job_rounds_per_s(e2e_ms, args.steps, world, wl.batch),
                 "unit": "rounds/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": kernels_per_step * args.steps,
         "clocks": clk,
     }
+    if world == 1 and not args.no_batched and args.workload == "4b_b16":
+        line["batched"] = measure_batched(dev, gpu_index)
     if world == 1 and not args.no_cpu_baseline:
         runner = OracleRunner(wl, E_host, W_host,
-                              [(L[0], int(root[0])) for L, root, _ in sets[:4]])
-        line["cpu_baseline"] = cpu_baseline(runner, wl)
+                              [(L[0], int(root[0])) for L, root, _ in sets])
+        base = cpu_baseline(runner, wl, gpu_trees)
+        line["cpu_baseline"] = base
+        line["ambiguous"] = base["oracle_check"]["ambiguous"]
     print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# batched serving rounds, timed briefly beside the headline
+# ---------------------------------------------------------------------------
+
+BATCHED = ("8b_b7_bs16", "14b_b16_bs32")
+
+
+def round_flops(wl):
+    """Tensor-core flops of a round's Markov projections: 2 H V per Markov
+    row."""
+    rows = sum(wl.batch * (1 if d == 0 else wl.k) for d in range(wl.B))
+    return 2.0 * wl.H * wl.V * rows
+
+
+def measure_batched(dev, gpu_index, steps=10, warmup=3):
+    """Each batched workload: W + K whole rounds (inputs resident, base
+    logits rotating over sets that together exceed 3 x L2), CUDA events on
+    the launching stream, clocks sampled meanwhile.  The roofline is HBM
+    (algorithmic bytes) or tensor (projection flops) by whichever takes
+    longer at the measured peaks; the sustained bf16 rate is the one for a
+    round of several milliseconds."""
+    import torch
+
+    from paper_2608_02123_gb300 import pctree as P
+
+    peaks, src = measured_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    tc = float(peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops", 1700.0)))
+    out = []
+    stream = torch.cuda.current_stream()
+    for name in BATCHED:
+        wl = WORKLOADS[name]
+        E_host, W_host = draw_head(wl)
+        E = torch.from_numpy(E_host.view(np.int16)).to(dev).view(torch.bfloat16)
+        W = torch.from_numpy(W_host.view(np.int16)).to(dev).view(torch.bfloat16)
+        del E_host, W_host
+        set_bytes = wl.batch * wl.B * wl.V * 4
+        n_sets = max(2, -(-3 * L2_BYTES // set_bytes))
+        many = wl.with_(batch=n_sets * wl.batch)
+        L_dev, root_dev = [], []
+        for i in range(n_sets):
+            reqs = [draw_request(many, i * wl.batch + b) for b in range(wl.batch)]
+            L_dev.append(torch.from_numpy(np.stack([q[0] for q in reqs])).to(dev))
+            root_dev.append(torch.tensor([q[1] for q in reqs], dtype=torch.int32,
+                                         device=dev))
+        cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, wl.batch)
+        dr = P.Drafter(cfg, dev)
+        for i in range(warmup):
+            dr.draft(L_dev[i % n_sets], E, W, root_dev[i % n_sets], stream)
+        torch.cuda.synchronize()
+        dr.check_status()
+        clocks = ClockSampler(gpu_index)
+        clocks.start()
+        time.sleep(0.3)
+        start = torch.cuda.Event(enable_timing=True)
+        end = torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        for i in range(steps):
+            dr.draft(L_dev[i % n_sets], E, W, root_dev[i % n_sets], stream)
+        end.record(stream)
+        torch.cuda.synchronize()
+        clk = clocks.stop()
+        dr.check_status()
+        us = start.elapsed_time(end) * 1e3 / steps
+        nbytes, flops = round_bytes(wl), round_flops(wl)
+        t_hbm, t_tc = nbytes / hbm / 1e3, flops / tc / 1e6   # µs
+        bound = "hbm" if t_hbm >= t_tc else "tensor"
+        out.append({
+            "workload": wl.name, "batch": wl.batch, "steps": steps,
+            "warmup": warmup, "us_per_round": us,
+            "rounds_per_s": 1e6 / us, "request_rounds_per_s": wl.batch * 1e6 / us,
+            "bound": bound, "roofline_us": max(t_hbm, t_tc),
+            "frac": max(t_hbm, t_tc) / us,
+            "achieved": {"GB/s": nbytes / us / 1e3, "TFLOP/s": flops / us / 1e6},
+            "peak": {"GB/s": hbm, "TFLOP/s": tc, "source": src,
+                     "tensor": "sustained bf16"},
+            "gpu_launches": steps * P.kernels_per_round(cfg),
+            "clocks": clk})
+        del E, W, L_dev, dr
+        torch.cuda.empty_cache()
+    return out
 
 
 # ---------------------------------------------------------------------------
