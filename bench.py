@@ -548,7 +548,7 @@ def run_ours(args, wl, rank, world, local_rank):
         "round_hbm_fraction": (bytes_round / (us_round * 1e-6) / 1e9) / peak,
         "roofline": {"bound": "hbm",
                      "kernel": ("round_fused_kernel" if fused
-                                else "markov_tc_kernel"),
+                                else "markov_fused_kernel"),
                      "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak if achieved else None,
                      "peak_source": peak_kind,

@@ -153,8 +153,11 @@ PCTREE_API int32_t pctree_pool_capacity(const pctree_config* cfg);
 
 /* Device workspace bytes pctree_draft needs for `cfg` (256-byte aligned
  * start required); 0 for a bad config.  The workspace holds the per-stage
- * Markov rows, the stage logits, the per-chunk softmax/top-k partials, the
- * candidate pool and the frontier; its contents are scratch between calls. */
+ * Markov rows, the softmax/top-k partials of each stage, the candidate pool
+ * and the frontier (and, for F32 heads only, the stage logits); its contents
+ * are scratch between calls.  bf16 heads never write stage logits to memory:
+ * 4.74 MB for V=151936, H=2560, B=16, k=8, N=64, batch 1; 25.6 MB for
+ * V=151936, H=5120, B=16, k=16, N=128, batch 32. */
 PCTREE_API size_t pctree_workspace_bytes(const pctree_config* cfg);
 
 /*
@@ -201,7 +204,7 @@ PCTREE_API pctree_status pctree_draft(const pctree_config* cfg, const float* bas
  * that loads it until the process exits; a round whose
  * pctree_workspace_bytes exceeds 16 MiB returns PCTREE_ERR_WORKSPACE before
  * any work (batch-1 Qwen3-shaped rounds fit: V=151936 with H=2560, B=16,
- * k=8, N=64 needs 9.47 MB; with H=5120, B=16, k=16, N=128, 14.7 MB).  The first call on
+ * k=8, N=64 needs 4.74 MB; with H=5120, B=16, k=16, N=128, 5.54 MB).  The first call on
  * a device, with that device current, looks up the array's address; make
  * that first call before any stream capture begins.  Every call on a device
  * shares the array, which keeps the previous call's contents (the round

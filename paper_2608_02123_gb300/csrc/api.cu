@@ -50,6 +50,9 @@ Layout make_layout(const pctree_config& c) {
          : l.rows_pad <= 128 ? 128 : 256;
   l.ldz = static_cast<int>(align_up(c.V, 64));
   l.n_chunks = (c.V + kChunk - 1) / kChunk;
+  // bf16 heads: one partial per (row, projection CTA); f32 heads: one per
+  // vocabulary chunk of the stage logits Z
+  l.part_slots = c.weight_dtype == PCTREE_BF16 ? kFusedMaxGrid : l.n_chunks;
   l.P = 1 + c.k + (c.B - 1) * c.k * c.k;
   l.x_elem = c.weight_dtype == PCTREE_BF16 ? 2 : 4;
   size_t off = 0;
@@ -60,11 +63,12 @@ Layout make_layout(const pctree_config& c) {
   };
   const size_t rows = static_cast<size_t>(l.rows_max);
   l.off_x = take(static_cast<size_t>(l.rows_pad) * c.H * l.x_elem);
-  l.off_z = take(rows * l.ldz * sizeof(float));
-  l.off_pm = take(rows * l.n_chunks * sizeof(float));
-  l.off_ps = take(rows * l.n_chunks * sizeof(float));
-  l.off_pz = take(rows * l.n_chunks * c.k * sizeof(float));
-  l.off_pt = take(rows * l.n_chunks * c.k * sizeof(int32_t));
+  // stage logits Z: only the f32 path writes them
+  l.off_z = take(c.weight_dtype == PCTREE_BF16 ? 0 : rows * l.ldz * sizeof(float));
+  l.off_pm = take(rows * l.part_slots * sizeof(float));
+  l.off_ps = take(rows * l.part_slots * sizeof(float));
+  l.off_pz = take(rows * l.part_slots * c.k * sizeof(float));
+  l.off_pt = take(rows * l.part_slots * c.k * sizeof(int32_t));
   l.off_pool_tok = take(static_cast<size_t>(c.batch) * l.P * sizeof(int32_t));
   l.off_pool_par = take(static_cast<size_t>(c.batch) * l.P * sizeof(int32_t));
   l.off_pool_s = take(static_cast<size_t>(c.batch) * l.P * sizeof(float2));
@@ -364,21 +368,29 @@ pctree_status pctree_draft(const pctree_config* cfg, const float* base_logits,
     const float* L_d = base_logits + static_cast<size_t>(d) * c.V;
     prof_record(0, stream);
     cudaError_t e;
+    int n_parts;
     if (c.weight_dtype == PCTREE_BF16) {
-      e = launch_markov_bf16(&tmap_w, &tmap_x, L_d, l_req_stride, Z, lay.ldz,
-                             c.V, c.H, rows, rpq, lay.bn, num_sms, out->status,
-                             stream);
+      // projection, normaliser and top-k partials in one pass over W_out
+      n_parts = fused_proj_parts(c.V, num_sms);
+      e = launch_markov_fused(&tmap_w, &tmap_x, L_d, l_req_stride, c.V, c.H, c.k,
+                              rows, rpq, lay.bn, num_sms,
+                              reinterpret_cast<float*>(ws + lay.off_pm),
+                              reinterpret_cast<float*>(ws + lay.off_ps),
+                              reinterpret_cast<float*>(ws + lay.off_pz),
+                              reinterpret_cast<int32_t*>(ws + lay.off_pt),
+                              out->status, stream);
+      prof_record(1, stream);
     } else {
+      n_parts = lay.n_chunks;
       e = launch_markov_f32(static_cast<const float*>(head_out),
                             reinterpret_cast<const float*>(ws + lay.off_x), L_d,
                             l_req_stride, Z, lay.ldz, c.V, c.H, rows, rpq,
                             out->status, stream);
+      prof_record(1, stream);
+      if (e == cudaSuccess) e = launch_partials(lay, c.k, c.V, rows, ws, out->status, stream);
     }
-    prof_record(1, stream);
     if (e != cudaSuccess) return PCTREE_ERR_CUDA;
-    st = cuda_status(launch_partials(lay, c.k, c.V, rows, ws, out->status, stream));
-    if (st != PCTREE_OK) return st;
-    st = cuda_status(launch_merge(c, lay, d, head_emb, ws, out->status, stream));
+    st = cuda_status(launch_merge(c, lay, d, n_parts, head_emb, ws, out->status, stream));
     if (st != PCTREE_OK) return st;
   }
   return cuda_status(launch_pack(c, lay, ws, *out, stream));

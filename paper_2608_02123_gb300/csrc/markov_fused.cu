@@ -1,0 +1,481 @@
+// Markov projection of one PCTree stage with the stage's log-softmax
+// normaliser and per-parent top-k folded into the epilogue (Eqs. 2-3), for
+// bf16 heads and any number of Markov rows (the batched serving rounds):
+//
+//   z[row][v] = L_d[req(row)][v] + sum_h W_out[v][h] * X[row][h]
+//
+// is formed tile by tile in tensor memory and never written to HBM.  For
+// every parent row the CTA keeps, over the vocabulary tiles it owns, a
+// running (max, sum of exp) and a sorted top-k list of (z, token); at the end
+// of the pass it publishes them as one partial per (row, CTA), which the
+// stage's merge combines into the row's normaliser and children.
+//
+// Layout of the work: persistent CTAs (one per SM) take vocabulary tiles of
+// 128 rows round-robin.  Warp 0 streams W_out tiles (MMA A, 128 x 64 bf16
+// boxes, L2 evict_first) and the pass's parent rows (MMA B, NC x 64) with TMA
+// into a shared-memory ring; warp 1 issues tcgen05.mma (M = 128 vocabulary
+// rows, N = NC parent rows, f32 accumulators in TMEM, two buffers so the
+// epilogue of one tile overlaps the MMAs of the next).  Warps 2..9 are the
+// epilogue.  Per 64-column chunk of the accumulator:
+//   A  each warp reads 32 TMEM lanes (its quadrant) x 32 columns with
+//      tcgen05.ld and writes them transposed into shared memory, so that
+//      one parent row's 128 logits of the tile lie contiguous;
+//   B  each warp takes 8 of the chunk's parent rows: per row, a float4 of
+//      logits per lane plus the base logits, a warp (max, sum-exp) folded
+//      into the row's running pair, and the row's top-k list updated with
+//      the logits that beat its current k-th entry (most tiles have none).
+// A CTA's first tile seeds each row's list with a sort of the lanes' best
+// logits.  Rows are always handled by the same warp in the same tile order,
+// so results are deterministic.
+#include <cuda_runtime.h>
+
+#include "pctree_common.cuh"
+#include "sm103_ptx.cuh"
+
+namespace pct {
+namespace {
+
+constexpr int kBM = 128;          // vocabulary rows per tile (MMA M)
+constexpr int kBK = 64;           // K elements per ring slot (128 B of bf16)
+constexpr int kUmmaK = 16;        // K per tcgen05.mma kind::f16
+constexpr int kEpiWarps = 8;
+constexpr int kEpiThreads = 32 * kEpiWarps;
+constexpr int kThreads = 64 + kEpiThreads;
+constexpr int kCC = 64;           // accumulator columns per transpose chunk
+constexpr int kRowsPerWarp = kCC / kEpiWarps;
+constexpr int kMaxStages = 8;
+constexpr int kSmemLimit = 227 * 1024;
+constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per bounded wait
+constexpr float kNegInf = -INFINITY;
+
+// Shared-memory plan of one instance (NC columns, k up to PCTREE_MAX_K).
+template <int NC>
+struct FusedProj {
+  static constexpr int kABytes = kBM * kBK * 2;          // 16 KB
+  static constexpr int kBBytes = NC * kBK * 2;           // 2..32 KB
+  static constexpr int kStageBytes = kABytes + kBBytes;  // multiple of 1024
+  static constexpr int kTmemCols = 2 * NC < 32 ? 32 : 2 * NC;
+  static constexpr size_t kZBytes = static_cast<size_t>(kCC) * kBM * sizeof(float);
+  // per-row running state: max, sum, k-th entry (value, token)
+  static constexpr size_t kRowBytes = static_cast<size_t>(NC) * 16;
+  static constexpr size_t kBarBytes = 256;
+  static size_t list_bytes(int k) { return static_cast<size_t>(NC) * k * 8; }
+  static size_t fixed_bytes(int k) {
+    return 1024 /*alignment slack*/ + kZBytes + kRowBytes + list_bytes(k) + kBarBytes;
+  }
+  static int stages(int k) {
+    const long long room = kSmemLimit - static_cast<long long>(fixed_bytes(k));
+    const long long s = room / kStageBytes;
+    return static_cast<int>(s > kMaxStages ? kMaxStages : s);
+  }
+  static size_t smem_bytes(int k) {
+    return fixed_bytes(k) + static_cast<size_t>(stages(k)) * kStageBytes;
+  }
+};
+
+struct ProjArgs {
+  const float* L;          // base logits of depth d, request 0
+  long long l_req_stride;  // floats between two requests' rows
+  int V, H, k, rows, rows_per_req, col0, n_stages;
+  float* part_m;           // [rows][n_parts] per-CTA max
+  float* part_s;           // [rows][n_parts] per-CTA sum of exp
+  float* part_z;           // [rows][n_parts][k] per-CTA top-k logits, best first
+  int32_t* part_t;         // [rows][n_parts][k] their tokens
+  int32_t* status;
+};
+
+__device__ __forceinline__ void epi_barrier() { named_barrier(1, kEpiThreads); }
+
+template <int NC>
+__global__ void __launch_bounds__(kThreads, 1)
+markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
+                    const __grid_constant__ CUtensorMap tmap_x,
+                    const __grid_constant__ ProjArgs a) {
+  using C = FusedProj<NC>;
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* base = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int n_stages = a.n_stages;
+  const int k = a.k;
+  unsigned char* ring = base;
+  float(*zs)[kBM] = reinterpret_cast<float(*)[kBM]>(ring + n_stages * C::kStageBytes);
+  float* row_m = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(zs) + C::kZBytes);
+  float* row_s = row_m + NC;
+  float* thr_v = row_s + NC;                          // the list's k-th entry
+  int* thr_t = reinterpret_cast<int*>(thr_v + NC);
+  float* lv = reinterpret_cast<float*>(thr_t + NC);   // [NC][k]
+  int* lt = reinterpret_cast<int*>(lv + NC * k);      // [NC][k]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(lt + NC * k);
+  uint64_t* full = bars;                              // [kMaxStages]
+  uint64_t* empty = bars + kMaxStages;                // [kMaxStages]
+  uint64_t* acc_full = bars + 2 * kMaxStages;         // [2]
+  uint64_t* acc_empty = acc_full + 2;                 // [2]
+  uint64_t* drain = acc_empty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+  int* stop_flag = abort_flag + 1;
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int n_tiles = (a.V + kBM - 1) / kBM;
+  const int n_k = (a.H + kBK - 1) / kBK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < n_stages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], kEpiWarps);   // one arrival per epilogue warp
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    *stop_flag = 0;
+    fence_barrier_init();
+    tma_prefetch_desc(&tmap_w);
+    tma_prefetch_desc(&tmap_x);
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  const uint32_t tmem_base = *tmem_slot;
+  volatile int* abort_v = abort_flag;
+
+  if (warp == 0) {
+    // --------------------------------------------------------------- producer
+    if (lane == 0) {
+      const uint64_t stream_policy = l2_policy_evict_first();
+      int stage = 0;
+      uint32_t phase = 0;
+      int armed[kMaxStages];
+      for (int s = 0; s < kMaxStages; ++s) armed[s] = -1;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+        for (int kc = 0; kc < n_k; ++kc) {
+          if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_v, kWaitLimitNs)) {
+            ok = false;
+            break;
+          }
+          unsigned char* a_dst = ring + stage * C::kStageBytes;
+          mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
+          tma_load_2d_hint(a_dst, &tmap_w, &full[stage], kc * kBK, tile * kBM,
+                           stream_policy);
+          tma_load_2d(a_dst + C::kABytes, &tmap_x, &full[stage], kc * kBK, a.col0);
+          armed[stage] = static_cast<int>(phase);
+          if (++stage == n_stages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        *abort_v = 1;
+        set_status(a.status, PCTREE_ERR_TIMEOUT);
+      }
+      // every copy issued here must land before the CTA may exit
+      volatile int never = 0;
+      for (int s = 0; s < n_stages; ++s)
+        if (armed[s] >= 0)
+          mbar_wait_bounded(&full[s], static_cast<uint32_t>(armed[s]), &never,
+                            kWaitLimitNs);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------- MMA issue
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(kBM, NC);
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+        if (!mbar_wait_bounded(&acc_empty[acc], acc_phase ^ 1u, abort_v, kWaitLimitNs)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after_sync();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * NC);
+        for (int kc = 0; kc < n_k; ++kc) {
+          if (!mbar_wait_bounded(&full[stage], phase, abort_v, kWaitLimitNs)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after_sync();
+          const uint32_t a_addr = smem_u32(ring + stage * C::kStageBytes);
+          const uint32_t b_addr = a_addr + C::kABytes;
+#pragma unroll
+          for (int kk = 0; kk < kBK / kUmmaK; ++kk)
+            tc_mma_bf16(d_tmem, desc_kmajor_sw128(a_addr + kk * kUmmaK * 2),
+                        desc_kmajor_sw128(b_addr + kk * kUmmaK * 2), idesc,
+                        (kc | kk) != 0 ? 1u : 0u);
+          tc_commit(&empty[stage]);   // frees the ring slot once read
+          if (++stage == n_stages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        tc_commit(&acc_full[acc]);    // accumulator ready for the epilogue
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1u;
+      }
+      if (!ok) {
+        *abort_v = 1;
+        set_status(a.status, PCTREE_ERR_TIMEOUT);
+      }
+      // every MMA issued here must be complete before TMEM is released
+      tc_commit(drain);
+      volatile int never = 0;
+      mbar_wait_bounded(drain, 0, &never, kWaitLimitNs);
+    }
+  } else {
+    // --------------------------------------------------------------- epilogue
+    const int ew = warp - 2;                 // 0..7
+    const int quad = warp & 3;               // TMEM lanes 32*quad .. +31
+    const int half = ew >> 2;                // chunk columns 32*half .. +31
+    const int tid = ew * 32 + lane;
+    const int cols = min(NC, a.rows - a.col0);   // valid columns of this pass
+    const int cols16 = (cols + 15) & ~15;
+    for (int r = tid; r < NC; r += kEpiThreads) {
+      row_m[r] = kNegInf;
+      row_s[r] = 0.0f;
+    }
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    bool bad = false;
+    bool first = true;                       // this CTA's first tile
+    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+      // the lanes agree before the warp-collective TMEM loads; then one
+      // decision for all eight warps, which meet at named barriers below
+      const bool got = __all_sync(kFull, mbar_wait_bounded(&acc_full[acc], acc_phase,
+                                                           abort_v, kWaitLimitNs));
+      if (!got && lane == 0) {
+        *abort_v = 1;
+        set_status(a.status, PCTREE_ERR_TIMEOUT);
+      }
+      epi_barrier();
+      if (tid == 0) *stop_flag = *abort_v;
+      epi_barrier();
+      if (*stop_flag) break;
+      tc_fence_after_sync();
+      const int v0 = tile * kBM;
+      const uint32_t t_lane = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                              static_cast<uint32_t>(acc * NC);
+      for (int c0 = 0; c0 < cols; c0 += kCC) {
+        // A: 32 lanes x (up to) 32 columns of this warp's quadrant, transposed
+        // into zs[column - c0][vocabulary row of the tile]
+#pragma unroll
+        for (int g = 0; g < 2; ++g) {
+          const int cg = c0 + half * 32 + g * 16;
+          if (cg < cols16) {
+            uint32_t r[16];
+            tmem_ld_32x32b_x16(t_lane + static_cast<uint32_t>(cg), r);
+            tmem_ld_wait();
+#pragma unroll
+            for (int j = 0; j < 16; ++j) zs[cg - c0 + j][quad * 32 + lane] = __uint_as_float(r[j]);
+          }
+        }
+        if (c0 + kCC >= cols) {
+          // this warp's last TMEM read of the tile: hand the buffer back
+          tc_fence_before_sync();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&acc_empty[acc]);
+        }
+        epi_barrier();
+        // B: rows c0 + 8 ew .. +7 of the pass
+#pragma unroll 1
+        for (int i = 0; i < kRowsPerWarp; ++i) {
+          const int rl = c0 + ew * kRowsPerWarp + i;    // pass-local row
+          if (rl >= cols) break;
+          const int row = a.col0 + rl;
+          const float* Lr = a.L + static_cast<long long>(row / a.rows_per_req) * a.l_req_stride;
+          const float4 acc4 = reinterpret_cast<const float4*>(zs[rl - c0])[lane];
+          const float av[4] = {acc4.x, acc4.y, acc4.z, acc4.w};
+          float z[4];
+          int t[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int v = v0 + lane * 4 + e;
+            z[e] = kNegInf;
+            t[e] = 0x7fffffff;
+            if (v < a.V) {
+              const float lval = __ldg(Lr + v);
+              z[e] = lval + av[e];
+              t[e] = v;
+              bad |= isnan(z[e]) || (isinf(z[e]) && !(isinf(lval) && lval < 0.0f));
+            }
+          }
+          // running log-sum-exp of the row (Eq. 2): the tile's warp maximum
+          // and sum of exp, folded into the row's pair by lane 0
+          float lm = fmaxf(fmaxf(z[0], z[1]), fmaxf(z[2], z[3]));
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) lm = fmaxf(lm, __shfl_xor_sync(kFull, lm, o));
+          float es = 0.0f;
+          if (lm > kNegInf) {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) es += __expf(z[e] - lm);
+          }
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) es += __shfl_xor_sync(kFull, es, o);
+          if (lane == 0) {
+            float m = row_m[rl], s = row_s[rl];
+            lse_merge(m, s, lm, es);
+            row_m[rl] = m;
+            row_s[rl] = s;
+          }
+          // top-k of the row over this CTA's tiles
+          WarpList lst;
+          int best = 0;
+#pragma unroll
+          for (int e = 1; e < 4; ++e)
+            if (cand_better(z[e], t[e], z[best], t[best])) best = e;
+          unsigned marks = 0;
+          if (first) {
+            // the list starts from the lanes' best logits (a sort), then
+            // takes the others that beat its k-th entry
+            float bv = z[0];
+            int bt = t[0];
+#pragma unroll
+            for (int e = 1; e < 4; ++e)
+              if (e == best) {
+                bv = z[e];
+                bt = t[e];
+              }
+            lst.seed(bv, bt, k);
+            const float tv = __shfl_sync(kFull, lst.v, k - 1);
+            const int tt = __shfl_sync(kFull, lst.t, k - 1);
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+              if (e != best && cand_better(z[e], t[e], tv, tt)) marks |= 1u << e;
+          } else {
+            const float tv = thr_v[rl];
+            const int tt = thr_t[rl];
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+              if (cand_better(z[e], t[e], tv, tt)) marks |= 1u << e;
+            if (!__any_sync(kFull, marks != 0)) continue;
+            if (lane < k) {
+              lst.v = lv[rl * k + lane];
+              lst.t = lt[rl * k + lane];
+            } else {
+              lst.reset();
+            }
+          }
+          while (__any_sync(kFull, marks != 0)) {
+            const int sel = marks != 0 ? __ffs(marks) - 1 : -1;
+            marks &= marks - 1;
+            float cv = kNegInf;
+            int ct = 0x7fffffff;
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+              if (e == sel) {
+                cv = z[e];
+                ct = t[e];
+              }
+            lst.offer(cv, ct, k);
+          }
+          if (lane < k) {
+            lv[rl * k + lane] = lst.v;
+            lt[rl * k + lane] = lst.t;
+          }
+          if (lane == k - 1) {
+            thr_v[rl] = lst.v;
+            thr_t[rl] = lst.t;
+          }
+        }
+        epi_barrier();   // zs is rewritten by the next chunk
+      }
+      first = false;
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1u;
+    }
+    if (bad) set_status(a.status, PCTREE_ERR_NONFINITE);
+    // this CTA's partial of every row of the pass (a CTA without tiles
+    // publishes empty partials: max -inf, no candidates)
+    epi_barrier();
+    if (!*stop_flag) {
+      const size_t n_parts = gridDim.x;
+      for (int rl = ew; rl < cols; rl += kEpiWarps) {
+        const size_t p = static_cast<size_t>(a.col0 + rl) * n_parts + blockIdx.x;
+        if (lane == 0) {
+          a.part_m[p] = row_m[rl];
+          a.part_s[p] = row_s[rl];
+        }
+        if (lane < k) {
+          const bool any = !first;
+          a.part_z[p * k + lane] = any ? lv[rl * k + lane] : kNegInf;
+          a.part_t[p * k + lane] = any ? lt[rl * k + lane] : 0x7fffffff;
+        }
+      }
+    }
+  }
+
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  if (warp == 1) tmem_dealloc(tmem_base, C::kTmemCols);
+}
+
+template <int NC>
+cudaError_t launch_nc(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
+                      ProjArgs a, int num_sms, cudaStream_t stream) {
+  using C = FusedProj<NC>;
+  const int stages = C::stages(a.k);
+  if (stages < 2) return cudaErrorInvalidValue;
+  const size_t smem = C::smem_bytes(a.k);
+  static SmemLimit limit;
+  cudaError_t e = limit.ensure(reinterpret_cast<const void*>(markov_fused_kernel<NC>),
+                               kSmemLimit);
+  if (e != cudaSuccess) return e;
+  a.n_stages = stages;
+  const int grid = fused_proj_parts(a.V, num_sms);
+  const int rows = a.rows;
+  for (int col0 = 0; col0 < rows; col0 += NC) {
+    a.col0 = col0;
+    markov_fused_kernel<NC><<<grid, kThreads, smem, stream>>>(*tmap_w, *tmap_x, a);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace
+
+int fused_proj_parts(int V, int num_sms) {
+  const int n_tiles = (V + kBM - 1) / kBM;
+  const int g = n_tiles < num_sms ? n_tiles : num_sms;
+  return g < kFusedMaxGrid ? g : kFusedMaxGrid;   // partial slots per row
+}
+
+cudaError_t launch_markov_fused(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
+                                const float* L, long long l_req_stride, int V,
+                                int H, int k, int rows, int rows_per_req, int bn,
+                                int num_sms, float* part_m, float* part_s,
+                                float* part_z, int32_t* part_t, int32_t* status,
+                                cudaStream_t stream) {
+  ProjArgs a{};
+  a.L = L;
+  a.l_req_stride = l_req_stride;
+  a.V = V;
+  a.H = H;
+  a.k = k;
+  a.rows = rows;
+  a.rows_per_req = rows_per_req;
+  a.part_m = part_m;
+  a.part_s = part_s;
+  a.part_z = part_z;
+  a.part_t = part_t;
+  a.status = status;
+  switch (bn) {
+    case 16: return launch_nc<16>(tmap_w, tmap_x, a, num_sms, stream);
+    case 32: return launch_nc<32>(tmap_w, tmap_x, a, num_sms, stream);
+    case 64: return launch_nc<64>(tmap_w, tmap_x, a, num_sms, stream);
+    case 128: return launch_nc<128>(tmap_w, tmap_x, a, num_sms, stream);
+    case 256: return launch_nc<256>(tmap_w, tmap_x, a, num_sms, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace pct

@@ -28,7 +28,7 @@ namespace pct {
 namespace {
 
 // 16 MiB: enough for batch-1 Qwen3-shaped rounds (pctree_workspace_bytes is
-// 9.47 MB for V=151936, H=2560, B=16, k=8, N=64 and 14.7 MB for V=151936,
+// 4.74 MB for V=151936, H=2560, B=16, k=8, N=64 and 5.54 MB for V=151936,
 // H=5120, B=16, k=16, N=128); larger rounds are rejected.
 constexpr size_t kStaticScratchBytes = size_t(16) << 20;
 

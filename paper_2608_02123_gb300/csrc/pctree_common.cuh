@@ -25,8 +25,9 @@ struct Layout {
   int rows_max;   // batch * k: Markov rows of a full stage
   int rows_pad;   // rows of the X buffer (multiple of 16)
   int bn;         // MMA N tile (rows per projection pass)
-  int ldz;        // row stride of the stage logits Z, in floats
-  int n_chunks;   // vocabulary chunks per row in the partials pass
+  int ldz;        // row stride of the stage logits Z, in floats (f32 heads)
+  int n_chunks;   // vocabulary chunks per row in the partials pass (f32)
+  int part_slots; // partials per row the workspace holds
   int P;          // candidate pool capacity per request
   int x_elem;     // bytes per X element
   size_t off_x, off_z, off_pm, off_ps, off_pz, off_pt;
@@ -284,9 +285,6 @@ class SmemLimit {
   bool done_[kMaxDevices] = {};
 };
 
-// Z[row][v] = L[req(row)][v] + sum_h W_out[v][h] X[row][h] for rows
-// [0, rows), req(row) = row / rows_per_req.  `L` points at depth d of
-// request 0; requests are `l_req_stride` floats apart.
 // SM count of the current device and the driver's tensor-map encoder, looked
 // up once per device (api.cu).
 pctree_status device_facts(int* num_sms);
@@ -299,13 +297,24 @@ pctree_status encode_bf16_map_nd(CUtensorMap* map, const void* base, int rank,
                                  const uint64_t* strides_bytes,
                                  const uint32_t* box);
 
-cudaError_t launch_markov_bf16(const CUtensorMap* tmap_w,
-                               const CUtensorMap* tmap_x, const float* L,
-                               long long l_req_stride, float* Z, int ldz,
-                               int V, int H, int rows, int rows_per_req,
-                               int bn, int num_sms, int32_t* status,
-                               cudaStream_t stream);
+// bf16 heads: the stage's projection with the log-softmax normaliser and
+// top-k folded into the epilogue (markov_fused.cu).  For rows [0, rows) it
+// writes one partial per (row, CTA): part_m/part_s[row * n_parts + cta] and
+// part_z/part_t[(row * n_parts + cta) * k + j], n_parts =
+// fused_proj_parts(V, num_sms).  `L` points at depth d of request 0.
+int fused_proj_parts(int V, int num_sms);
 
+cudaError_t launch_markov_fused(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
+                                const float* L, long long l_req_stride, int V,
+                                int H, int k, int rows, int rows_per_req, int bn,
+                                int num_sms, float* part_m, float* part_s,
+                                float* part_z, int32_t* part_t, int32_t* status,
+                                cudaStream_t stream);
+
+// f32 heads: Z[row][v] = L[req(row)][v] + sum_h W_out[v][h] X[row][h] for
+// rows [0, rows), req(row) = row / rows_per_req; `L` points at depth d of
+// request 0, requests `l_req_stride` floats apart.  partials_kernel then
+// reduces Z chunk by chunk.
 cudaError_t launch_markov_f32(const float* W_out, const float* X,
                               const float* L, long long l_req_stride, float* Z,
                               int ldz, int V, int H, int rows,
@@ -332,8 +341,10 @@ inline int rows_per_request(const pctree_config& c, int d) {
   return c.mode == PCTREE_MODE_SHARED ? 1 : (d == 0 ? 1 : c.k);
 }
 
+// n_parts: partials per row (vocabulary chunks of the f32 path, or the
+// projection's CTAs of the bf16 path).
 cudaError_t launch_merge(const pctree_config& c, const Layout& lay, int d,
-                         const void* E_in, unsigned char* ws,
+                         int n_parts, const void* E_in, unsigned char* ws,
                          int32_t* status, cudaStream_t stream);
 
 cudaError_t launch_pack(const pctree_config& c, const Layout& lay,

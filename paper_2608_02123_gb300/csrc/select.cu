@@ -696,7 +696,7 @@ cudaError_t launch_partials(const Layout& lay, int k, int V, int rows,
 }
 
 cudaError_t launch_merge(const pctree_config& c, const Layout& lay, int d,
-                         const void* E_in, unsigned char* ws,
+                         int n_parts, const void* E_in, unsigned char* ws,
                          int32_t* status, cudaStream_t stream) {
   const int b_d = d == 0 ? 1 : c.k;
   const int rpq = rows_per_request(c, d);
@@ -704,7 +704,7 @@ cudaError_t launch_merge(const pctree_config& c, const Layout& lay, int d,
   const int threads = rpq * 32 > 256 ? rpq * 32 : 256;
   merge_kernel<<<c.batch, threads, smem, stream>>>(
       d, c.B, c.k, b_d, rpq, c.mode == PCTREE_MODE_SHARED ? 1 : 0, c.V, c.H,
-      lay.P, lay.n_chunks, lay.x_elem,
+      lay.P, n_parts, lay.x_elem,
       reinterpret_cast<const float*>(ws + lay.off_pm),
       reinterpret_cast<const float*>(ws + lay.off_ps),
       reinterpret_cast<const float*>(ws + lay.off_pz),

@@ -368,8 +368,11 @@ def kernels_per_round(cfg: Config, path: int = PATH_AUTO) -> int:
     for d in range(cfg.B):
         rpq = 1 if (cfg.mode == MODE_SHARED or d == 0) else cfg.k
         rows = cfg.batch * rpq
-        passes = (rows + 255) // 256 if cfg.weight_dtype == PCTREE_BF16 else 1
-        launches += passes + 2        # projection, partials, merge
+        if cfg.weight_dtype == PCTREE_BF16:
+            # projection passes (normaliser and top-k partials folded in), merge
+            launches += (rows + 255) // 256 + 1
+        else:
+            launches += 3             # projection, partials, merge
     return launches
 
 

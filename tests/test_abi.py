@@ -56,7 +56,10 @@ def test_sizes(P):
     c = P.make_config(151936, 2560, 16, 8, 64, 1)
     assert P.pctree_pool_capacity(c) == 1 + 8 + 15 * 64
     ws = P.pctree_workspace_bytes(c)
-    assert ws % 256 == 0 and ws > 8 * 151936 * 4
+    # bf16 heads never hold a stage's logits (8 rows x V floats) in memory
+    assert ws % 256 == 0 and ws < 8 * 151936 * 4
+    c32 = P.make_config(151936, 2560, 16, 8, 64, 1, 0, "f32")
+    assert P.pctree_workspace_bytes(c32) > 8 * 151936 * 4
     assert P.pctree_workspace_bytes(P.make_config(10, 8, 2, 11, 4, 1)) == 0
 
 
