@@ -149,8 +149,8 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
       const uint64_t stream_policy = l2_policy_evict_first();
       int stage = 0;
       uint32_t phase = 0;
-      int armed[kMaxStages];
-      for (int s = 0; s < kMaxStages; ++s) armed[s] = -1;
+      // ring slots holding a copy issued here, and the phase each was armed in
+      uint32_t armed = 0, armed_phase = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
         for (int kc = 0; kc < n_k; ++kc) {
@@ -163,7 +163,8 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
           tma_load_2d_hint(a_dst, &tmap_w, &full[stage], kc * kBK, tile * kBM,
                            stream_policy);
           tma_load_2d(a_dst + C::kABytes, &tmap_x, &full[stage], kc * kBK, a.col0);
-          armed[stage] = static_cast<int>(phase);
+          armed |= 1u << stage;
+          armed_phase = (armed_phase & ~(1u << stage)) | (phase << stage);
           if (++stage == n_stages) {
             stage = 0;
             phase ^= 1u;
@@ -177,9 +178,8 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
       // every copy issued here must land before the CTA may exit
       volatile int never = 0;
       for (int s = 0; s < n_stages; ++s)
-        if (armed[s] >= 0)
-          mbar_wait_bounded(&full[s], static_cast<uint32_t>(armed[s]), &never,
-                            kWaitLimitNs);
+        if ((armed >> s) & 1u)
+          mbar_wait_bounded(&full[s], (armed_phase >> s) & 1u, &never, kWaitLimitNs);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------- MMA issue
@@ -284,105 +284,157 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
           if (lane == 0) mbar_arrive(&acc_empty[acc]);
         }
         epi_barrier();
-        // B: rows c0 + 8 ew .. +7 of the pass
+        // B: rows r0 .. r0 + 7 of the pass, processed together so that their
+        // loads and warp reductions overlap (compile-time row indices keep
+        // every value in registers)
+        const int r0 = c0 + ew * kRowsPerWarp;       // pass-local rows
+        const int nr = min(kRowsPerWarp, cols - r0);
+        if (nr > 0) {
+          float z[kRowsPerWarp][4];
+#pragma unroll
+          for (int i = 0; i < kRowsPerWarp; ++i) {
+            const float4 acc4 = reinterpret_cast<const float4*>(zs[r0 - c0 + i])[lane];
+            z[i][0] = acc4.x;
+            z[i][1] = acc4.y;
+            z[i][2] = acc4.z;
+            z[i][3] = acc4.w;
+          }
+          const int vb = v0 + lane * 4;
+#pragma unroll
+          for (int i = 0; i < kRowsPerWarp; ++i) {
+            const int row = a.col0 + r0 + (i < nr ? i : 0);
+            const float* Lr = a.L + static_cast<long long>(row / a.rows_per_req) * a.l_req_stride;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              if (i < nr && vb + e < a.V) {
+                const float lval = __ldg(Lr + vb + e);
+                z[i][e] += lval;
+                bad |= isnan(z[i][e]) || (isinf(z[i][e]) && !(isinf(lval) && lval < 0.0f));
+              } else {
+                z[i][e] = kNegInf;
+              }
+            }
+          }
+          // running log-sum-exp of each row (Eq. 2): the tile's warp maximum
+          // and sum of exp; lane i folds row i's pair into its running one
+          float lm[kRowsPerWarp], es[kRowsPerWarp];
+#pragma unroll
+          for (int i = 0; i < kRowsPerWarp; ++i)
+            lm[i] = fmaxf(fmaxf(z[i][0], z[i][1]), fmaxf(z[i][2], z[i][3]));
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+            for (int i = 0; i < kRowsPerWarp; ++i)
+              lm[i] = fmaxf(lm[i], __shfl_xor_sync(kFull, lm[i], o));
+          }
+#pragma unroll
+          for (int i = 0; i < kRowsPerWarp; ++i) {
+            es[i] = 0.0f;
+            if (lm[i] > kNegInf) {
+#pragma unroll
+              for (int e = 0; e < 4; ++e) es[i] += __expf(z[i][e] - lm[i]);
+            }
+          }
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+            for (int i = 0; i < kRowsPerWarp; ++i)
+              es[i] += __shfl_xor_sync(kFull, es[i], o);
+          }
+          {
+            float my_m = kNegInf, my_s = 0.0f;
+#pragma unroll
+            for (int i = 0; i < kRowsPerWarp; ++i)
+              if (lane == i) {
+                my_m = lm[i];
+                my_s = es[i];
+              }
+            if (lane < nr) {
+              float m = row_m[r0 + lane], s = row_s[r0 + lane];
+              lse_merge(m, s, my_m, my_s);
+              row_m[r0 + lane] = m;
+              row_s[r0 + lane] = s;
+            }
+          }
+          // top-k of each row over this CTA's tiles: bits 4i..4i+3 of `mk`
+          // mark this lane's logits of row i that beat the row's k-th entry
+          uint32_t mk = 0;
+          if (!first) {
+#pragma unroll
+            for (int i = 0; i < kRowsPerWarp; ++i) {
+              if (i < nr) {
+                const float tv = thr_v[r0 + i];
+                const int tt = thr_t[r0 + i];
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                  if (cand_better(z[i][e], vb + e, tv, tt)) mk |= 1u << (4 * i + e);
+              }
+            }
+          }
+          if (first || __any_sync(kFull, mk != 0)) {
 #pragma unroll 1
-        for (int i = 0; i < kRowsPerWarp; ++i) {
-          const int rl = c0 + ew * kRowsPerWarp + i;    // pass-local row
-          if (rl >= cols) break;
-          const int row = a.col0 + rl;
-          const float* Lr = a.L + static_cast<long long>(row / a.rows_per_req) * a.l_req_stride;
-          const float4 acc4 = reinterpret_cast<const float4*>(zs[rl - c0])[lane];
-          const float av[4] = {acc4.x, acc4.y, acc4.z, acc4.w};
-          float z[4];
-          int t[4];
+            for (int i = 0; i < nr; ++i) {
+              unsigned marks = (mk >> (4 * i)) & 15u;
+              if (!first && !__any_sync(kFull, marks != 0)) continue;
+              float zz[4];
+              int tk[4];
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const int v = v0 + lane * 4 + e;
-            z[e] = kNegInf;
-            t[e] = 0x7fffffff;
-            if (v < a.V) {
-              const float lval = __ldg(Lr + v);
-              z[e] = lval + av[e];
-              t[e] = v;
-              bad |= isnan(z[e]) || (isinf(z[e]) && !(isinf(lval) && lval < 0.0f));
-            }
-          }
-          // running log-sum-exp of the row (Eq. 2): the tile's warp maximum
-          // and sum of exp, folded into the row's pair by lane 0
-          float lm = fmaxf(fmaxf(z[0], z[1]), fmaxf(z[2], z[3]));
+              for (int e = 0; e < 4; ++e) {
+                zz[e] = kNegInf;
 #pragma unroll
-          for (int o = 16; o > 0; o >>= 1) lm = fmaxf(lm, __shfl_xor_sync(kFull, lm, o));
-          float es = 0.0f;
-          if (lm > kNegInf) {
-#pragma unroll
-            for (int e = 0; e < 4; ++e) es += __expf(z[e] - lm);
-          }
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) es += __shfl_xor_sync(kFull, es, o);
-          if (lane == 0) {
-            float m = row_m[rl], s = row_s[rl];
-            lse_merge(m, s, lm, es);
-            row_m[rl] = m;
-            row_s[rl] = s;
-          }
-          // top-k of the row over this CTA's tiles
-          WarpList lst;
-          int best = 0;
-#pragma unroll
-          for (int e = 1; e < 4; ++e)
-            if (cand_better(z[e], t[e], z[best], t[best])) best = e;
-          unsigned marks = 0;
-          if (first) {
-            // the list starts from the lanes' best logits (a sort), then
-            // takes the others that beat its k-th entry
-            float bv = z[0];
-            int bt = t[0];
-#pragma unroll
-            for (int e = 1; e < 4; ++e)
-              if (e == best) {
-                bv = z[e];
-                bt = t[e];
+                for (int ii = 0; ii < kRowsPerWarp; ++ii)
+                  if (ii == i) zz[e] = z[ii][e];
+                tk[e] = vb + e < a.V ? vb + e : 0x7fffffff;
               }
-            lst.seed(bv, bt, k);
-            const float tv = __shfl_sync(kFull, lst.v, k - 1);
-            const int tt = __shfl_sync(kFull, lst.t, k - 1);
+              const int rl = r0 + i;
+              WarpList lst;
+              if (first) {
+                // the list starts from the lanes' best logits (a sort), then
+                // takes the others that beat its k-th entry
+                float bv = zz[0];
+                int bt = tk[0], best = 0;
 #pragma unroll
-            for (int e = 0; e < 4; ++e)
-              if (e != best && cand_better(z[e], t[e], tv, tt)) marks |= 1u << e;
-          } else {
-            const float tv = thr_v[rl];
-            const int tt = thr_t[rl];
+                for (int e = 1; e < 4; ++e)
+                  if (cand_better(zz[e], tk[e], bv, bt)) {
+                    bv = zz[e];
+                    bt = tk[e];
+                    best = e;
+                  }
+                lst.seed(bv, bt, k);
+                const float tv = __shfl_sync(kFull, lst.v, k - 1);
+                const int tt = __shfl_sync(kFull, lst.t, k - 1);
+                marks = 0;
 #pragma unroll
-            for (int e = 0; e < 4; ++e)
-              if (cand_better(z[e], t[e], tv, tt)) marks |= 1u << e;
-            if (!__any_sync(kFull, marks != 0)) continue;
-            if (lane < k) {
-              lst.v = lv[rl * k + lane];
-              lst.t = lt[rl * k + lane];
-            } else {
-              lst.reset();
-            }
-          }
-          while (__any_sync(kFull, marks != 0)) {
-            const int sel = marks != 0 ? __ffs(marks) - 1 : -1;
-            marks &= marks - 1;
-            float cv = kNegInf;
-            int ct = 0x7fffffff;
-#pragma unroll
-            for (int e = 0; e < 4; ++e)
-              if (e == sel) {
-                cv = z[e];
-                ct = t[e];
+                for (int e = 0; e < 4; ++e)
+                  if (e != best && cand_better(zz[e], tk[e], tv, tt)) marks |= 1u << e;
+              } else if (lane < k) {
+                lst.v = lv[rl * k + lane];
+                lst.t = lt[rl * k + lane];
+              } else {
+                lst.reset();
               }
-            lst.offer(cv, ct, k);
-          }
-          if (lane < k) {
-            lv[rl * k + lane] = lst.v;
-            lt[rl * k + lane] = lst.t;
-          }
-          if (lane == k - 1) {
-            thr_v[rl] = lst.v;
-            thr_t[rl] = lst.t;
+              while (__any_sync(kFull, marks != 0)) {
+                const int sel = marks != 0 ? __ffs(marks) - 1 : -1;
+                marks &= marks - 1;
+                float cv = kNegInf;
+                int ct = 0x7fffffff;
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                  if (e == sel) {
+                    cv = zz[e];
+                    ct = tk[e];
+                  }
+                lst.offer(cv, ct, k);
+              }
+              if (lane < k) {
+                lv[rl * k + lane] = lst.v;
+                lt[rl * k + lane] = lst.t;
+              }
+              if (lane == k - 1) {
+                thr_v[rl] = lst.v;
+                thr_t[rl] = lst.t;
+              }
+            }
           }
         }
         epi_barrier();   // zs is rewritten by the next chunk
