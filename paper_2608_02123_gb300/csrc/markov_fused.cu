@@ -47,6 +47,8 @@ constexpr int kMaxStages = 8;
 constexpr int kSmemLimit = 227 * 1024;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per bounded wait
 constexpr float kNegInf = -INFINITY;
+constexpr float kPosInf = INFINITY;
+constexpr float kLog2e = 1.4426950408889634f;
 
 // Shared-memory plan of one instance (NC columns, k up to PCTREE_MAX_K).
 template <int NC>
@@ -56,8 +58,8 @@ struct FusedProj {
   static constexpr int kStageBytes = kABytes + kBBytes;  // multiple of 1024
   static constexpr int kTmemCols = 2 * NC < 32 ? 32 : 2 * NC;
   static constexpr size_t kZBytes = static_cast<size_t>(kCC) * kBM * sizeof(float);
-  // per-row running state: max, sum, k-th entry (value, token)
-  static constexpr size_t kRowBytes = static_cast<size_t>(NC) * 16;
+  // per-row k-th entry of the top-k list (the insertion threshold)
+  static constexpr size_t kRowBytes = static_cast<size_t>(NC) * 4;
   static constexpr size_t kBarBytes = 256;
   static size_t list_bytes(int k) { return static_cast<size_t>(NC) * k * 8; }
   static size_t fixed_bytes(int k) {
@@ -99,11 +101,8 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
   const int k = a.k;
   unsigned char* ring = base;
   float(*zs)[kBM] = reinterpret_cast<float(*)[kBM]>(ring + n_stages * C::kStageBytes);
-  float* row_m = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(zs) + C::kZBytes);
-  float* row_s = row_m + NC;
-  float* thr_v = row_s + NC;                          // the list's k-th entry
-  int* thr_t = reinterpret_cast<int*>(thr_v + NC);
-  float* lv = reinterpret_cast<float*>(thr_t + NC);   // [NC][k]
+  float* thr_v = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(zs) + C::kZBytes);
+  float* lv = thr_v + NC;                             // [NC][k]
   int* lt = reinterpret_cast<int*>(lv + NC * k);      // [NC][k]
   uint64_t* bars = reinterpret_cast<uint64_t*>(lt + NC * k);
   uint64_t* full = bars;                              // [kMaxStages]
@@ -238,10 +237,19 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
     const int tid = ew * 32 + lane;
     const int cols = min(NC, a.rows - a.col0);   // valid columns of this pass
     const int cols16 = (cols + 15) & ~15;
-    for (int r = tid; r < NC; r += kEpiThreads) {
-      row_m[r] = kNegInf;
-      row_s[r] = 0.0f;
-    }
+    // This warp's rows are c * 64 + 8 ew + i (chunk c, i < 8) in every
+    // tile.  Each lane keeps, per row, a running (max, sum of exp) over its
+    // own logits of the row (Eq. 2); the lanes' pairs are combined once, at
+    // the end of the pass.
+    constexpr int kChunks = (NC + kCC - 1) / kCC;
+    float run_m[kChunks][kRowsPerWarp], run_s[kChunks][kRowsPerWarp];
+#pragma unroll
+    for (int c = 0; c < kChunks; ++c)
+#pragma unroll
+      for (int i = 0; i < kRowsPerWarp; ++i) {
+        run_m[c][i] = kNegInf;
+        run_s[c][i] = 0.0f;
+      }
     int acc = 0;
     uint32_t acc_phase = 0;
     bool bad = false;
@@ -261,9 +269,13 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
       if (*stop_flag) break;
       tc_fence_after_sync();
       const int v0 = tile * kBM;
+      const int vb = v0 + lane * 4;          // this lane's 4 logits of a row
       const uint32_t t_lane = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
                               static_cast<uint32_t>(acc * NC);
-      for (int c0 = 0; c0 < cols; c0 += kCC) {
+#pragma unroll
+      for (int c = 0; c < kChunks; ++c) {
+        const int c0 = c * kCC;
+        if (c0 >= cols) break;
         // A: 32 lanes x (up to) 32 columns of this warp's quadrant, transposed
         // into zs[column - c0][vocabulary row of the tile]
 #pragma unroll
@@ -285,8 +297,8 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
         }
         epi_barrier();
         // B: rows r0 .. r0 + 7 of the pass, processed together so that their
-        // loads and warp reductions overlap (compile-time row indices keep
-        // every value in registers)
+        // loads overlap (compile-time row indices keep every value in
+        // registers)
         const int r0 = c0 + ew * kRowsPerWarp;       // pass-local rows
         const int nr = min(kRowsPerWarp, cols - r0);
         if (nr > 0) {
@@ -299,7 +311,6 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
             z[i][2] = acc4.z;
             z[i][3] = acc4.w;
           }
-          const int vb = v0 + lane * 4;
 #pragma unroll
           for (int i = 0; i < kRowsPerWarp; ++i) {
             const int row = a.col0 + r0 + (i < nr ? i : 0);
@@ -308,66 +319,43 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
             for (int e = 0; e < 4; ++e) {
               if (i < nr && vb + e < a.V) {
                 const float lval = __ldg(Lr + vb + e);
+                // non-finite: a Markov bias that is not finite, or a NaN /
+                // +inf base logit (-inf base logits are legal)
+                bad |= !(fabsf(z[i][e]) < kPosInf) || !(lval < kPosInf);
                 z[i][e] += lval;
-                bad |= isnan(z[i][e]) || (isinf(z[i][e]) && !(isinf(lval) && lval < 0.0f));
               } else {
                 z[i][e] = kNegInf;
               }
             }
           }
-          // running log-sum-exp of each row (Eq. 2): the tile's warp maximum
-          // and sum of exp; lane i folds row i's pair into its running one
-          float lm[kRowsPerWarp], es[kRowsPerWarp];
-#pragma unroll
-          for (int i = 0; i < kRowsPerWarp; ++i)
-            lm[i] = fmaxf(fmaxf(z[i][0], z[i][1]), fmaxf(z[i][2], z[i][3]));
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) {
-#pragma unroll
-            for (int i = 0; i < kRowsPerWarp; ++i)
-              lm[i] = fmaxf(lm[i], __shfl_xor_sync(kFull, lm[i], o));
-          }
+          // running (max, sum of exp) of this lane's logits of each row
 #pragma unroll
           for (int i = 0; i < kRowsPerWarp; ++i) {
-            es[i] = 0.0f;
-            if (lm[i] > kNegInf) {
-#pragma unroll
-              for (int e = 0; e < 4; ++e) es[i] += __expf(z[i][e] - lm[i]);
+            const float mx = fmaxf(fmaxf(z[i][0], z[i][1]), fmaxf(z[i][2], z[i][3]));
+            float& m = run_m[c][i];
+            float& sm = run_s[c][i];
+            if (mx > m) {
+              sm *= ex2_approx((m - mx) * kLog2e);   // m = -inf: sm is 0
+              m = mx;
             }
-          }
+            if (m > kNegInf) {
+              const float mb = m * kLog2e;
 #pragma unroll
-          for (int o = 16; o > 0; o >>= 1) {
-#pragma unroll
-            for (int i = 0; i < kRowsPerWarp; ++i)
-              es[i] += __shfl_xor_sync(kFull, es[i], o);
-          }
-          {
-            float my_m = kNegInf, my_s = 0.0f;
-#pragma unroll
-            for (int i = 0; i < kRowsPerWarp; ++i)
-              if (lane == i) {
-                my_m = lm[i];
-                my_s = es[i];
-              }
-            if (lane < nr) {
-              float m = row_m[r0 + lane], s = row_s[r0 + lane];
-              lse_merge(m, s, my_m, my_s);
-              row_m[r0 + lane] = m;
-              row_s[r0 + lane] = s;
+              for (int e = 0; e < 4; ++e) sm += ex2_approx(fmaf(z[i][e], kLog2e, -mb));
             }
           }
           // top-k of each row over this CTA's tiles: bits 4i..4i+3 of `mk`
-          // mark this lane's logits of row i that beat the row's k-th entry
+          // mark this lane's logits of row i at or above the row's k-th
+          // entry (offer() applies the exact (value, token) order)
           uint32_t mk = 0;
           if (!first) {
 #pragma unroll
             for (int i = 0; i < kRowsPerWarp; ++i) {
               if (i < nr) {
                 const float tv = thr_v[r0 + i];
-                const int tt = thr_t[r0 + i];
 #pragma unroll
                 for (int e = 0; e < 4; ++e)
-                  if (cand_better(z[i][e], vb + e, tv, tt)) mk |= 1u << (4 * i + e);
+                  if (z[i][e] >= tv) mk |= 1u << (4 * i + e);
               }
             }
           }
@@ -430,10 +418,7 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
                 lv[rl * k + lane] = lst.v;
                 lt[rl * k + lane] = lst.t;
               }
-              if (lane == k - 1) {
-                thr_v[rl] = lst.v;
-                thr_t[rl] = lst.t;
-              }
+              if (lane == k - 1) thr_v[rl] = lst.v;
             }
           }
         }
@@ -444,21 +429,34 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
       if (acc == 0) acc_phase ^= 1u;
     }
     if (bad) set_status(a.status, PCTREE_ERR_NONFINITE);
-    // this CTA's partial of every row of the pass (a CTA without tiles
-    // publishes empty partials: max -inf, no candidates)
+    // this CTA's partial of every row of the pass: the lanes' (max, sum-exp)
+    // pairs combined, and the row's top-k list
     epi_barrier();
     if (!*stop_flag) {
       const size_t n_parts = gridDim.x;
-      for (int rl = ew; rl < cols; rl += kEpiWarps) {
-        const size_t p = static_cast<size_t>(a.col0 + rl) * n_parts + blockIdx.x;
-        if (lane == 0) {
-          a.part_m[p] = row_m[rl];
-          a.part_s[p] = row_s[rl];
-        }
-        if (lane < k) {
-          const bool any = !first;
-          a.part_z[p * k + lane] = any ? lv[rl * k + lane] : kNegInf;
-          a.part_t[p * k + lane] = any ? lt[rl * k + lane] : 0x7fffffff;
+#pragma unroll
+      for (int c = 0; c < kChunks; ++c) {
+#pragma unroll
+        for (int i = 0; i < kRowsPerWarp; ++i) {
+          const int rl = c * kCC + ew * kRowsPerWarp + i;
+          float m = run_m[c][i], sm = run_s[c][i];
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) {
+            const float m2 = __shfl_xor_sync(kFull, m, o);
+            const float s2 = __shfl_xor_sync(kFull, sm, o);
+            lse_merge(m, sm, m2, s2);
+          }
+          if (rl < cols) {
+            const size_t p = static_cast<size_t>(a.col0 + rl) * n_parts + blockIdx.x;
+            if (lane == 0) {
+              a.part_m[p] = m;
+              a.part_s[p] = sm;
+            }
+            if (lane < k) {
+              a.part_z[p * k + lane] = first ? kNegInf : lv[rl * k + lane];
+              a.part_t[p * k + lane] = first ? 0x7fffffff : lt[rl * k + lane];
+            }
+          }
         }
       }
     }
