@@ -89,7 +89,7 @@ struct ProjArgs {
 __device__ __forceinline__ void epi_barrier() { named_barrier(1, kEpiThreads); }
 
 template <int NC>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __maxnreg__(200)
 markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
                     const __grid_constant__ CUtensorMap tmap_x,
                     const __grid_constant__ ProjArgs a) {
@@ -344,9 +344,13 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
               for (int e = 0; e < 4; ++e) sm += ex2_approx(fmaf(z[i][e], kLog2e, -mb));
             }
           }
-          // top-k of each row over this CTA's tiles: bits 4i..4i+3 of `mk`
-          // mark this lane's logits of row i at or above the row's k-th
-          // entry (offer() applies the exact (value, token) order)
+          // top-k of each row over this CTA's tiles.  Bits 4i..4i+3 of `mk`
+          // mark this lane's logits of row i that are candidates: at or above
+          // the row's k-th entry (the first tile: those left after seeding).
+          // The eight rows' lists live in registers and take their
+          // candidates in lockstep, one per row per step, so the rows'
+          // dependent warp operations overlap; insert() applies the exact
+          // (value desc, token asc) order and drops what falls below k.
           uint32_t mk = 0;
           if (!first) {
 #pragma unroll
@@ -360,65 +364,73 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
             }
           }
           if (first || __any_sync(kFull, mk != 0)) {
-#pragma unroll 1
-            for (int i = 0; i < nr; ++i) {
-              unsigned marks = (mk >> (4 * i)) & 15u;
-              if (!first && !__any_sync(kFull, marks != 0)) continue;
-              float zz[4];
-              int tk[4];
+            WarpList lst[kRowsPerWarp];
 #pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                zz[e] = kNegInf;
-#pragma unroll
-                for (int ii = 0; ii < kRowsPerWarp; ++ii)
-                  if (ii == i) zz[e] = z[ii][e];
-                tk[e] = vb + e < a.V ? vb + e : 0x7fffffff;
-              }
-              const int rl = r0 + i;
-              WarpList lst;
+            for (int i = 0; i < kRowsPerWarp; ++i) {
               if (first) {
-                // the list starts from the lanes' best logits (a sort), then
-                // takes the others that beat its k-th entry
-                float bv = zz[0];
-                int bt = tk[0], best = 0;
+                // the list starts from the lanes' best logits (a sort); the
+                // lane's other logits that beat its k-th entry are marked
+                float bv = z[i][0];
+                int bt = vb < a.V ? vb : 0x7fffffff, best = 0;
 #pragma unroll
-                for (int e = 1; e < 4; ++e)
-                  if (cand_better(zz[e], tk[e], bv, bt)) {
-                    bv = zz[e];
-                    bt = tk[e];
+                for (int e = 1; e < 4; ++e) {
+                  const int te = vb + e < a.V ? vb + e : 0x7fffffff;
+                  if (cand_better(z[i][e], te, bv, bt)) {
+                    bv = z[i][e];
+                    bt = te;
                     best = e;
                   }
-                lst.seed(bv, bt, k);
-                const float tv = __shfl_sync(kFull, lst.v, k - 1);
-                const int tt = __shfl_sync(kFull, lst.t, k - 1);
-                marks = 0;
+                }
+                lst[i].seed(i < nr ? bv : kNegInf, i < nr ? bt : 0x7fffffff, k);
+                const float tv = __shfl_sync(kFull, lst[i].v, k - 1);
+                const int tt = __shfl_sync(kFull, lst[i].t, k - 1);
 #pragma unroll
-                for (int e = 0; e < 4; ++e)
-                  if (e != best && cand_better(zz[e], tk[e], tv, tt)) marks |= 1u << e;
-              } else if (lane < k) {
-                lst.v = lv[rl * k + lane];
-                lst.t = lt[rl * k + lane];
+                for (int e = 0; e < 4; ++e) {
+                  const int te = vb + e < a.V ? vb + e : 0x7fffffff;
+                  if (i < nr && e != best && cand_better(z[i][e], te, tv, tt))
+                    mk |= 1u << (4 * i + e);
+                }
+              } else if (i < nr && lane < k) {
+                lst[i].v = lv[(r0 + i) * k + lane];
+                lst[i].t = lt[(r0 + i) * k + lane];
               } else {
-                lst.reset();
+                lst[i].reset();
               }
-              while (__any_sync(kFull, marks != 0)) {
-                const int sel = marks != 0 ? __ffs(marks) - 1 : -1;
-                marks &= marks - 1;
-                float cv = kNegInf;
-                int ct = 0x7fffffff;
+            }
+            while (__any_sync(kFull, mk != 0)) {
 #pragma unroll
-                for (int e = 0; e < 4; ++e)
-                  if (e == sel) {
-                    cv = zz[e];
-                    ct = tk[e];
-                  }
-                lst.offer(cv, ct, k);
+              for (int i = 0; i < kRowsPerWarp; ++i) {
+                // the lowest lane with a candidate of row i offers its first
+                // one (no lane: the sentinel, which changes nothing)
+                const uint32_t mine = (mk >> (4 * i)) & 15u;
+                const uint32_t lanes = __ballot_sync(kFull, mine != 0);
+                const int src = lanes ? __ffs(lanes) - 1 : 0;
+                const int e = mine ? __ffs(mine) - 1 : 0;
+                float cv = z[i][0];
+#pragma unroll
+                for (int q = 1; q < 4; ++q)
+                  if (e == q) cv = z[i][q];
+                int ct = vb + e < a.V ? vb + e : 0x7fffffff;
+                if (!mine) {
+                  cv = kNegInf;
+                  ct = 0x7fffffff;
+                }
+                cv = __shfl_sync(kFull, cv, src);
+                ct = __shfl_sync(kFull, ct, src);
+                if (lane == src && mine) mk &= ~(1u << (4 * i + e));
+                lst[i].insert(cv, ct, k);
               }
-              if (lane < k) {
-                lv[rl * k + lane] = lst.v;
-                lt[rl * k + lane] = lst.t;
+            }
+#pragma unroll
+            for (int i = 0; i < kRowsPerWarp; ++i) {
+              if (i < nr) {
+                const int rl = r0 + i;
+                if (lane < k) {
+                  lv[rl * k + lane] = lst[i].v;
+                  lt[rl * k + lane] = lst[i].t;
+                }
+                if (lane == k - 1) thr_v[rl] = lst[i].v;
               }
-              if (lane == k - 1) thr_v[rl] = lst.v;
             }
           }
         }
