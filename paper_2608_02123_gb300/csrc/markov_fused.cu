@@ -58,8 +58,9 @@ struct FusedProj {
   static constexpr int kStageBytes = kABytes + kBBytes;  // multiple of 1024
   static constexpr int kTmemCols = 2 * NC < 32 ? 32 : 2 * NC;
   static constexpr size_t kZBytes = static_cast<size_t>(kCC) * kBM * sizeof(float);
-  // per-row k-th entry of the top-k list (the insertion threshold)
-  static constexpr size_t kRowBytes = static_cast<size_t>(NC) * 4;
+  // per-row running max and sum of exp, and the k-th entry of the row's
+  // top-k list (the insertion threshold)
+  static constexpr size_t kRowBytes = static_cast<size_t>(NC) * 12;
   static constexpr size_t kBarBytes = 256;
   static size_t list_bytes(int k) { return static_cast<size_t>(NC) * k * 8; }
   static size_t fixed_bytes(int k) {
@@ -89,7 +90,7 @@ struct ProjArgs {
 __device__ __forceinline__ void epi_barrier() { named_barrier(1, kEpiThreads); }
 
 template <int NC>
-__global__ void __maxnreg__(200)
+__global__ void __launch_bounds__(kThreads, 1)
 markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
                     const __grid_constant__ CUtensorMap tmap_x,
                     const __grid_constant__ ProjArgs a) {
@@ -101,7 +102,9 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
   const int k = a.k;
   unsigned char* ring = base;
   float(*zs)[kBM] = reinterpret_cast<float(*)[kBM]>(ring + n_stages * C::kStageBytes);
-  float* thr_v = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(zs) + C::kZBytes);
+  float* row_m = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(zs) + C::kZBytes);
+  float* row_s = row_m + NC;
+  float* thr_v = row_s + NC;                          // the list's k-th entry
   float* lv = thr_v + NC;                             // [NC][k]
   int* lt = reinterpret_cast<int*>(lv + NC * k);      // [NC][k]
   uint64_t* bars = reinterpret_cast<uint64_t*>(lt + NC * k);
@@ -238,18 +241,12 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
     const int cols = min(NC, a.rows - a.col0);   // valid columns of this pass
     const int cols16 = (cols + 15) & ~15;
     // This warp's rows are c * 64 + 8 ew + i (chunk c, i < 8) in every
-    // tile.  Each lane keeps, per row, a running (max, sum of exp) over its
-    // own logits of the row (Eq. 2); the lanes' pairs are combined once, at
-    // the end of the pass.
+    // tile; each keeps a running (max, sum of exp) in shared memory (Eq. 2).
     constexpr int kChunks = (NC + kCC - 1) / kCC;
-    float run_m[kChunks][kRowsPerWarp], run_s[kChunks][kRowsPerWarp];
-#pragma unroll
-    for (int c = 0; c < kChunks; ++c)
-#pragma unroll
-      for (int i = 0; i < kRowsPerWarp; ++i) {
-        run_m[c][i] = kNegInf;
-        run_s[c][i] = 0.0f;
-      }
+    for (int r = tid; r < NC; r += kEpiThreads) {
+      row_m[r] = kNegInf;
+      row_s[r] = 0.0f;
+    }
     int acc = 0;
     uint32_t acc_phase = 0;
     bool bad = false;
@@ -272,7 +269,7 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
       const int vb = v0 + lane * 4;          // this lane's 4 logits of a row
       const uint32_t t_lane = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
                               static_cast<uint32_t>(acc * NC);
-#pragma unroll
+#pragma unroll 1
       for (int c = 0; c < kChunks; ++c) {
         const int c0 = c * kCC;
         if (c0 >= cols) break;
@@ -328,20 +325,46 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
               }
             }
           }
-          // running (max, sum of exp) of this lane's logits of each row
+          // the tile's (max, sum of exp) of each row: eight warp reductions
+          // side by side; lane i folds row i's pair into its running one
+          float lm[kRowsPerWarp], es[kRowsPerWarp];
+#pragma unroll
+          for (int i = 0; i < kRowsPerWarp; ++i)
+            lm[i] = fmaxf(fmaxf(z[i][0], z[i][1]), fmaxf(z[i][2], z[i][3]));
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+            for (int i = 0; i < kRowsPerWarp; ++i)
+              lm[i] = fmaxf(lm[i], __shfl_xor_sync(kFull, lm[i], o));
+          }
 #pragma unroll
           for (int i = 0; i < kRowsPerWarp; ++i) {
-            const float mx = fmaxf(fmaxf(z[i][0], z[i][1]), fmaxf(z[i][2], z[i][3]));
-            float& m = run_m[c][i];
-            float& sm = run_s[c][i];
-            if (mx > m) {
-              sm *= ex2_approx((m - mx) * kLog2e);   // m = -inf: sm is 0
-              m = mx;
-            }
-            if (m > kNegInf) {
-              const float mb = m * kLog2e;
+            es[i] = 0.0f;
+            if (lm[i] > kNegInf) {
+              const float mb = lm[i] * kLog2e;
 #pragma unroll
-              for (int e = 0; e < 4; ++e) sm += ex2_approx(fmaf(z[i][e], kLog2e, -mb));
+              for (int e = 0; e < 4; ++e) es[i] += ex2_approx(fmaf(z[i][e], kLog2e, -mb));
+            }
+          }
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+            for (int i = 0; i < kRowsPerWarp; ++i)
+              es[i] += __shfl_xor_sync(kFull, es[i], o);
+          }
+          {
+            float my_m = kNegInf, my_s = 0.0f;
+#pragma unroll
+            for (int i = 0; i < kRowsPerWarp; ++i)
+              if (lane == i) {
+                my_m = lm[i];
+                my_s = es[i];
+              }
+            if (lane < nr) {
+              float m = row_m[r0 + lane], sm = row_s[r0 + lane];
+              lse_merge(m, sm, my_m, my_s);
+              row_m[r0 + lane] = m;
+              row_s[r0 + lane] = sm;
             }
           }
           // top-k of each row over this CTA's tiles.  Bits 4i..4i+3 of `mk`
@@ -441,34 +464,19 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
       if (acc == 0) acc_phase ^= 1u;
     }
     if (bad) set_status(a.status, PCTREE_ERR_NONFINITE);
-    // this CTA's partial of every row of the pass: the lanes' (max, sum-exp)
-    // pairs combined, and the row's top-k list
+    // this CTA's partial of every row of the pass
     epi_barrier();
     if (!*stop_flag) {
       const size_t n_parts = gridDim.x;
-#pragma unroll
-      for (int c = 0; c < kChunks; ++c) {
-#pragma unroll
-        for (int i = 0; i < kRowsPerWarp; ++i) {
-          const int rl = c * kCC + ew * kRowsPerWarp + i;
-          float m = run_m[c][i], sm = run_s[c][i];
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) {
-            const float m2 = __shfl_xor_sync(kFull, m, o);
-            const float s2 = __shfl_xor_sync(kFull, sm, o);
-            lse_merge(m, sm, m2, s2);
-          }
-          if (rl < cols) {
-            const size_t p = static_cast<size_t>(a.col0 + rl) * n_parts + blockIdx.x;
-            if (lane == 0) {
-              a.part_m[p] = m;
-              a.part_s[p] = sm;
-            }
-            if (lane < k) {
-              a.part_z[p * k + lane] = first ? kNegInf : lv[rl * k + lane];
-              a.part_t[p * k + lane] = first ? 0x7fffffff : lt[rl * k + lane];
-            }
-          }
+      for (int rl = ew; rl < cols; rl += kEpiWarps) {
+        const size_t p = static_cast<size_t>(a.col0 + rl) * n_parts + blockIdx.x;
+        if (lane == 0) {
+          a.part_m[p] = row_m[rl];
+          a.part_s[p] = row_s[rl];
+        }
+        if (lane < k) {
+          a.part_z[p * k + lane] = first ? kNegInf : lv[rl * k + lane];
+          a.part_t[p * k + lane] = first ? 0x7fffffff : lt[rl * k + lane];
         }
       }
     }
