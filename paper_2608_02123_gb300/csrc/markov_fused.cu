@@ -56,7 +56,10 @@ struct FusedProj {
   static constexpr int kABytes = kBM * kBK * 2;          // 16 KB
   static constexpr int kBBytes = NC * kBK * 2;           // 2..32 KB
   static constexpr int kStageBytes = kABytes + kBBytes;  // multiple of 1024
-  static constexpr int kTmemCols = 2 * NC < 32 ? 32 : 2 * NC;
+  // accumulator buffers: as many as the 512 TMEM columns hold, up to 4, so
+  // the MMAs run ahead of a slow epilogue tile
+  static constexpr int kAccBufs = 512 / NC > 4 ? 4 : 512 / NC;
+  static constexpr int kTmemCols = kAccBufs * NC < 32 ? 32 : kAccBufs * NC;
   static constexpr size_t kZBytes = static_cast<size_t>(kCC) * kBM * sizeof(float);
   // per-row running max and sum of exp, and the k-th entry of the row's
   // top-k list (the insertion threshold)
@@ -110,9 +113,9 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
   uint64_t* bars = reinterpret_cast<uint64_t*>(lt + NC * k);
   uint64_t* full = bars;                              // [kMaxStages]
   uint64_t* empty = bars + kMaxStages;                // [kMaxStages]
-  uint64_t* acc_full = bars + 2 * kMaxStages;         // [2]
-  uint64_t* acc_empty = acc_full + 2;                 // [2]
-  uint64_t* drain = acc_empty + 2;
+  uint64_t* acc_full = bars + 2 * kMaxStages;         // [kAccBufs]
+  uint64_t* acc_empty = acc_full + 4;                 // [kAccBufs]
+  uint64_t* drain = acc_empty + 4;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
   int* stop_flag = abort_flag + 1;
@@ -127,7 +130,7 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < C::kAccBufs; ++i) {
       mbar_init(&acc_full[i], 1);
       mbar_init(&acc_empty[i], kEpiWarps);   // one arrival per epilogue warp
     }
@@ -220,8 +223,10 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
         }
         if (!ok) break;
         tc_commit(&acc_full[acc]);    // accumulator ready for the epilogue
-        acc ^= 1;
-        if (acc == 0) acc_phase ^= 1u;
+        if (++acc == C::kAccBufs) {
+          acc = 0;
+          acc_phase ^= 1u;
+        }
       }
       if (!ok) {
         *abort_v = 1;
@@ -247,6 +252,25 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
       row_m[r] = kNegInf;
       row_s[r] = 0.0f;
     }
+    // The base logits a warp needs for one chunk: rows c * 64 + 8 ew + i,
+    // this lane's four vocabulary entries of `tile`.  They are loaded one
+    // chunk ahead (the next tile's first chunk during a tile's last), so the
+    // loads' latency overlaps a chunk's work.
+    auto load_l = [&](int tile, int c, float (&dst)[kRowsPerWarp][4]) {
+#pragma unroll
+      for (int i = 0; i < kRowsPerWarp; ++i) {
+        const int rl = c * kCC + ew * kRowsPerWarp + i;
+        const float* Lr = a.L + static_cast<long long>((a.col0 + (rl < cols ? rl : 0)) /
+                                                       a.rows_per_req) * a.l_req_stride;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int v = tile * kBM + lane * 4 + e;
+          dst[i][e] = (tile < n_tiles && rl < cols && v < a.V) ? __ldg(Lr + v) : 0.0f;
+        }
+      }
+    };
+    float lnx[kRowsPerWarp][4];
+    load_l(blockIdx.x, 0, lnx);
     int acc = 0;
     uint32_t acc_phase = 0;
     bool bad = false;
@@ -273,6 +297,15 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
       for (int c = 0; c < kChunks; ++c) {
         const int c0 = c * kCC;
         if (c0 >= cols) break;
+        float lcur[kRowsPerWarp][4];
+#pragma unroll
+        for (int i = 0; i < kRowsPerWarp; ++i)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) lcur[i][e] = lnx[i][e];
+        if (c0 + kCC < cols)
+          load_l(tile, c + 1, lnx);
+        else
+          load_l(tile + gridDim.x, 0, lnx);
         // A: 32 lanes x (up to) 32 columns of this warp's quadrant, transposed
         // into zs[column - c0][vocabulary row of the tile]
 #pragma unroll
@@ -310,12 +343,10 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
           }
 #pragma unroll
           for (int i = 0; i < kRowsPerWarp; ++i) {
-            const int row = a.col0 + r0 + (i < nr ? i : 0);
-            const float* Lr = a.L + static_cast<long long>(row / a.rows_per_req) * a.l_req_stride;
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
               if (i < nr && vb + e < a.V) {
-                const float lval = __ldg(Lr + vb + e);
+                const float lval = lcur[i][e];
                 // non-finite: a Markov bias that is not finite, or a NaN /
                 // +inf base logit (-inf base logits are legal)
                 bad |= !(fabsf(z[i][e]) < kPosInf) || !(lval < kPosInf);
@@ -420,12 +451,18 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
                 lst[i].reset();
               }
             }
+            // one mark word per row, so that the rows' steps do not depend
+            // on one another
+            uint32_t mr[kRowsPerWarp];
+#pragma unroll
+            for (int i = 0; i < kRowsPerWarp; ++i) mr[i] = (mk >> (4 * i)) & 15u;
             while (__any_sync(kFull, mk != 0)) {
+              mk = 0;
 #pragma unroll
               for (int i = 0; i < kRowsPerWarp; ++i) {
                 // the lowest lane with a candidate of row i offers its first
                 // one (no lane: the sentinel, which changes nothing)
-                const uint32_t mine = (mk >> (4 * i)) & 15u;
+                const uint32_t mine = mr[i];
                 const uint32_t lanes = __ballot_sync(kFull, mine != 0);
                 const int src = lanes ? __ffs(lanes) - 1 : 0;
                 const int e = mine ? __ffs(mine) - 1 : 0;
@@ -440,9 +477,11 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
                 }
                 cv = __shfl_sync(kFull, cv, src);
                 ct = __shfl_sync(kFull, ct, src);
-                if (lane == src && mine) mk &= ~(1u << (4 * i + e));
+                if (lane == src) mr[i] &= ~(1u << e);
                 lst[i].insert(cv, ct, k);
               }
+#pragma unroll
+              for (int i = 0; i < kRowsPerWarp; ++i) mk |= mr[i];
             }
 #pragma unroll
             for (int i = 0; i < kRowsPerWarp; ++i) {
@@ -460,8 +499,10 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
         epi_barrier();   // zs is rewritten by the next chunk
       }
       first = false;
-      acc ^= 1;
-      if (acc == 0) acc_phase ^= 1u;
+      if (++acc == C::kAccBufs) {
+        acc = 0;
+        acc_phase ^= 1u;
+      }
     }
     if (bad) set_status(a.status, PCTREE_ERR_NONFINITE);
     // this CTA's partial of every row of the pass
