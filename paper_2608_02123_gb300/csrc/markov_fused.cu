@@ -92,6 +92,22 @@ struct ProjArgs {
 
 __device__ __forceinline__ void epi_barrier() { named_barrier(1, kEpiThreads); }
 
+// WarpList::insert without branches (selects only), so that the inserts of
+// several independent lists interleave: lane i < k holds entry i; (cv, ct)
+// lands at its rank if that is below k, the entries after it move down one
+// and the k-th drops out.
+__device__ __forceinline__ void insert_nb(WarpList& l, float cv, int ct, int k) {
+  const int lane = threadIdx.x & 31;
+  const bool ahead = lane < k && cand_better(l.v, l.t, cv, ct);
+  const int pos = __popc(__ballot_sync(kFull, ahead));
+  const float uv = __shfl_up_sync(kFull, l.v, 1);
+  const int ut = __shfl_up_sync(kFull, l.t, 1);
+  const bool here = lane == pos;
+  const bool down = lane > pos && lane < k;
+  l.v = here ? cv : (down ? uv : l.v);
+  l.t = here ? ct : (down ? ut : l.t);
+}
+
 template <int NC>
 __global__ void __launch_bounds__(kThreads, 1)
 markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
@@ -471,14 +487,12 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
                 for (int q = 1; q < 4; ++q)
                   if (e == q) cv = z[i][q];
                 int ct = vb + e < a.V ? vb + e : 0x7fffffff;
-                if (!mine) {
-                  cv = kNegInf;
-                  ct = 0x7fffffff;
-                }
+                cv = mine ? cv : kNegInf;
+                ct = mine ? ct : 0x7fffffff;
                 cv = __shfl_sync(kFull, cv, src);
                 ct = __shfl_sync(kFull, ct, src);
-                if (lane == src) mr[i] &= ~(1u << e);
-                lst[i].insert(cv, ct, k);
+                mr[i] = lane == src ? (mr[i] & ~(1u << e)) : mr[i];
+                insert_nb(lst[i], cv, ct, k);
               }
 #pragma unroll
               for (int i = 0; i < kRowsPerWarp; ++i) mk |= mr[i];
