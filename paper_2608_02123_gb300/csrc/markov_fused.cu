@@ -92,21 +92,6 @@ struct ProjArgs {
 
 __device__ __forceinline__ void epi_barrier() { named_barrier(1, kEpiThreads); }
 
-// WarpList::insert without branches (selects only), so that the inserts of
-// several independent lists interleave: lane i < k holds entry i; (cv, ct)
-// lands at its rank if that is below k, the entries after it move down one
-// and the k-th drops out.
-__device__ __forceinline__ void insert_nb(WarpList& l, float cv, int ct, int k) {
-  const int lane = threadIdx.x & 31;
-  const bool ahead = lane < k && cand_better(l.v, l.t, cv, ct);
-  const int pos = __popc(__ballot_sync(kFull, ahead));
-  const float uv = __shfl_up_sync(kFull, l.v, 1);
-  const int ut = __shfl_up_sync(kFull, l.t, 1);
-  const bool here = lane == pos;
-  const bool down = lane > pos && lane < k;
-  l.v = here ? cv : (down ? uv : l.v);
-  l.t = here ? ct : (down ? ut : l.t);
-}
 
 template <int NC>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -434,78 +419,142 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
             }
           }
           if (first || __any_sync(kFull, mk != 0)) {
-            WarpList lst[kRowsPerWarp];
+            // The eight lists are worked on side by side: every loop below
+            // runs one operation for all eight rows before the next, so the
+            // rows' warp shuffles and votes overlap instead of queueing.
+            float sv[kRowsPerWarp];
+            int st[kRowsPerWarp];
+            if (first) {
+              // the list starts from the lanes' best logits (a warp bitonic
+              // sort); the lane's other logits that beat its k-th entry are
+              // marked
+              int best[kRowsPerWarp];
 #pragma unroll
-            for (int i = 0; i < kRowsPerWarp; ++i) {
-              if (first) {
-                // the list starts from the lanes' best logits (a sort); the
-                // lane's other logits that beat its k-th entry are marked
-                float bv = z[i][0];
-                int bt = vb < a.V ? vb : 0x7fffffff, best = 0;
+              for (int i = 0; i < kRowsPerWarp; ++i) {
+                sv[i] = z[i][0];
+                st[i] = vb < a.V ? vb : 0x7fffffff;
+                best[i] = 0;
 #pragma unroll
                 for (int e = 1; e < 4; ++e) {
                   const int te = vb + e < a.V ? vb + e : 0x7fffffff;
-                  if (cand_better(z[i][e], te, bv, bt)) {
-                    bv = z[i][e];
-                    bt = te;
-                    best = e;
+                  if (cand_better(z[i][e], te, sv[i], st[i])) {
+                    sv[i] = z[i][e];
+                    st[i] = te;
+                    best[i] = e;
                   }
                 }
-                lst[i].seed(i < nr ? bv : kNegInf, i < nr ? bt : 0x7fffffff, k);
-                const float tv = __shfl_sync(kFull, lst[i].v, k - 1);
-                const int tt = __shfl_sync(kFull, lst[i].t, k - 1);
+                if (i >= nr) {
+                  sv[i] = kNegInf;
+                  st[i] = 0x7fffffff;
+                }
+              }
+#pragma unroll
+              for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+                for (int j = size >> 1; j > 0; j >>= 1) {
+                  float ov[kRowsPerWarp];
+                  int ot[kRowsPerWarp];
+#pragma unroll
+                  for (int i = 0; i < kRowsPerWarp; ++i) ov[i] = __shfl_xor_sync(kFull, sv[i], j);
+#pragma unroll
+                  for (int i = 0; i < kRowsPerWarp; ++i) ot[i] = __shfl_xor_sync(kFull, st[i], j);
+                  const bool take_best = ((lane & j) == 0) == ((lane & size) == 0);
+#pragma unroll
+                  for (int i = 0; i < kRowsPerWarp; ++i) {
+                    const bool sw = take_best ? cand_better(ov[i], ot[i], sv[i], st[i])
+                                              : cand_better(sv[i], st[i], ov[i], ot[i]);
+                    sv[i] = sw ? ov[i] : sv[i];
+                    st[i] = sw ? ot[i] : st[i];
+                  }
+                }
+              }
+              float tv[kRowsPerWarp];
+              int tt[kRowsPerWarp];
+#pragma unroll
+              for (int i = 0; i < kRowsPerWarp; ++i) tv[i] = __shfl_sync(kFull, sv[i], k - 1);
+#pragma unroll
+              for (int i = 0; i < kRowsPerWarp; ++i) tt[i] = __shfl_sync(kFull, st[i], k - 1);
+#pragma unroll
+              for (int i = 0; i < kRowsPerWarp; ++i) {
+                if (lane >= k) {
+                  sv[i] = kNegInf;
+                  st[i] = 0x7fffffff;
+                }
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
                   const int te = vb + e < a.V ? vb + e : 0x7fffffff;
-                  if (i < nr && e != best && cand_better(z[i][e], te, tv, tt))
+                  if (i < nr && e != best[i] && cand_better(z[i][e], te, tv[i], tt[i]))
                     mk |= 1u << (4 * i + e);
                 }
-              } else if (i < nr && lane < k) {
-                lst[i].v = lv[(r0 + i) * k + lane];
-                lst[i].t = lt[(r0 + i) * k + lane];
-              } else {
-                lst[i].reset();
+              }
+            } else {
+#pragma unroll
+              for (int i = 0; i < kRowsPerWarp; ++i) {
+                const bool has = i < nr && lane < k;
+                sv[i] = has ? lv[(r0 + i) * k + lane] : kNegInf;
+                st[i] = has ? lt[(r0 + i) * k + lane] : 0x7fffffff;
               }
             }
-            // one mark word per row, so that the rows' steps do not depend
-            // on one another
+            // Candidates go in one per row per step: the lowest lane with a
+            // candidate of row i offers its first one (no lane: the sentinel,
+            // which changes nothing).  An insert places (cv, ct) at its rank
+            // below k, moves the later entries down one and drops the k-th.
+            // One mark word per row keeps the rows independent.
             uint32_t mr[kRowsPerWarp];
 #pragma unroll
             for (int i = 0; i < kRowsPerWarp; ++i) mr[i] = (mk >> (4 * i)) & 15u;
             while (__any_sync(kFull, mk != 0)) {
+              uint32_t lanes[kRowsPerWarp];
+              float cv[kRowsPerWarp];
+              int ct[kRowsPerWarp], src[kRowsPerWarp], ee[kRowsPerWarp];
+#pragma unroll
+              for (int i = 0; i < kRowsPerWarp; ++i) lanes[i] = __ballot_sync(kFull, mr[i] != 0);
+#pragma unroll
+              for (int i = 0; i < kRowsPerWarp; ++i) {
+                src[i] = lanes[i] ? __ffs(lanes[i]) - 1 : 0;
+                ee[i] = mr[i] ? __ffs(mr[i]) - 1 : 0;
+                // z[i][ee[i]] by two bit selects (an indexed read would put
+                // z in local memory)
+                const float c01 = (ee[i] & 1) ? z[i][1] : z[i][0];
+                const float c23 = (ee[i] & 1) ? z[i][3] : z[i][2];
+                cv[i] = mr[i] ? ((ee[i] & 2) ? c23 : c01) : kNegInf;
+                ct[i] = mr[i] && vb + ee[i] < a.V ? vb + ee[i] : 0x7fffffff;
+              }
+#pragma unroll
+              for (int i = 0; i < kRowsPerWarp; ++i) cv[i] = __shfl_sync(kFull, cv[i], src[i]);
+#pragma unroll
+              for (int i = 0; i < kRowsPerWarp; ++i) ct[i] = __shfl_sync(kFull, ct[i], src[i]);
+              int pos[kRowsPerWarp];
+#pragma unroll
+              for (int i = 0; i < kRowsPerWarp; ++i) {
+                mr[i] = lane == src[i] ? (mr[i] & ~(1u << ee[i])) : mr[i];
+                pos[i] = __popc(__ballot_sync(kFull, lane < k && cand_better(sv[i], st[i], cv[i], ct[i])));
+              }
+              float uv[kRowsPerWarp];
+              int ut[kRowsPerWarp];
+#pragma unroll
+              for (int i = 0; i < kRowsPerWarp; ++i) uv[i] = __shfl_up_sync(kFull, sv[i], 1);
+#pragma unroll
+              for (int i = 0; i < kRowsPerWarp; ++i) ut[i] = __shfl_up_sync(kFull, st[i], 1);
               mk = 0;
 #pragma unroll
               for (int i = 0; i < kRowsPerWarp; ++i) {
-                // the lowest lane with a candidate of row i offers its first
-                // one (no lane: the sentinel, which changes nothing)
-                const uint32_t mine = mr[i];
-                const uint32_t lanes = __ballot_sync(kFull, mine != 0);
-                const int src = lanes ? __ffs(lanes) - 1 : 0;
-                const int e = mine ? __ffs(mine) - 1 : 0;
-                float cv = z[i][0];
-#pragma unroll
-                for (int q = 1; q < 4; ++q)
-                  if (e == q) cv = z[i][q];
-                int ct = vb + e < a.V ? vb + e : 0x7fffffff;
-                cv = mine ? cv : kNegInf;
-                ct = mine ? ct : 0x7fffffff;
-                cv = __shfl_sync(kFull, cv, src);
-                ct = __shfl_sync(kFull, ct, src);
-                mr[i] = lane == src ? (mr[i] & ~(1u << e)) : mr[i];
-                insert_nb(lst[i], cv, ct, k);
+                const bool here = lane == pos[i];
+                const bool down = lane > pos[i] && lane < k;
+                sv[i] = here ? cv[i] : (down ? uv[i] : sv[i]);
+                st[i] = here ? ct[i] : (down ? ut[i] : st[i]);
+                mk |= mr[i];
               }
-#pragma unroll
-              for (int i = 0; i < kRowsPerWarp; ++i) mk |= mr[i];
             }
 #pragma unroll
             for (int i = 0; i < kRowsPerWarp; ++i) {
               if (i < nr) {
                 const int rl = r0 + i;
                 if (lane < k) {
-                  lv[rl * k + lane] = lst[i].v;
-                  lt[rl * k + lane] = lst[i].t;
+                  lv[rl * k + lane] = sv[i];
+                  lt[rl * k + lane] = st[i];
                 }
-                if (lane == k - 1) thr_v[rl] = lst[i].v;
+                if (lane == k - 1) thr_v[rl] = sv[i];
               }
             }
           }
