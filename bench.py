@@ -70,6 +70,10 @@ def parse_args():
                     choices=sorted(COMPACT_WORKLOADS))
     ap.add_argument("--attn-workload", default="14b_b16_bs32",
                     choices=sorted(ATTN_WORKLOADS))
+    ap.add_argument("--head-layout", default="tiled", choices=["tiled", "rowmajor"],
+                    help="storage of W_out: tiled (repacked once at load with "
+                         "pctree_pack_head, outside the timed region) or the "
+                         "row-major [V][H] matrix")
     ap.add_argument("--path", default="auto", choices=["auto", "stagewise"],
                     help="kernel path: fused round where it applies, or the "
                          "per-stage kernels for every round")
@@ -410,8 +414,13 @@ def run_ours(args, wl, rank, world, local_rank):
     root_dev = [torch.from_numpy(root).to(dev) for _, root, _ in sets]
     greedy_dev = [torch.from_numpy(g.astype(np.int64)).to(dev)
                   for _, _, g in sets]
+    layout = args.head_layout if wl.weight_dtype == "bf16" else "rowmajor"
     cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, wl.batch, wl.pos_offset,
-                        wl.weight_dtype, wl.mode)
+                        wl.weight_dtype, wl.mode, layout)
+    if layout == "tiled":
+        # the weights are fixed: repacked once, as a serving process does at load
+        W = P.pack_head(cfg, W)
+        torch.cuda.synchronize()
     path = P.PATH_AUTO if args.path == "auto" else P.PATH_STAGEWISE
     P.pctree_set_path(path)
     fused = P.uses_fused_round(cfg, path)
@@ -540,6 +549,9 @@ def run_ours(args, wl, rank, world, local_rank):
                    "k": wl.k, "N": wl.N, "batch": wl.batch,
                    "parallelism": f"replicas x{world}",
                    "kernel_path": args.path, "mode": wl.mode,
+                   "head_layout": (f"{layout} (W_out repacked once at load by "
+                                   "pctree_pack_head, outside the timed region)"
+                                   if layout == "tiled" else layout),
                    "l2": f"inputs larger than L2: W_out "
                          f"({wl.V * wl.H * (2 if wl.weight_dtype == 'bf16' else 4) / 1e6:.0f} MB) "
                          f"streamed per stage; base logits rotate over "
@@ -570,7 +582,7 @@ def run_ours(args, wl, rank, world, local_rank):
         "clocks": clk,
     }
     if world == 1 and not args.no_batched and args.workload == "4b_b16":
-        line["batched"] = measure_batched(dev, gpu_index)
+        line["batched"] = measure_batched(dev, gpu_index, layout)
     if world == 1 and not args.no_cpu_baseline:
         runner = OracleRunner(wl, E_host, W_host,
                               [(L[0], int(root[0])) for L, root, _ in sets])
@@ -594,7 +606,7 @@ def round_flops(wl):
     return 2.0 * wl.H * wl.V * rows
 
 
-def measure_batched(dev, gpu_index, steps=10, warmup=3):
+def measure_batched(dev, gpu_index, layout, steps=10, warmup=3):
     """Each batched workload: W + K whole rounds (inputs resident, base
     logits rotating over sets that together exceed 3 x L2), CUDA events on
     the launching stream, clocks sampled meanwhile.  The roofline is HBM
@@ -625,7 +637,10 @@ def measure_batched(dev, gpu_index, steps=10, warmup=3):
             L_dev.append(torch.from_numpy(np.stack([q[0] for q in reqs])).to(dev))
             root_dev.append(torch.tensor([q[1] for q in reqs], dtype=torch.int32,
                                          device=dev))
-        cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, wl.batch)
+        cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, wl.batch, 0, "bf16",
+                            "parent", layout)
+        if layout == "tiled":
+            W = P.pack_head(cfg, W)
         dr = P.Drafter(cfg, dev)
         for i in range(warmup):
             dr.draft(L_dev[i % n_sets], E, W, root_dev[i % n_sets], stream)
@@ -649,6 +664,7 @@ def measure_batched(dev, gpu_index, steps=10, warmup=3):
         bound = "hbm" if t_hbm >= t_tc else "tensor"
         out.append({
             "workload": wl.name, "batch": wl.batch, "steps": steps,
+            "head_layout": layout,
             "warmup": warmup, "us_per_round": us,
             "rounds_per_s": 1e6 / us, "request_rounds_per_s": wl.batch * 1e6 / us,
             "bound": bound, "roofline_us": max(t_hbm, t_tc),

@@ -69,6 +69,19 @@ typedef enum { PCTREE_F32 = 0, PCTREE_BF16 = 1 } pctree_dtype;
  * k = 1 with either mode is DSpark's single chain (Sec. 4.2). */
 typedef enum { PCTREE_MODE_PARENT = 0, PCTREE_MODE_SHARED = 1 } pctree_mode;
 
+/* Storage of the Markov-head output projection W_out (bf16 heads).
+ *   PCTREE_HEAD_ROWMAJOR  [V][H], row-major, as trained.
+ *   PCTREE_HEAD_TILED     the same values in vocabulary tiles: an array
+ *                         [ceil(V/128)][ceil(H/64)][128][64] whose block
+ *                         (t, c) holds rows 128 t .. 128 t + 127 and columns
+ *                         64 c .. 64 c + 63 of W_out, row-major within the
+ *                         block, zero where a row >= V or a column >= H.
+ *                         Every 16 KB block the round streams is then one
+ *                         contiguous piece of memory.  pctree_pack_head makes
+ *                         it once from the row-major matrix (the weights are
+ *                         fixed, so a serving process packs them at load). */
+typedef enum { PCTREE_HEAD_ROWMAJOR = 0, PCTREE_HEAD_TILED = 1 } pctree_head_layout;
+
 /* Compiled limits. */
 #define PCTREE_MAX_K 32        /* per-parent top-k and frontier width        */
 #define PCTREE_MAX_N 1024      /* node budget, root included                 */
@@ -92,11 +105,13 @@ typedef enum { PCTREE_MODE_PARENT = 0, PCTREE_MODE_SHARED = 1 } pctree_mode;
  *                (Appendix A).
  *   weight_dtype storage type of both head matrices (pctree_dtype).
  *   mode         child scoring (pctree_mode).
+ *   head_layout  storage of head_out (pctree_head_layout); TILED needs
+ *                BF16 weights.  E_in is always row-major.
  * The candidate pool holds 1 + k + (B-1) k^2 nodes (Sec. 4.1); it must not
  * exceed PCTREE_MAX_POOL.
  */
 typedef struct {
-  int32_t V, H, B, k, N, batch, pos_offset, weight_dtype, mode;
+  int32_t V, H, B, k, N, batch, pos_offset, weight_dtype, mode, head_layout;
 } pctree_config;
 
 /*
@@ -166,8 +181,9 @@ PCTREE_API size_t pctree_workspace_bytes(const pctree_config* cfg);
  *                request (Sec. 3.2 "Parallel backbone"); -inf allowed.
  *   head_emb     [V][H] E_in  (weight_dtype), 16-byte aligned: Markov-head
  *                input rows, one per parent token.
- *   head_out     [V][H] W_out (weight_dtype), 16-byte aligned: Markov-head
- *                output projection.  The head's bias for parent p is
+ *   head_out     W_out (weight_dtype), 16-byte aligned, [V][H] or tiled as
+ *                cfg->head_layout says: Markov-head output projection.
+ *                The head's bias for parent p is
  *                Markov(p)[v] = sum_h W_out[v][h] * E_in[p][h] (Sec. 3.2,
  *                "low-rank Markov head"), accumulated in float32.
  *   root_token   [batch] int32: the last verified token x_t of each request;
@@ -220,6 +236,24 @@ PCTREE_API pctree_status pctree_draft_noalloc(const pctree_config* cfg,
                                               const int32_t* root_token,
                                               const pctree_tree* out,
                                               void* stream);
+
+/* Bytes of head_out in the PCTREE_HEAD_TILED layout for cfg's V and H:
+ * ceil(V/128) * ceil(H/64) * 128 * 64 * 2; 0 for a bad config or F32
+ * weights. */
+PCTREE_API size_t pctree_packed_head_bytes(const pctree_config* cfg);
+
+/*
+ * A storage transform with no counterpart in the paper (the head's values
+ * are unchanged).  Repacks a row-major bf16 W_out [V][H] (16-byte aligned)
+ * into the
+ * PCTREE_HEAD_TILED layout in `packed` (pctree_packed_head_bytes(cfg) bytes,
+ * 16-byte aligned, not overlapping head_out); padding is written as zeros.
+ * cfg->head_layout is ignored.  Stream-ordered; reads and writes each byte
+ * once.  Returns PCTREE_ERR_INVALID_ARG for F32 weights, NULL or misaligned
+ * pointers, PCTREE_ERR_CUDA if the launch fails.
+ */
+PCTREE_API pctree_status pctree_pack_head(const pctree_config* cfg, const void* head_out,
+                                          void* packed, void* stream);
 
 /*
  * Greedy tree acceptance (Sec. 4.2 "standard greedy tree rule"; Appendix A).

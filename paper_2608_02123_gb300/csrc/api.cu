@@ -31,6 +31,10 @@ pctree_status check_config(const pctree_config* c) {
     return PCTREE_ERR_INVALID_ARG;
   if (c->mode != PCTREE_MODE_PARENT && c->mode != PCTREE_MODE_SHARED)
     return PCTREE_ERR_INVALID_ARG;
+  if (c->head_layout != PCTREE_HEAD_ROWMAJOR && c->head_layout != PCTREE_HEAD_TILED)
+    return PCTREE_ERR_INVALID_ARG;
+  if (c->head_layout == PCTREE_HEAD_TILED && c->weight_dtype != PCTREE_BF16)
+    return PCTREE_ERR_INVALID_ARG;
   if (c->weight_dtype == PCTREE_BF16 && (c->H % 8) != 0)
     return PCTREE_ERR_INVALID_ARG;
   if (c->k > PCTREE_MAX_K || c->N > PCTREE_MAX_N) return PCTREE_ERR_UNSUPPORTED;
@@ -165,6 +169,21 @@ namespace {
 // 2-D bf16 tensor [rows][cols] (cols contiguous), box = box_rows x 64 with
 // the 128-byte swizzle the MMA descriptors expect.
 pctree_status encode_bf16_map(CUtensorMap* map, const void* base, int rows,
+                              int cols, int box_rows);
+
+// W_out's tensor map: [V][H] boxes of 128 x 64, or the tiled layout as a
+// [n_tiles * n_k * 128][64] matrix whose 128 x 64 boxes are contiguous.
+pctree_status encode_head_map(CUtensorMap* map, const void* head_out,
+                              const pctree_config& c) {
+  if (c.head_layout == PCTREE_HEAD_TILED) {
+    const long long rows = static_cast<long long>((c.V + 127) / 128) *
+                           ((c.H + 63) / 64) * 128;
+    if (rows > (1ll << 31) - 1) return PCTREE_ERR_UNSUPPORTED;
+    return encode_bf16_map(map, head_out, static_cast<int>(rows), 64, 128);
+  }
+  return encode_bf16_map(map, head_out, c.V, c.H, 128);
+}
+pctree_status encode_bf16_map(CUtensorMap* map, const void* base, int rows,
                               int cols, int box_rows) {
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols),
                         static_cast<cuuint64_t>(rows)};
@@ -218,7 +237,7 @@ pctree_status draft_fused(const pctree_config& c, const Layout& lay,
                           const pctree_tree& out, unsigned char* ws,
                           int num_sms, cudaStream_t stream) {
   CUtensorMap tmap_w, tmap_x;
-  pctree_status st = encode_bf16_map(&tmap_w, head_out, c.V, c.H, 128);
+  pctree_status st = encode_head_map(&tmap_w, head_out, c);
   if (st != PCTREE_OK) return st;
   st = encode_bf16_map(&tmap_x, ws + lay.off_x, kFusedRows, c.H, kFusedRows);
   if (st != PCTREE_OK) return st;
@@ -233,6 +252,7 @@ pctree_status draft_fused(const pctree_config& c, const Layout& lay,
   a.k = c.k;
   a.batch = c.batch;
   a.shared = c.mode == PCTREE_MODE_SHARED ? 1 : 0;
+  a.tiled = c.head_layout == PCTREE_HEAD_TILED ? 1 : 0;
   a.P = lay.P;
   a.n_k = (c.H + 63) / 64;
   a.n_tiles = n_tiles;
@@ -276,7 +296,7 @@ using namespace pct;
 
 extern "C" {
 
-int32_t pctree_version(void) { return 101; }
+int32_t pctree_version(void) { return 102; }
 
 const char* pctree_status_string(int32_t s) {
   switch (s) {
@@ -344,7 +364,7 @@ pctree_status pctree_draft(const pctree_config* cfg, const float* base_logits,
                                         root_token, *out, ws, num_sms, stream);
   CUtensorMap tmap_w, tmap_x;
   if (c.weight_dtype == PCTREE_BF16) {
-    st = encode_bf16_map(&tmap_w, head_out, c.V, c.H, 128);
+    st = encode_head_map(&tmap_w, head_out, c);
     if (st != PCTREE_OK) return st;
     st = encode_bf16_map(&tmap_x, ws + lay.off_x, lay.rows_pad, c.H, lay.bn);
     if (st != PCTREE_OK) return st;
@@ -373,7 +393,8 @@ pctree_status pctree_draft(const pctree_config* cfg, const float* base_logits,
       // projection, normaliser and top-k partials in one pass over W_out
       n_parts = fused_proj_parts(c.V, num_sms);
       e = launch_markov_fused(&tmap_w, &tmap_x, L_d, l_req_stride, c.V, c.H, c.k,
-                              rows, rpq, lay.bn, num_sms,
+                              rows, rpq, lay.bn, c.head_layout == PCTREE_HEAD_TILED,
+                              num_sms,
                               reinterpret_cast<float*>(ws + lay.off_pm),
                               reinterpret_cast<float*>(ws + lay.off_ps),
                               reinterpret_cast<float*>(ws + lay.off_pz),
@@ -394,6 +415,26 @@ pctree_status pctree_draft(const pctree_config* cfg, const float* base_logits,
     if (st != PCTREE_OK) return st;
   }
   return cuda_status(launch_pack(c, lay, ws, *out, stream));
+}
+
+size_t pctree_packed_head_bytes(const pctree_config* cfg) {
+  if (check_config(cfg) != PCTREE_OK || cfg->weight_dtype != PCTREE_BF16) return 0;
+  return packed_head_bytes(cfg->V, cfg->H);
+}
+
+pctree_status pctree_pack_head(const pctree_config* cfg, const void* head_out,
+                               void* packed, void* stream) {
+  NvtxRange range("pctree_pack_head");
+  pctree_status st = check_config(cfg);
+  if (st != PCTREE_OK) return st;
+  if (cfg->weight_dtype != PCTREE_BF16 || head_out == nullptr || packed == nullptr ||
+      !aligned(head_out, 16) || !aligned(packed, 16))
+    return PCTREE_ERR_INVALID_ARG;
+  int num_sms = 0;
+  st = device_facts(&num_sms);
+  if (st != PCTREE_OK) return st;
+  return cuda_status(launch_pack_head(head_out, packed, cfg->V, cfg->H, num_sms,
+                                      static_cast<cudaStream_t>(stream)));
 }
 
 pctree_status pctree_accept(const pctree_config* cfg, const pctree_tree* tree,

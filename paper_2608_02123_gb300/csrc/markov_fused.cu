@@ -83,6 +83,7 @@ struct ProjArgs {
   const float* L;          // base logits of depth d, request 0
   long long l_req_stride;  // floats between two requests' rows
   int V, H, k, rows, rows_per_req, col0, n_stages;
+  int tiled;               // 1: W_out in the tiled layout (PCTREE_HEAD_TILED)
   float* part_m;           // [rows][n_parts] per-CTA max
   float* part_s;           // [rows][n_parts] per-CTA sum of exp
   float* part_z;           // [rows][n_parts][k] per-CTA top-k logits, best first
@@ -165,9 +166,10 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
             break;
           }
           unsigned char* a_dst = ring + stage * C::kStageBytes;
+          int wx, wy;
+          w_box(a.tiled, tile, kc, n_k, wx, wy);
           mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
-          tma_load_2d_hint(a_dst, &tmap_w, &full[stage], kc * kBK, tile * kBM,
-                           stream_policy);
+          tma_load_2d_hint(a_dst, &tmap_w, &full[stage], wx, wy, stream_policy);
           tma_load_2d(a_dst + C::kABytes, &tmap_x, &full[stage], kc * kBK, a.col0);
           armed |= 1u << stage;
           armed_phase = (armed_phase & ~(1u << stage)) | (phase << stage);
@@ -625,7 +627,7 @@ int fused_proj_parts(int V, int num_sms) {
 
 cudaError_t launch_markov_fused(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
                                 const float* L, long long l_req_stride, int V,
-                                int H, int k, int rows, int rows_per_req, int bn,
+                                int H, int k, int rows, int rows_per_req, int bn, int tiled,
                                 int num_sms, float* part_m, float* part_s,
                                 float* part_z, int32_t* part_t, int32_t* status,
                                 cudaStream_t stream) {
@@ -637,6 +639,7 @@ cudaError_t launch_markov_fused(const CUtensorMap* tmap_w, const CUtensorMap* tm
   a.k = k;
   a.rows = rows;
   a.rows_per_req = rows_per_req;
+  a.tiled = tiled;
   a.part_m = part_m;
   a.part_s = part_s;
   a.part_z = part_z;

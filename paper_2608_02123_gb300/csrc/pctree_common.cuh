@@ -49,6 +49,7 @@ struct FusedArgs {
   const float* L;        // [batch][B][V] base logits
   int V, H, B, k, batch, P, n_k, n_tiles;
   int shared;            // 1: Shared-Markov control (one chain row per request)
+  int tiled;             // 1: W_out in the tiled layout (PCTREE_HEAD_TILED)
   int32_t* pool_tok;     // [batch][P]
   int32_t* pool_par;     // [batch][P]
   float2* pool_s;        // [batch][P] joint score as (hi, lo)
@@ -304,9 +305,23 @@ pctree_status encode_bf16_map_nd(CUtensorMap* map, const void* base, int rank,
 // fused_proj_parts(V, num_sms).  `L` points at depth d of request 0.
 int fused_proj_parts(int V, int num_sms);
 
+// Coordinates of the W_out box of (vocabulary tile, K chunk) in the tensor
+// map: row-major [V][H] (x = 64 kc, y = 128 tile), or the tiled layout seen
+// as a [n_tiles * n_k * 128][64] matrix (x = 0, y = 128 (tile * n_k + kc)).
+__device__ __forceinline__ void w_box(int tiled, int tile, int kc, int n_k,
+                                      int& x, int& y) {
+  x = tiled ? 0 : kc * 64;
+  y = tiled ? (tile * n_k + kc) * 128 : tile * 128;
+}
+
+// Tiled-layout bytes for V x H (pack_head.cu) and the repacking launch.
+size_t packed_head_bytes(int V, int H);
+cudaError_t launch_pack_head(const void* W, void* packed, int V, int H, int num_sms,
+                             cudaStream_t stream);
+
 cudaError_t launch_markov_fused(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
                                 const float* L, long long l_req_stride, int V,
-                                int H, int k, int rows, int rows_per_req, int bn,
+                                int H, int k, int rows, int rows_per_req, int bn, int tiled,
                                 int num_sms, float* part_m, float* part_s,
                                 float* part_z, int32_t* part_t, int32_t* status,
                                 cudaStream_t stream);

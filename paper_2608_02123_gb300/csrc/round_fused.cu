@@ -176,9 +176,11 @@ __device__ void produce(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
           break;
         }
         const int kx = chunk_at(d, kc, c0, c1);
+        int wx, wy;
+        w_box(a.tiled, tile, kx, a.n_k, wx, wy);
         mbar_arrive_expect_tx(&S->full[stage], tx);
-        tma_load_2d_hint(ring + stage * kStageBytes, tmap_w, &S->full[stage],
-                         kx * kBK, tile * kBM, stream_policy);
+        tma_load_2d_hint(ring + stage * kStageBytes, tmap_w, &S->full[stage], wx, wy,
+                         stream_policy);
         if (have) {
           issue_rows(stage, kx);
         } else {

@@ -38,7 +38,8 @@ class Config(ctypes.Structure):
                 ("B", ctypes.c_int32), ("k", ctypes.c_int32),
                 ("N", ctypes.c_int32), ("batch", ctypes.c_int32),
                 ("pos_offset", ctypes.c_int32),
-                ("weight_dtype", ctypes.c_int32), ("mode", ctypes.c_int32)]
+                ("weight_dtype", ctypes.c_int32), ("mode", ctypes.c_int32),
+                ("head_layout", ctypes.c_int32)]
 
 
 class CompactLayout(ctypes.Structure):
@@ -87,6 +88,10 @@ def _load() -> ctypes.CDLL:
     lib.pctree_draft_noalloc.argtypes = [cfgp, vp, vp, vp, vp,
                                          ctypes.POINTER(_Tree), vp]
     lib.pctree_draft_noalloc.restype = ctypes.c_int
+    lib.pctree_packed_head_bytes.argtypes = [cfgp]
+    lib.pctree_packed_head_bytes.restype = ctypes.c_size_t
+    lib.pctree_pack_head.argtypes = [cfgp, vp, vp, vp]
+    lib.pctree_pack_head.restype = ctypes.c_int
     lib.pctree_accept.argtypes = [cfgp, ctypes.POINTER(_Tree), vp, vp, vp, vp,
                                   vp]
     lib.pctree_accept.restype = ctypes.c_int
@@ -120,15 +125,46 @@ LIB_PATH = _LIB_PATH
 
 
 MODE_PARENT, MODE_SHARED = 0, 1
+HEAD_ROWMAJOR, HEAD_TILED = 0, 1
 
 
 def make_config(V: int, H: int, B: int, k: int, N: int, batch: int = 1,
                 pos_offset: int = 0, weight_dtype: str = "bf16",
-                mode: str = "parent") -> Config:
-    """``mode``: "parent" (PCTree) or "shared" (the Shared-Markov control)."""
+                mode: str = "parent", head_layout: str = "rowmajor") -> Config:
+    """``mode``: "parent" (PCTree) or "shared" (the Shared-Markov control).
+    ``head_layout``: "rowmajor" ([V][H]) or "tiled" (see pctree_pack_head)."""
     return Config(V, H, B, k, N, batch, pos_offset,
                   PCTREE_BF16 if weight_dtype == "bf16" else PCTREE_F32,
-                  MODE_SHARED if mode == "shared" else MODE_PARENT)
+                  MODE_SHARED if mode == "shared" else MODE_PARENT,
+                  HEAD_TILED if head_layout == "tiled" else HEAD_ROWMAJOR)
+
+
+def pctree_packed_head_bytes(cfg: Config) -> int:
+    return LIB.pctree_packed_head_bytes(ctypes.byref(cfg))
+
+
+def pctree_pack_head(cfg: Config, head_out: torch.Tensor, packed: torch.Tensor,
+                     stream: Optional[torch.cuda.Stream] = None) -> None:
+    """Enqueue the repacking of a row-major bf16 W_out into the tiled layout
+    (see pctree_pack_head in include/pctree.h)."""
+    if not head_out.is_cuda or not head_out.is_contiguous() or not packed.is_cuda:
+        raise ValueError("head_out and packed must be CUDA tensors (head_out contiguous)")
+    if packed.numel() * packed.element_size() < pctree_packed_head_bytes(cfg):
+        raise ValueError("packed is smaller than pctree_packed_head_bytes")
+    rc = LIB.pctree_pack_head(ctypes.byref(cfg), head_out.data_ptr(),
+                              packed.data_ptr(), _stream_ptr(stream))
+    if rc != PCTREE_OK:
+        raise PctreeError(rc, "pctree_pack_head")
+
+
+def pack_head(cfg: Config, head_out: torch.Tensor) -> torch.Tensor:
+    """A new device tensor holding head_out in the tiled layout."""
+    nbytes = pctree_packed_head_bytes(cfg)
+    if nbytes == 0:
+        raise PctreeError(-1, "pctree_packed_head_bytes")
+    packed = torch.empty(nbytes // 2, dtype=torch.bfloat16, device=head_out.device)
+    pctree_pack_head(cfg, head_out, packed)
+    return packed
 
 
 def pctree_check_config(cfg: Config) -> int:

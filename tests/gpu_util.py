@@ -106,15 +106,20 @@ def canary_drafter(P, cfg, with_pool: bool):
 
 
 def run_gpu(inp: RoundInputs, with_pool=True, accept=True,
-            path: int = 0) -> Dict[str, np.ndarray]:
+            path: int = 0, tiled: bool = False) -> Dict[str, np.ndarray]:
     """One round through the C ABI; ``path`` 0 = automatic (fused round
-    kernel where it applies), 1 = per-stage kernels.  Every output tensor
-    and the workspace are canary-padded and checked afterwards."""
+    kernel where it applies), 1 = per-stage kernels; ``tiled``: W_out
+    repacked by pctree_pack_head and drafted in the tiled layout.  Every
+    output tensor and the workspace are canary-padded and checked
+    afterwards."""
     from paper_2608_02123_gb300 import pctree as P
     wl = inp.wl
     cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, inp.L.shape[0],
-                        wl.pos_offset, wl.weight_dtype, wl.mode)
+                        wl.pos_offset, wl.weight_dtype, wl.mode,
+                        "tiled" if tiled else "rowmajor")
     L, E, W, root = device_inputs(inp)
+    if tiled:
+        W = P.pack_head(cfg, W)
     dr, canaries = canary_drafter(P, cfg, with_pool)
     P.pctree_set_path(path)
     try:

@@ -143,3 +143,15 @@ def test_batch1_qwen3_rounds_fit_the_noalloc_array(P):
                           (151936, 4096, 7, 8, 64), (151936, 5120, 16, 16, 128)):
         ws = P.pctree_workspace_bytes(P.make_config(V, H, B, k, N, 1))
         assert 0 < ws <= limit, (V, H, B, k, N, ws)
+
+
+def test_tiled_head_layout_config(P):
+    mk = P.make_config
+    assert P.pctree_check_config(mk(151936, 2560, 16, 8, 64, 1, 0, "bf16", "parent", "tiled")) == 0
+    assert P.pctree_check_config(mk(1024, 64, 4, 4, 8, 1, 0, "f32", "parent", "tiled")) == -1
+    bad = mk(1024, 64, 4, 4, 8)
+    bad.head_layout = 7
+    assert P.pctree_check_config(bad) == -1
+    # ceil(V/128) * ceil(H/64) blocks of 128 x 64 bf16
+    assert P.pctree_packed_head_bytes(mk(151936, 2560, 16, 8, 64)) == 1187 * 40 * 128 * 64 * 2
+    assert P.pctree_packed_head_bytes(mk(3000, 72, 2, 2, 4)) == 24 * 2 * 128 * 64 * 2
