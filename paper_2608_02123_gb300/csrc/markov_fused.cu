@@ -43,6 +43,7 @@ constexpr int kEpiThreads = 32 * kEpiWarps;
 constexpr int kThreads = 64 + kEpiThreads;
 constexpr int kCC = 64;           // accumulator columns per transpose chunk
 constexpr int kRowsPerWarp = kCC / kEpiWarps;
+constexpr int kCand = 16;         // compacted candidates per row and round
 constexpr int kMaxStages = 8;
 constexpr int kSmemLimit = 227 * 1024;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per bounded wait
@@ -65,9 +66,12 @@ struct FusedProj {
   // top-k list (the insertion threshold)
   static constexpr size_t kRowBytes = static_cast<size_t>(NC) * 12;
   static constexpr size_t kBarBytes = 256;
+  // per epilogue warp, per row of a chunk: kCand compacted candidates
+  static constexpr size_t kCandBytes = static_cast<size_t>(kEpiWarps) * kRowsPerWarp * kCand * 8;
   static size_t list_bytes(int k) { return static_cast<size_t>(NC) * k * 8; }
   static size_t fixed_bytes(int k) {
-    return 1024 /*alignment slack*/ + kZBytes + kRowBytes + list_bytes(k) + kBarBytes;
+    return 1024 /*alignment slack*/ + kZBytes + kRowBytes + list_bytes(k) + kCandBytes +
+           kBarBytes;
   }
   static int stages(int k) {
     const long long room = kSmemLimit - static_cast<long long>(fixed_bytes(k));
@@ -112,7 +116,9 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
   float* thr_v = row_s + NC;                          // the list's k-th entry
   float* lv = thr_v + NC;                             // [NC][k]
   int* lt = reinterpret_cast<int*>(lv + NC * k);      // [NC][k]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(lt + NC * k);
+  float* cbv = reinterpret_cast<float*>(lt + NC * k);  // [warp][row][kCand]
+  int* cbt = reinterpret_cast<int*>(cbv + kEpiWarps * kRowsPerWarp * kCand);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(cbt + kEpiWarps * kRowsPerWarp * kCand);
   uint64_t* full = bars;                              // [kMaxStages]
   uint64_t* empty = bars + kMaxStages;                // [kMaxStages]
   uint64_t* acc_full = bars + 2 * kMaxStages;         // [kAccBufs]
@@ -416,11 +422,67 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
                 const float tv = thr_v[r0 + i];
 #pragma unroll
                 for (int e = 0; e < 4; ++e)
-                  if (z[i][e] >= tv) mk |= 1u << (4 * i + e);
+                  if (z[i][e] >= tv && vb + e < a.V) mk |= 1u << (4 * i + e);
               }
             }
           }
-          if (first || __any_sync(kFull, mk != 0)) {
+          if (!first && __any_sync(kFull, mk != 0)) {
+            // Later tiles: few candidates, so one lane per row inserts them
+            // into the row's list in shared memory.  Each round compacts up
+            // to kCand candidates per row (ballots, in (entry, lane) order)
+            // into this warp's buffer; lane i then walks row i's candidates.
+            float* cv_w = cbv + ew * kRowsPerWarp * kCand;
+            int* ct_w = cbt + ew * kRowsPerWarp * kCand;
+            const unsigned below = (1u << lane) - 1u;
+            while (__any_sync(kFull, mk != 0)) {
+              int n_mine = 0;
+#pragma unroll
+              for (int i = 0; i < kRowsPerWarp; ++i) {
+                int base = 0;
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                  const bool m = (mk >> (4 * i + e)) & 1u;
+                  const unsigned b = __ballot_sync(kFull, m);
+                  const int slot = base + __popc(b & below);
+                  if (m && slot < kCand) {
+                    cv_w[i * kCand + slot] = z[i][e];
+                    ct_w[i * kCand + slot] = vb + e;
+                    mk &= ~(1u << (4 * i + e));
+                  }
+                  base += __popc(b);
+                }
+                if (lane == i) n_mine = base < kCand ? base : kCand;
+              }
+              __syncwarp();
+              if (lane < nr) {
+                const int rl = r0 + lane;
+                float* Lv = lv + rl * k;
+                int* Lt = lt + rl * k;
+                float kv = Lv[k - 1];
+                int kt = Lt[k - 1];
+                for (int c = 0; c < n_mine; ++c) {
+                  const float v = cv_w[lane * kCand + c];
+                  const int t = ct_w[lane * kCand + c];
+                  if (!cand_better(v, t, kv, kt)) continue;
+                  int j = k - 1;
+                  while (j > 0) {
+                    const float pv = Lv[j - 1];
+                    const int pt = Lt[j - 1];
+                    if (!cand_better(v, t, pv, pt)) break;
+                    Lv[j] = pv;
+                    Lt[j] = pt;
+                    --j;
+                  }
+                  Lv[j] = v;
+                  Lt[j] = t;
+                  kv = Lv[k - 1];
+                  kt = Lt[k - 1];
+                }
+                thr_v[rl] = kv;
+              }
+              __syncwarp();
+            }
+          } else if (first) {
             // The eight lists are worked on side by side: every loop below
             // runs one operation for all eight rows before the next, so the
             // rows' warp shuffles and votes overlap instead of queueing.
