@@ -407,15 +407,81 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
               row_s[r0 + lane] = sm;
             }
           }
-          // top-k of each row over this CTA's tiles.  Bits 4i..4i+3 of `mk`
-          // mark this lane's logits of row i that are candidates: at or above
-          // the row's k-th entry (the first tile: those left after seeding).
-          // The eight rows' lists live in registers and take their
-          // candidates in lockstep, one per row per step, so the rows'
-          // dependent warp operations overlap; insert() applies the exact
-          // (value desc, token asc) order and drops what falls below k.
+          // Top-k of each row over this CTA's tiles.  Bits 4i..4i+3 of `mk`
+          // mark this lane's logits of row i that are candidates for the
+          // row's list: at or above its k-th entry (in the first tile: those
+          // left after seeding).
           uint32_t mk = 0;
-          if (!first) {
+          if (first) {
+            // The list starts from the lanes' best logits, sorted by a warp
+            // bitonic network; the eight rows go through it side by side
+            // (every loop runs one operation for all rows before the next).
+            float sv[kRowsPerWarp];
+            int st[kRowsPerWarp], best[kRowsPerWarp];
+#pragma unroll
+            for (int i = 0; i < kRowsPerWarp; ++i) {
+              sv[i] = z[i][0];
+              st[i] = vb < a.V ? vb : 0x7fffffff;
+              best[i] = 0;
+#pragma unroll
+              for (int e = 1; e < 4; ++e) {
+                const int te = vb + e < a.V ? vb + e : 0x7fffffff;
+                if (cand_better(z[i][e], te, sv[i], st[i])) {
+                  sv[i] = z[i][e];
+                  st[i] = te;
+                  best[i] = e;
+                }
+              }
+              if (i >= nr) {
+                sv[i] = kNegInf;
+                st[i] = 0x7fffffff;
+              }
+            }
+#pragma unroll
+            for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+              for (int j = size >> 1; j > 0; j >>= 1) {
+                float ov[kRowsPerWarp];
+                int ot[kRowsPerWarp];
+#pragma unroll
+                for (int i = 0; i < kRowsPerWarp; ++i) ov[i] = __shfl_xor_sync(kFull, sv[i], j);
+#pragma unroll
+                for (int i = 0; i < kRowsPerWarp; ++i) ot[i] = __shfl_xor_sync(kFull, st[i], j);
+                const bool take_best = ((lane & j) == 0) == ((lane & size) == 0);
+#pragma unroll
+                for (int i = 0; i < kRowsPerWarp; ++i) {
+                  const bool sw = take_best ? cand_better(ov[i], ot[i], sv[i], st[i])
+                                            : cand_better(sv[i], st[i], ov[i], ot[i]);
+                  sv[i] = sw ? ov[i] : sv[i];
+                  st[i] = sw ? ot[i] : st[i];
+                }
+              }
+            }
+            float tv[kRowsPerWarp];
+            int tt[kRowsPerWarp];
+#pragma unroll
+            for (int i = 0; i < kRowsPerWarp; ++i) tv[i] = __shfl_sync(kFull, sv[i], k - 1);
+#pragma unroll
+            for (int i = 0; i < kRowsPerWarp; ++i) tt[i] = __shfl_sync(kFull, st[i], k - 1);
+#pragma unroll
+            for (int i = 0; i < kRowsPerWarp; ++i) {
+              if (i < nr) {
+                const int rl = r0 + i;
+                if (lane < k) {
+                  lv[rl * k + lane] = sv[i];
+                  lt[rl * k + lane] = st[i];
+                }
+                if (lane == k - 1) thr_v[rl] = sv[i];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                  const int te = vb + e < a.V ? vb + e : 0x7fffffff;
+                  if (e != best[i] && cand_better(z[i][e], te, tv[i], tt[i]))
+                    mk |= 1u << (4 * i + e);
+                }
+              }
+            }
+            __syncwarp();
+          } else {
 #pragma unroll
             for (int i = 0; i < kRowsPerWarp; ++i) {
               if (i < nr) {
@@ -426,11 +492,13 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
               }
             }
           }
-          if (!first && __any_sync(kFull, mk != 0)) {
-            // Later tiles: few candidates, so one lane per row inserts them
-            // into the row's list in shared memory.  Each round compacts up
-            // to kCand candidates per row (ballots, in (entry, lane) order)
-            // into this warp's buffer; lane i then walks row i's candidates.
+          if (__any_sync(kFull, mk != 0)) {
+            // Candidates are few, so one lane per row inserts them into the
+            // row's list in shared memory.  Each round compacts up to kCand
+            // candidates per row (ballots, in (entry, lane) order) into this
+            // warp's buffer; lane i then walks row i's candidates, each one
+            // placed by an insertion step (exact (value desc, token asc)
+            // order; what falls below the k-th drops out).
             float* cv_w = cbv + ew * kRowsPerWarp * kCand;
             int* ct_w = cbt + ew * kRowsPerWarp * kCand;
             const unsigned below = (1u << lane) - 1u;
@@ -481,145 +549,6 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
                 thr_v[rl] = kv;
               }
               __syncwarp();
-            }
-          } else if (first) {
-            // The eight lists are worked on side by side: every loop below
-            // runs one operation for all eight rows before the next, so the
-            // rows' warp shuffles and votes overlap instead of queueing.
-            float sv[kRowsPerWarp];
-            int st[kRowsPerWarp];
-            if (first) {
-              // the list starts from the lanes' best logits (a warp bitonic
-              // sort); the lane's other logits that beat its k-th entry are
-              // marked
-              int best[kRowsPerWarp];
-#pragma unroll
-              for (int i = 0; i < kRowsPerWarp; ++i) {
-                sv[i] = z[i][0];
-                st[i] = vb < a.V ? vb : 0x7fffffff;
-                best[i] = 0;
-#pragma unroll
-                for (int e = 1; e < 4; ++e) {
-                  const int te = vb + e < a.V ? vb + e : 0x7fffffff;
-                  if (cand_better(z[i][e], te, sv[i], st[i])) {
-                    sv[i] = z[i][e];
-                    st[i] = te;
-                    best[i] = e;
-                  }
-                }
-                if (i >= nr) {
-                  sv[i] = kNegInf;
-                  st[i] = 0x7fffffff;
-                }
-              }
-#pragma unroll
-              for (int size = 2; size <= 32; size <<= 1) {
-#pragma unroll
-                for (int j = size >> 1; j > 0; j >>= 1) {
-                  float ov[kRowsPerWarp];
-                  int ot[kRowsPerWarp];
-#pragma unroll
-                  for (int i = 0; i < kRowsPerWarp; ++i) ov[i] = __shfl_xor_sync(kFull, sv[i], j);
-#pragma unroll
-                  for (int i = 0; i < kRowsPerWarp; ++i) ot[i] = __shfl_xor_sync(kFull, st[i], j);
-                  const bool take_best = ((lane & j) == 0) == ((lane & size) == 0);
-#pragma unroll
-                  for (int i = 0; i < kRowsPerWarp; ++i) {
-                    const bool sw = take_best ? cand_better(ov[i], ot[i], sv[i], st[i])
-                                              : cand_better(sv[i], st[i], ov[i], ot[i]);
-                    sv[i] = sw ? ov[i] : sv[i];
-                    st[i] = sw ? ot[i] : st[i];
-                  }
-                }
-              }
-              float tv[kRowsPerWarp];
-              int tt[kRowsPerWarp];
-#pragma unroll
-              for (int i = 0; i < kRowsPerWarp; ++i) tv[i] = __shfl_sync(kFull, sv[i], k - 1);
-#pragma unroll
-              for (int i = 0; i < kRowsPerWarp; ++i) tt[i] = __shfl_sync(kFull, st[i], k - 1);
-#pragma unroll
-              for (int i = 0; i < kRowsPerWarp; ++i) {
-                if (lane >= k) {
-                  sv[i] = kNegInf;
-                  st[i] = 0x7fffffff;
-                }
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                  const int te = vb + e < a.V ? vb + e : 0x7fffffff;
-                  if (i < nr && e != best[i] && cand_better(z[i][e], te, tv[i], tt[i]))
-                    mk |= 1u << (4 * i + e);
-                }
-              }
-            } else {
-#pragma unroll
-              for (int i = 0; i < kRowsPerWarp; ++i) {
-                const bool has = i < nr && lane < k;
-                sv[i] = has ? lv[(r0 + i) * k + lane] : kNegInf;
-                st[i] = has ? lt[(r0 + i) * k + lane] : 0x7fffffff;
-              }
-            }
-            // Candidates go in one per row per step: the lowest lane with a
-            // candidate of row i offers its first one (no lane: the sentinel,
-            // which changes nothing).  An insert places (cv, ct) at its rank
-            // below k, moves the later entries down one and drops the k-th.
-            // One mark word per row keeps the rows independent.
-            uint32_t mr[kRowsPerWarp];
-#pragma unroll
-            for (int i = 0; i < kRowsPerWarp; ++i) mr[i] = (mk >> (4 * i)) & 15u;
-            while (__any_sync(kFull, mk != 0)) {
-              uint32_t lanes[kRowsPerWarp];
-              float cv[kRowsPerWarp];
-              int ct[kRowsPerWarp], src[kRowsPerWarp], ee[kRowsPerWarp];
-#pragma unroll
-              for (int i = 0; i < kRowsPerWarp; ++i) lanes[i] = __ballot_sync(kFull, mr[i] != 0);
-#pragma unroll
-              for (int i = 0; i < kRowsPerWarp; ++i) {
-                src[i] = lanes[i] ? __ffs(lanes[i]) - 1 : 0;
-                ee[i] = mr[i] ? __ffs(mr[i]) - 1 : 0;
-                // z[i][ee[i]] by two bit selects (an indexed read would put
-                // z in local memory)
-                const float c01 = (ee[i] & 1) ? z[i][1] : z[i][0];
-                const float c23 = (ee[i] & 1) ? z[i][3] : z[i][2];
-                cv[i] = mr[i] ? ((ee[i] & 2) ? c23 : c01) : kNegInf;
-                ct[i] = mr[i] && vb + ee[i] < a.V ? vb + ee[i] : 0x7fffffff;
-              }
-#pragma unroll
-              for (int i = 0; i < kRowsPerWarp; ++i) cv[i] = __shfl_sync(kFull, cv[i], src[i]);
-#pragma unroll
-              for (int i = 0; i < kRowsPerWarp; ++i) ct[i] = __shfl_sync(kFull, ct[i], src[i]);
-              int pos[kRowsPerWarp];
-#pragma unroll
-              for (int i = 0; i < kRowsPerWarp; ++i) {
-                mr[i] = lane == src[i] ? (mr[i] & ~(1u << ee[i])) : mr[i];
-                pos[i] = __popc(__ballot_sync(kFull, lane < k && cand_better(sv[i], st[i], cv[i], ct[i])));
-              }
-              float uv[kRowsPerWarp];
-              int ut[kRowsPerWarp];
-#pragma unroll
-              for (int i = 0; i < kRowsPerWarp; ++i) uv[i] = __shfl_up_sync(kFull, sv[i], 1);
-#pragma unroll
-              for (int i = 0; i < kRowsPerWarp; ++i) ut[i] = __shfl_up_sync(kFull, st[i], 1);
-              mk = 0;
-#pragma unroll
-              for (int i = 0; i < kRowsPerWarp; ++i) {
-                const bool here = lane == pos[i];
-                const bool down = lane > pos[i] && lane < k;
-                sv[i] = here ? cv[i] : (down ? uv[i] : sv[i]);
-                st[i] = here ? ct[i] : (down ? ut[i] : st[i]);
-                mk |= mr[i];
-              }
-            }
-#pragma unroll
-            for (int i = 0; i < kRowsPerWarp; ++i) {
-              if (i < nr) {
-                const int rl = r0 + i;
-                if (lane < k) {
-                  lv[rl * k + lane] = sv[i];
-                  lt[rl * k + lane] = st[i];
-                }
-                if (lane == k - 1) thr_v[rl] = sv[i];
-              }
             }
           }
         }
