@@ -426,11 +426,10 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
 #pragma unroll
               for (int e = 1; e < 4; ++e) {
                 const int te = vb + e < a.V ? vb + e : 0x7fffffff;
-                if (cand_better(z[i][e], te, sv[i], st[i])) {
-                  sv[i] = z[i][e];
-                  st[i] = te;
-                  best[i] = e;
-                }
+                const bool bt = cand_better(z[i][e], te, sv[i], st[i]);
+                sv[i] = bt ? z[i][e] : sv[i];
+                st[i] = bt ? te : st[i];
+                best[i] = bt ? e : best[i];
               }
               if (i >= nr) {
                 sv[i] = kNegInf;
@@ -450,8 +449,9 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
                 const bool take_best = ((lane & j) == 0) == ((lane & size) == 0);
 #pragma unroll
                 for (int i = 0; i < kRowsPerWarp; ++i) {
-                  const bool sw = take_best ? cand_better(ov[i], ot[i], sv[i], st[i])
-                                            : cand_better(sv[i], st[i], ov[i], ot[i]);
+                  const bool b1 = cand_better(ov[i], ot[i], sv[i], st[i]);
+                  const bool b2 = cand_better(sv[i], st[i], ov[i], ot[i]);
+                  const bool sw = (take_best & b1) | (!take_best & b2);
                   sv[i] = sw ? ov[i] : sv[i];
                   st[i] = sw ? ot[i] : st[i];
                 }
@@ -475,8 +475,8 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
                   const int te = vb + e < a.V ? vb + e : 0x7fffffff;
-                  if (e != best[i] && cand_better(z[i][e], te, tv[i], tt[i]))
-                    mk |= 1u << (4 * i + e);
+                  const bool m = (e != best[i]) & cand_better(z[i][e], te, tv[i], tt[i]);
+                  mk |= static_cast<uint32_t>(m) << (4 * i + e);
                 }
               }
             }

@@ -96,8 +96,27 @@ __device__ __forceinline__ uint32_t desc_key(float x) {
 }
 
 // Candidate order inside one parent: larger logit first, then lower token.
+// Written with bitwise operators: short-circuit forms compile to branches,
+// which diverge between lanes when the comparisons differ per lane.
 __device__ __forceinline__ bool cand_better(float a, int ta, float b, int tb) {
-  return a > b || (a == b && ta < tb);
+  return (a > b) | ((a == b) & (ta < tb));
+}
+
+// a[idx] for a register array of N entries (N a power of two), by a tree of
+// selects on idx's bits: an indexed read would move the array to local
+// memory, and one comparison per entry may compile to divergent branches.
+template <int N, typename T>
+__device__ __forceinline__ T pick(const T (&a)[N], int idx) {
+  T lvl[N];
+#pragma unroll
+  for (int j = 0; j < N; ++j) lvl[j] = a[j];
+#pragma unroll
+  for (int w = N / 2, b = 0; w >= 1; w /= 2, ++b) {
+    const bool hi = (idx >> b) & 1;
+#pragma unroll
+    for (int j = 0; j < w; ++j) lvl[j] = hi ? lvl[2 * j + 1] : lvl[2 * j];
+  }
+  return lvl[0];
 }
 
 // ---------------------------------------------------------------------------
@@ -115,19 +134,15 @@ struct WarpList {
   // Inserts the warp-uniform candidate (cv, ct), dropping the k-th entry.
   __device__ __forceinline__ void insert(float cv, int ct, int k) {
     const int lane = threadIdx.x & 31;
-    const bool ahead = lane < k && cand_better(v, t, cv, ct);
+    const bool ahead = (lane < k) & cand_better(v, t, cv, ct);
     const int pos = __popc(__ballot_sync(kFull, ahead));
     const float uv = __shfl_up_sync(kFull, v, 1);
     const int ut = __shfl_up_sync(kFull, t, 1);
-    if (pos < k) {
-      if (lane == pos) {
-        v = cv;
-        t = ct;
-      } else if (lane > pos && lane < k) {
-        v = uv;
-        t = ut;
-      }
-    }
+    // selects, not branches (pos == k leaves every entry below k as it is)
+    const bool here = lane == pos;
+    const bool down = (lane > pos) & (lane < k);
+    v = here ? cv : (down ? uv : v);
+    t = here ? ct : (down ? ut : t);
   }
   // Starts the list from one candidate per lane (the list must be empty):
   // a warp bitonic sort puts the best first, lanes >= k take the sentinel.
@@ -142,12 +157,13 @@ struct WarpList {
         const float ov = __shfl_xor_sync(kFull, v, j);
         const int ot = __shfl_xor_sync(kFull, t, j);
         const bool take_best = ((lane & j) == 0) == ((lane & size) == 0);
-        const bool swap = take_best ? cand_better(ov, ot, v, t)
-                                    : cand_better(v, t, ov, ot);
-        if (swap) {
-          v = ov;
-          t = ot;
-        }
+        // both orders evaluated, then selected: a lane-dependent choice
+        // between two calls compiles to divergent branches
+        const bool b1 = cand_better(ov, ot, v, t);
+        const bool b2 = cand_better(v, t, ov, ot);
+        const bool swap = (take_best & b1) | (!take_best & b2);
+        v = swap ? ov : v;
+        t = swap ? ot : t;
       }
     }
     if (lane >= k) reset();
@@ -172,12 +188,12 @@ struct WarpList {
 // terms exp(x), x <= 0, use the fast exponential: its relative error (a few
 // 1e-7) stays far below the 1e-4 tolerance on log-probabilities.
 __device__ __forceinline__ void lse_push(float& m, float& s, float z) {
-  if (z > m) {
-    s = s * __expf(m - z) + 1.0f;
-    m = z;
-  } else if (z > -__int_as_float(0x7f800000)) {
-    s += __expf(z - m);
-  }
+  // one exponential and selects (no lane-dependent branch): a new maximum
+  // rescales the sum, anything else adds exp(z - m); -inf adds nothing
+  const bool up = z > m;
+  const float e = __expf(up ? m - z : z - m);
+  s = up ? s * e + 1.0f : (z > -__int_as_float(0x7f800000) ? s + e : s);
+  m = up ? z : m;
 }
 
 __device__ __forceinline__ void lse_merge(float& m, float& s, float m2,

@@ -340,11 +340,10 @@ __device__ void merge_stage(const CUtensorMap* tmap_w, const FusedArgs& a,
     int bt = ft[0], bu = 0;
 #pragma unroll
     for (int u = 1; u < kG; ++u) {
-      if (cand_better(fz[u], ft[u], bz, bt)) {
-        bz = fz[u];
-        bt = ft[u];
-        bu = u;
-      }
+      const bool b = cand_better(fz[u], ft[u], bz, bt);
+      bz = b ? fz[u] : bz;
+      bt = b ? ft[u] : bt;
+      bu = b ? u : bu;
     }
     WarpList lst;
     lst.seed(bz, bt, k);
@@ -354,20 +353,13 @@ __device__ void merge_stage(const CUtensorMap* tmap_w, const FusedArgs& a,
       unsigned marks = 0;
 #pragma unroll
       for (int u = 0; u < kG; ++u)
-        if (u != bu && cand_better(fz[u], ft[u], tz, tt)) marks |= 1u << u;
+        marks |= static_cast<unsigned>((u != bu) & cand_better(fz[u], ft[u], tz, tt)) << u;
 #pragma unroll 1
       while (__any_sync(kFull, marks != 0)) {
         const int sel = marks != 0 ? __ffs(marks) - 1 : -1;
         marks &= marks - 1;
-        float cv = kNegInf;
-        int cti = 0x7fffffff;
-#pragma unroll
-        for (int u = 0; u < kG; ++u) {
-          if (u == sel) {
-            cv = fz[u];
-            cti = ft[u];
-          }
-        }
+        const float cv = sel >= 0 ? pick(fz, sel) : kNegInf;
+        const int cti = sel >= 0 ? pick(ft, sel) : 0x7fffffff;
         lst.offer(cv, cti, k);
       }
     }

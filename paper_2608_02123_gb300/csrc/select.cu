@@ -165,21 +165,14 @@ partials_kernel(const float* __restrict__ Z, int ldz, int V, int k,
     for (int i = 0; i < kPartVals; ++i) {
       const int o = b + (i >> 2) * 128 + lane * 4 + (i & 3);
       const int tok = o < len ? tbase + (i >> 2) * 128 + (i & 3) : 0x7fffffff;
-      if (cand_better(z[i], tok, tv, tt)) marks |= 1u << i;
+      marks |= static_cast<unsigned>(cand_better(z[i], tok, tv, tt)) << i;
     }
     marks &= ~skip;
     while (__any_sync(kFull, marks != 0)) {
       const int sel = marks != 0 ? __ffs(marks) - 1 : -1;
       marks &= marks - 1;
-      float cv = kNegInf;
-      int ct = 0x7fffffff;
-#pragma unroll
-      for (int i = 0; i < kPartVals; ++i) {
-        if (i == sel) {
-          cv = z[i];
-          ct = tbase + (i >> 2) * 128 + (i & 3);
-        }
-      }
+      const float cv = sel >= 0 ? pick(z, sel) : kNegInf;
+      const int ct = sel >= 0 ? tbase + (sel >> 2) * 128 + (sel & 3) : 0x7fffffff;
       lst.offer(cv, ct, k);
     }
   }
@@ -304,11 +297,10 @@ merge_kernel(int d, int B, int k, int b_d, int rpq, int shared, int V, int H,
         int bi = ci[0], bu = 0;
 #pragma unroll
         for (int u = 1; u < kUnroll; ++u) {
-          if (cand_better(cv[u], ci[u], bv, bi)) {
-            bv = cv[u];
-            bi = ci[u];
-            bu = u;
-          }
+          const bool b = cand_better(cv[u], ci[u], bv, bi);
+          bv = b ? cv[u] : bv;
+          bi = b ? ci[u] : bi;
+          bu = b ? u : bu;
         }
         lst.seed(bv, bi, k);
         skip = 1u << bu;
@@ -318,20 +310,13 @@ merge_kernel(int d, int B, int k, int b_d, int rpq, int shared, int V, int H,
       unsigned marks = 0;
 #pragma unroll
       for (int u = 0; u < kUnroll; ++u)
-        if (cand_better(cv[u], ci[u], tv, tt)) marks |= 1u << u;
+        marks |= static_cast<unsigned>(cand_better(cv[u], ci[u], tv, tt)) << u;
       marks &= ~skip;
       while (__any_sync(kFull, marks != 0)) {
         const int sel = marks != 0 ? __ffs(marks) - 1 : -1;
         marks &= marks - 1;
-        float ov = kNegInf;
-        int ot = 0x7fffffff;
-#pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-          if (u == sel) {
-            ov = cv[u];
-            ot = ci[u];
-          }
-        }
+        const float ov = sel >= 0 ? pick(cv, sel) : kNegInf;
+        const int ot = sel >= 0 ? pick(ci, sel) : 0x7fffffff;
         lst.offer(ov, ot, k);
       }
     }
