@@ -44,6 +44,7 @@ constexpr int kThreads = 64 + kEpiThreads;
 constexpr int kCC = 64;           // accumulator columns per transpose chunk
 constexpr int kRowsPerWarp = kCC / kEpiWarps;
 constexpr int kCand = 16;         // compacted candidates per row and round
+constexpr int kRegList = 16;      // k up to this: a row's list in registers
 constexpr int kMaxStages = 8;
 constexpr int kSmemLimit = 227 * 1024;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per bounded wait
@@ -407,6 +408,12 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
               row_s[r0 + lane] = sm;
             }
           }
+          // the rows' logits go back to zs: the candidate compaction below
+          // reads them there, so that z's registers are free for the lists
+#pragma unroll
+          for (int i = 0; i < kRowsPerWarp; ++i)
+            reinterpret_cast<float4*>(zs[r0 - c0 + i])[lane] =
+                make_float4(z[i][0], z[i][1], z[i][2], z[i][3]);
           // Top-k of each row over this CTA's tiles.  Bits 4i..4i+3 of `mk`
           // mark this lane's logits of row i that are candidates for the
           // row's list: at or above its k-th entry (in the first tile: those
@@ -513,7 +520,7 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
                   const unsigned b = __ballot_sync(kFull, m);
                   const int slot = base + __popc(b & below);
                   if (m && slot < kCand) {
-                    cv_w[i * kCand + slot] = z[i][e];
+                    cv_w[i * kCand + slot] = zs[r0 - c0 + i][lane * 4 + e];
                     ct_w[i * kCand + slot] = vb + e;
                     mk &= ~(1u << (4 * i + e));
                   }
@@ -522,7 +529,41 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
                 if (lane == i) n_mine = base < kCand ? base : kCand;
               }
               __syncwarp();
-              if (lane < nr) {
+              if (lane < nr && k <= kRegList) {
+                // the row's list in registers (entries >= k are sentinels):
+                // each candidate goes through a fixed insertion network,
+                // all comparisons against the old entries, then selects
+                const int rl = r0 + lane;
+                float rv[kRegList];
+                int rt[kRegList];
+#pragma unroll
+                for (int j = 0; j < kRegList; ++j) {
+                  rv[j] = j < k ? lv[rl * k + j] : kNegInf;
+                  rt[j] = j < k ? lt[rl * k + j] : 0x7fffffff;
+                }
+                for (int c = 0; c < n_mine; ++c) {
+                  const float v = cv_w[lane * kCand + c];
+                  const int t = ct_w[lane * kCand + c];
+                  bool bt[kRegList];
+#pragma unroll
+                  for (int j = 0; j < kRegList; ++j) bt[j] = cand_better(v, t, rv[j], rt[j]);
+#pragma unroll
+                  for (int j = kRegList - 1; j > 0; --j) {
+                    rv[j] = bt[j - 1] ? rv[j - 1] : (bt[j] ? v : rv[j]);
+                    rt[j] = bt[j - 1] ? rt[j - 1] : (bt[j] ? t : rt[j]);
+                  }
+                  rv[0] = bt[0] ? v : rv[0];
+                  rt[0] = bt[0] ? t : rt[0];
+                }
+#pragma unroll
+                for (int j = 0; j < kRegList; ++j) {
+                  if (j < k) {
+                    lv[rl * k + j] = rv[j];
+                    lt[rl * k + j] = rt[j];
+                  }
+                }
+                thr_v[rl] = pick(rv, k - 1);
+              } else if (lane < nr) {
                 const int rl = r0 + lane;
                 float* Lv = lv + rl * k;
                 int* Lt = lt + rl * k;
