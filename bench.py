@@ -566,7 +566,7 @@ def run_ours(args, wl, rank, world, local_rank):
                      "peak_source": peak_kind,
                      "launches": launches,
                      "avg_launch_us": proj_ms * 1e3 / launches if launches else None,
-                     "traffic": recorded_traffic(wl, fused)},
+                     "traffic": recorded_traffic(wl, fused and layout == "tiled")},
         "draft_us": {"p10": draft_us[len(draft_us) // 10],
                      "p50": draft_us[len(draft_us) // 2],
                      "p90": draft_us[(9 * len(draft_us)) // 10]},
