@@ -699,6 +699,12 @@ def run_sweep(args, wl, local_rank):
     E_host, W_host = draw_head(base)
     E = torch.from_numpy(E_host.view(np.int16)).to(dev).view(torch.bfloat16)
     W = torch.from_numpy(W_host.view(np.int16)).to(dev).view(torch.bfloat16)
+    layout = args.head_layout
+    if layout == "tiled":
+        # one tiled copy serves every (B, k, N) point (it depends on V, H only)
+        W = P.pack_head(P.make_config(base.V, base.H, 1, 1, 1, 1, 0, "bf16", "parent",
+                                      "tiled"), W)
+        torch.cuda.synchronize()
     n_sets = N_SETS
     many = base.with_(batch=n_sets)
     reqs = [draw_request(many, i) for i in range(n_sets)]
@@ -715,7 +721,7 @@ def run_sweep(args, wl, local_rank):
         for k in SWEEP_K:
             for N in SWEEP_N:
                 wk = base.with_(B=B, k=k, N=N)
-                cfg = P.make_config(wk.V, wk.H, B, k, N, 1, 0, "bf16", wk.mode)
+                cfg = P.make_config(wk.V, wk.H, B, k, N, 1, 0, "bf16", wk.mode, layout)
                 dr = P.Drafter(cfg, dev)
                 taus = []
 
@@ -742,6 +748,7 @@ def run_sweep(args, wl, local_rank):
                 tau = float(torch.stack(taus).float().mean()) + 1.0
                 print(json.dumps({
                     "sweep": "kN", "workload": wk.name, "mode": wk.mode,
+                    "head_layout": layout, "rounds": steps,
                     "B": B, "k": k, "N": N, "us_per_round": ms * 1e3,
                     "rounds_per_s": 1e3 / ms,
                     "round_hbm_fraction": round_bytes(wk) / (ms * 1e-3) / 1e9 / peak,
