@@ -2,11 +2,12 @@
 // states of the accepted path to the slots right after the verified prefix
 // (Appendix A, "Tensor implementation").
 //
-// Work split: one warp per 512-byte column chunk of one (layer, plane,
-// request) row block, plus one warp per 512-byte chunk of each request's
-// hidden-state rows; the warp checks the request's path cooperatively (one
-// coalesced load of the accepted indices, ballots), then each lane moves its
-// 16-byte column for every accepted node.  The cache is compacted in place:
+// Work split: one thread per 16-byte column of one (layer, plane, request)
+// row block, or of one request's hidden-state rows; consecutive threads take
+// consecutive columns.  Each thread checks its request's path (the indices
+// are loaded eight at a time with all loads in flight, so a path costs one
+// or two memory round trips, not one per node), then moves its column for
+// every accepted node.  The cache is compacted in place:
 // accepted indices strictly increase from a[0] = 0, so a[j] >= j and slot
 // T + a[j] is never one of the slots T + 1 .. T + j - 1 already written.  A
 // lane therefore loads a batch of sources before it stores the batch, and
@@ -41,23 +42,50 @@ struct CompactArgs {
 
 // Validity of request r's path and prefix (the rule pctree_accept follows:
 // root first, then strictly increasing packed indices below N).  Returns
-// the accepted length L, or -1 when the request must be left untouched.
-__device__ __forceinline__ int checked_len(const CompactArgs& a, int r, int* T_out) {
+// the accepted length L, or -1 when the request must be left untouched;
+// *j0_out is the first j >= 1 with a[j] != j (the nodes before it are
+// already in their slots).  The indices are read kPathBatch at a time, every
+// load of a batch issued before any is used.
+constexpr int kPathBatch = 4;
+
+__device__ __forceinline__ int checked_len(const CompactArgs& a, int r, int* T_out,
+                                           int* j0_out) {
   const int B = a.lay.B, N = a.lay.N;
-  const int L = a.len[r];
-  const int T = a.prefix[r];
+  const int32_t* p = a.acc + static_cast<size_t>(r) * (B + 1);
+  // the length, the prefix and the first batch of indices in one round trip
+  // (the indices up to B are always in bounds, whatever L is)
+  const int L = __ldg(a.len + r);
+  const int T = __ldg(a.prefix + r);
+  int x0[kPathBatch];
+#pragma unroll
+  for (int u = 0; u < kPathBatch; ++u) x0[u] = u <= B ? __ldg(p + u) : 0;
   *T_out = T;
+  *j0_out = 1;
   if (L < 0 || L > B || T < 0 || static_cast<long long>(T) + N > a.lay.max_slots)
     return -1;
-  const int32_t* p = a.acc + static_cast<size_t>(r) * (B + 1);
-  int prev = p[0];
-  if (prev != 0) return -1;
-  for (int j = 1; j <= L; ++j) {
-    const int x = p[j];
-    if (x <= prev || x >= N) return -1;
-    prev = x;
+  int prev = -1;
+  bool ok = true, in_place = true;
+  int j0 = L + 1;
+  for (int j = 0; j <= L; j += kPathBatch) {
+    int x[kPathBatch];
+#pragma unroll
+    for (int u = 0; u < kPathBatch; ++u)
+      x[u] = j == 0 ? x0[u] : (j + u <= L ? __ldg(p + j + u) : 0);
+#pragma unroll
+    for (int u = 0; u < kPathBatch; ++u) {
+      const int jj = j + u;
+      if (jj <= L) {
+        ok &= jj == 0 ? x[u] == 0 : (x[u] > prev && x[u] < N);
+        prev = x[u];
+        if (jj >= 1 && in_place && x[u] != jj) {
+          in_place = false;
+          j0 = jj;
+        }
+      }
+    }
   }
-  return L;
+  *j0_out = j0;
+  return ok ? L : -1;
 }
 
 // Moves rows j0 .. L of one 16-byte column: row j <- row p[j] of `src`.
@@ -104,7 +132,8 @@ compact_kernel(CompactArgs a) {
       r = h / a.hidden_vecs;
       off = 0;
     }
-    const int L = checked_len(a, r, &T);
+    int j0;
+    const int L = checked_len(a, r, &T, &j0);
     if (L < 0) {
       if (a.status != nullptr && col == 0 && (!in_cache || u < a.row_vecs * a.lay.batch))
         *a.status = PCTREE_ERR_INVALID_ARG;
@@ -113,9 +142,7 @@ compact_kernel(CompactArgs a) {
     const int32_t* p = a.acc + static_cast<size_t>(r) * (a.lay.B + 1);
     if (in_cache) {
       // in place after the verified prefix; nodes already in their slots
-      // (a[j] == j at the head of the path) stay
-      int j0 = 1;
-      while (j0 <= L && p[j0] == j0) ++j0;
+      // (a[j] == j at the head of the path, before j0) stay
       unsigned char* base = a.cache + off + T * a.lay.slot_stride + col * 16;
       move_column(base, base, a.lay.slot_stride, a.lay.slot_stride, p, j0, L);
     } else {
