@@ -53,6 +53,11 @@ def parse_args():
                     help="skip the short timing of the batched serving "
                          "workloads (8B-shaped batch 16, 14B-shaped batch 32) "
                          "that the default line carries under 'batched'")
+    ap.add_argument("--no-around", action="store_true",
+                    help="skip the short timing of the steps around the "
+                         "round (a tree-attention layer and the compaction "
+                         "at the 14B-shaped batch-32 shapes) that the default "
+                         "line carries under 'around_round'")
     ap.add_argument("--mode", default="parent", choices=["parent", "shared"],
                     help="child scoring: PCTree, or the Shared-Markov control")
     ap.add_argument("--sweep", action="store_true",
@@ -583,6 +588,13 @@ def run_ours(args, wl, rank, world, local_rank):
     }
     if world == 1 and not args.no_batched and args.workload == "4b_b16":
         line["batched"] = measure_batched(dev, gpu_index, layout)
+    if world == 1 and not args.no_around and args.workload == "4b_b16":
+        # the steps of a serving round around the draft, at the 14B-shaped
+        # batch-32 serving shapes: one verification attention layer and the
+        # compaction after acceptance
+        line["around_round"] = [
+            measure_attention("14b_b16_bs32", local_rank, 2000, 10, gpu_index),
+            measure_compact("14b_b16_bs32", local_rank, 8000, 10, gpu_index)]
     if world == 1 and not args.no_cpu_baseline:
         runner = OracleRunner(wl, E_host, W_host,
                               [(L[0], int(root[0])) for L, root, _ in sets])
@@ -771,17 +783,18 @@ def compact_bytes(cw, acc, lens):
     return total
 
 
-def run_compact(args, local_rank):
+def measure_compact(name, local_rank, steps, warmup, gpu_index=None):
     """Accepted-row compaction (the step after acceptance) on one GPU: a
     cache of the workload's shape resident in HBM, accepted paths and
     prefix lengths rotating over 16 seeded sets, so a launch's rows were
     last touched 15 launches (and, at the large workloads, over 1 GB of
-    other rows) earlier: inputs larger than L2, no flush."""
+    other rows) earlier: inputs larger than L2, no flush.  Returns the
+    measurement as a dict."""
     import torch
 
     from paper_2608_02123_gb300 import pctree as P
 
-    cw = COMPACT_WORKLOADS[args.compact_workload]
+    cw = COMPACT_WORKLOADS[name]
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
     gen = torch.Generator(device=dev)
@@ -808,7 +821,7 @@ def run_compact(args, local_rank):
         P.pctree_compact(lay, acc[j], lens[j], pre[j], cache, hin, hout,
                          status, s if s is not None else stream)
 
-    for i in range(max(args.warmup, 3)):
+    for i in range(max(warmup, 3)):
         step(i)
     torch.cuda.synchronize()
     # A launch moves a few MB in a few microseconds, less than a Python
@@ -822,13 +835,13 @@ def run_compact(args, local_rank):
         for i in range(N_SETS):
             step(i, torch.cuda.current_stream())
     torch.cuda.synchronize()
-    reps = max(1, args.steps // N_SETS)
+    reps = max(1, steps // N_SETS)
     for _ in range(2):
         graph.replay()
     torch.cuda.synchronize()
     start = torch.cuda.Event(enable_timing=True)
     end = torch.cuda.Event(enable_timing=True)
-    clocks = ClockSampler(local_rank)
+    clocks = ClockSampler(local_rank if gpu_index is None else gpu_index)
     clocks.start()
     start.record(stream)
     for _ in range(reps):
@@ -836,19 +849,21 @@ def run_compact(args, local_rank):
     end.record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
-    args.steps = reps * N_SETS
+    steps = reps * N_SETS
     if int(status.item()) != 0:
         raise RuntimeError(f"pctree_compact status {int(status.item())}")
     total_ms = start.elapsed_time(end)
-    moved = sum(nbytes[i % N_SETS] for i in range(args.steps))
+    moved = sum(nbytes[i % N_SETS] for i in range(steps))
     peaks, src = measured_peaks()
     peak = float(peaks["hbm_gbs"])
     achieved = moved / (total_ms * 1e-3) / 1e9
-    us = total_ms * 1e3 / args.steps
-    print(json.dumps({
+    us = total_ms * 1e3 / steps
+    del cache, hin, hout, graph
+    torch.cuda.empty_cache()
+    return {
         "metric": "accepted-row compaction µs/round (KV planes + hidden states)",
         "value": us, "unit": "us/round", "higher_is_better": False,
-        "n_gpus": 1, "steps": args.steps, "warmup": max(args.warmup, 3),
+        "n_gpus": 1, "steps": steps, "warmup": max(warmup, 3),
         "dtype": "u8", "data": "synthetic (seeded cache bytes and accepted paths)",
         "config": {"workload": cw.name, "layers": cw.layers,
                    "planes": cw.planes, "row_bytes": cw.row_bytes,
@@ -856,12 +871,17 @@ def run_compact(args, local_rank):
                    "batch": cw.batch, "slots": cw.slots,
                    "l2": "16 rotating path sets; rows larger than L2 between reuses",
                    "launch": "timed launches replayed from a CUDA graph of the 16 path sets"},
-        "bytes_per_round": moved / args.steps,
+        "bytes_per_round": moved / steps,
         "roofline": {"bound": "hbm", "kernel": "compact_kernel",
                      "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_source": src,
                      "traffic": None},
-        "gpu_launches": args.steps, "clocks": clk}), flush=True)
+        "gpu_launches": steps, "clocks": clk}
+
+
+def run_compact(args, local_rank):
+    print(json.dumps(measure_compact(args.compact_workload, local_rank,
+                                     args.steps, args.warmup)), flush=True)
 
 
 def attention_work(ai):
@@ -883,16 +903,16 @@ def attention_work(ai):
     return nbytes, flops
 
 
-def run_attention(args, local_rank):
+def measure_attention(name, local_rank, steps, warmup, gpu_index=None):
     """One tree-verification attention layer (the target's forward that
     verifies the packed tree) on one GPU: the workload's caches resident in
     HBM, rotated over enough copies that a launch's K/V were last read more
-    than 3 x L2 earlier."""
+    than 3 x L2 earlier.  Returns the measurement as a dict."""
     import torch
 
     from paper_2608_02123_gb300 import pctree as P
 
-    aw = ATTN_WORKLOADS[args.attn_workload]
+    aw = ATTN_WORKLOADS[name]
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
     ai = draw_attention(aw)
@@ -919,22 +939,24 @@ def run_attention(args, local_rank):
         P.pctree_tree_attention(cfg, q, ks[i % n_sets], vs[i % n_sets], pre, nn,
                                 par, out, ws, status, stream)
 
-    for i in range(max(args.warmup, 3)):
+    for i in range(max(warmup, 3)):
         step(i)
     torch.cuda.synchronize()
     start = torch.cuda.Event(enable_timing=True)
     end = torch.cuda.Event(enable_timing=True)
-    clocks = ClockSampler(local_rank)
+    clocks = ClockSampler(local_rank if gpu_index is None else gpu_index)
     clocks.start()
     start.record(stream)
-    for i in range(args.steps):
+    for i in range(steps):
         step(i)
     end.record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
     if int(status.item()) != 0:
         raise RuntimeError(f"pctree_tree_attention status {int(status.item())}")
-    ms = start.elapsed_time(end) / args.steps
+    ms = start.elapsed_time(end) / steps
+    del q, k, v, ks, vs, out, ws
+    torch.cuda.empty_cache()
     nbytes, flops = attention_work(ai)
     peaks, src = measured_peaks()
     hbm = float(peaks["hbm_gbs"])
@@ -949,10 +971,10 @@ def run_attention(args, local_rank):
     roof.update({"kernel": "tree_attn_kernel", "peak_source": src,
                  "traffic": None, "other": {"GB/s": gbs, "hbm_frac": gbs / hbm,
                                             "TFLOP/s": tfs, "tensor_frac": tfs / tc}})
-    print(json.dumps({
+    return {
         "metric": "tree-verification attention µs/layer (prefix + ancestors, GQA)",
         "value": ms * 1e3, "unit": "us/layer", "higher_is_better": False,
-        "n_gpus": 1, "steps": args.steps, "warmup": max(args.warmup, 3),
+        "n_gpus": 1, "steps": steps, "warmup": max(warmup, 3),
         "dtype": "bf16", "data": "synthetic (seeded Q/K/V, random breadth-first trees)",
         "config": {"workload": aw.name, "batch": aw.batch, "N": aw.N,
                    "Hq": aw.Hq, "Hkv": aw.Hkv, "D": aw.D,
@@ -960,7 +982,12 @@ def run_attention(args, local_rank):
                    "mean_prefix": float(ai.prefix_len.mean()),
                    "l2": f"K/V rotated over {n_sets} copies (>= 3x L2)"},
         "bytes_per_layer": nbytes, "flops_per_layer": flops,
-        "roofline": roof, "gpu_launches": args.steps, "clocks": clk}), flush=True)
+        "roofline": roof, "gpu_launches": steps, "clocks": clk}
+
+
+def run_attention(args, local_rank):
+    print(json.dumps(measure_attention(args.attn_workload, local_rank,
+                                       args.steps, args.warmup)), flush=True)
 
 
 def main():

@@ -91,6 +91,7 @@ Layout make_layout(const pctree_config& c) {
   l.off_fxch = l.rows_max <= kFusedRows
                    ? take(2 * fparts * kFusedTileRows * sizeof(float))
                    : l.off_xtok;
+  l.off_gthr = take(rows * sizeof(unsigned long long));
   l.total = off;
   return l;
 }
@@ -399,7 +400,8 @@ pctree_status pctree_draft(const pctree_config* cfg, const float* base_logits,
                               reinterpret_cast<float*>(ws + lay.off_ps),
                               reinterpret_cast<float*>(ws + lay.off_pz),
                               reinterpret_cast<int32_t*>(ws + lay.off_pt),
-                              out->status, stream);
+                              reinterpret_cast<unsigned long long*>(ws + lay.off_gthr),
+                              static_cast<unsigned>(d + 1), out->status, stream);
       prof_record(1, stream);
     } else {
       n_parts = lay.n_chunks;

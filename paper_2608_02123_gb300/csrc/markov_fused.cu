@@ -25,8 +25,13 @@
 //      into the row's running pair, and the row's top-k list updated with
 //      the logits that beat its current k-th entry (most tiles have none).
 // A CTA's first tile seeds each row's list with a sort of the lanes' best
-// logits.  Rows are always handled by the same warp in the same tile order,
-// so results are deterministic.
+// logits.  The CTAs also share, per row, the best k-th list entry any of
+// them holds (a 64-bit word in global memory raised with atomicMax after each
+// tile): a logit below it is beaten by k logits of that CTA's slice alone,
+// so it cannot be one of the row's k children and is not inserted.  The
+// shared value only removes candidates that lose anyway, so the merged
+// children do not depend on when a CTA reads it.  Rows are always handled
+// by the same warp in the same tile order.
 #include <cuda_runtime.h>
 
 #include "pctree_common.cuh"
@@ -93,8 +98,22 @@ struct ProjArgs {
   float* part_s;           // [rows][n_parts] per-CTA sum of exp
   float* part_z;           // [rows][n_parts][k] per-CTA top-k logits, best first
   int32_t* part_t;         // [rows][n_parts][k] their tokens
+  // [rows] per row: (tag << 32) | order key of the best k-th list entry of
+  // any CTA; entries of earlier stages carry smaller tags and count as empty
+  unsigned long long* gthr;
+  unsigned tag;            // stage + 1
   int32_t* status;
 };
+
+// Order-preserving 32-bit key of a float (a larger float gives a larger
+// unsigned key; no NaNs reach it) and its inverse.
+__device__ __forceinline__ uint32_t float_key(float f) {
+  const uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float key_float(uint32_t key) {
+  return __uint_as_float((key & 0x80000000u) ? (key & 0x7fffffffu) : ~key);
+}
 
 __device__ __forceinline__ void epi_barrier() { named_barrier(1, kEpiThreads); }
 
@@ -307,6 +326,17 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
       for (int c = 0; c < kChunks; ++c) {
         const int c0 = c * kCC;
         if (c0 >= cols) break;
+        // the shared threshold of this warp's row c0 + 8 ew + lane (lanes
+        // 0..7), read past L1 now so that the load overlaps phase A
+        float gl = kNegInf;
+        {
+          const int rl = c0 + ew * kRowsPerWarp + lane;
+          if (!first && lane < kRowsPerWarp && rl < cols) {
+            const unsigned long long w = __ldcg(a.gthr + a.col0 + rl);
+            if (static_cast<unsigned>(w >> 32) == a.tag)
+              gl = key_float(static_cast<uint32_t>(w));
+          }
+        }
         float lcur[kRowsPerWarp][4];
 #pragma unroll
         for (int i = 0; i < kRowsPerWarp; ++i)
@@ -491,14 +521,17 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
           } else {
 #pragma unroll
             for (int i = 0; i < kRowsPerWarp; ++i) {
+              const float gi = __shfl_sync(kFull, gl, i);
               if (i < nr) {
-                const float tv = thr_v[r0 + i];
+                const float tv = fmaxf(thr_v[r0 + i], gi);
 #pragma unroll
                 for (int e = 0; e < 4; ++e)
                   if (z[i][e] >= tv && vb + e < a.V) mk |= 1u << (4 * i + e);
               }
             }
           }
+          // lane i: row r0 + i's list changed in this chunk
+          bool changed = first;
           if (__any_sync(kFull, mk != 0)) {
             // Candidates are few, so one lane per row inserts them into the
             // row's list in shared memory.  Each round compacts up to kCand
@@ -528,41 +561,57 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
                 }
                 if (lane == i) n_mine = base < kCand ? base : kCand;
               }
+              changed |= n_mine > 0;
               __syncwarp();
-              if (lane < nr && k <= kRegList) {
-                // the row's list in registers (entries >= k are sentinels):
-                // each candidate goes through a fixed insertion network,
-                // all comparisons against the old entries, then selects
-                const int rl = r0 + lane;
-                float rv[kRegList];
-                int rt[kRegList];
+              if (k <= kRegList) {
+                // the row's list in registers, four lanes per row: lane
+                // 4 i + q holds entries 4 q .. 4 q + 3 of row r0 + i
+                // (entries >= k are sentinels).  A candidate goes through
+                // every entry at once: each lane compares it with its four
+                // entries, takes the entry shifted out of the previous
+                // lane's segment, and selects.
+                const int ri = lane >> 2, q = lane & 3;
+                const int rl = r0 + ri;
+                const int n_row = __shfl_sync(kFull, n_mine, ri);
+                const int n_max = __reduce_max_sync(kFull, n_row);
+                float rv[4];
+                int rt[4];
 #pragma unroll
-                for (int j = 0; j < kRegList; ++j) {
-                  rv[j] = j < k ? lv[rl * k + j] : kNegInf;
-                  rt[j] = j < k ? lt[rl * k + j] : 0x7fffffff;
+                for (int j = 0; j < 4; ++j) {
+                  const int e = 4 * q + j;
+                  const bool live = ri < nr && e < k;
+                  rv[j] = live ? lv[rl * k + e] : kNegInf;
+                  rt[j] = live ? lt[rl * k + e] : 0x7fffffff;
                 }
-                for (int c = 0; c < n_mine; ++c) {
-                  const float v = cv_w[lane * kCand + c];
-                  const int t = ct_w[lane * kCand + c];
-                  bool bt[kRegList];
+                for (int c = 0; c < n_max; ++c) {
+                  const bool act = c < n_row;
+                  const float v = act ? cv_w[ri * kCand + c] : kNegInf;
+                  const int t = act ? ct_w[ri * kCand + c] : 0x7fffffff;
+                  bool bt[4];
 #pragma unroll
-                  for (int j = 0; j < kRegList; ++j) bt[j] = cand_better(v, t, rv[j], rt[j]);
+                  for (int j = 0; j < 4; ++j) bt[j] = act & cand_better(v, t, rv[j], rt[j]);
+                  const float pv = __shfl_up_sync(kFull, rv[3], 1);
+                  const int pt = __shfl_up_sync(kFull, rt[3], 1);
+                  const bool pb = (__shfl_up_sync(kFull, static_cast<int>(bt[3]), 1) != 0) & (q != 0);
 #pragma unroll
-                  for (int j = kRegList - 1; j > 0; --j) {
+                  for (int j = 3; j > 0; --j) {
                     rv[j] = bt[j - 1] ? rv[j - 1] : (bt[j] ? v : rv[j]);
                     rt[j] = bt[j - 1] ? rt[j - 1] : (bt[j] ? t : rt[j]);
                   }
-                  rv[0] = bt[0] ? v : rv[0];
-                  rt[0] = bt[0] ? t : rt[0];
+                  rv[0] = pb ? pv : (bt[0] ? v : rv[0]);
+                  rt[0] = pb ? pt : (bt[0] ? t : rt[0]);
                 }
+                if (ri < nr && n_row > 0) {
 #pragma unroll
-                for (int j = 0; j < kRegList; ++j) {
-                  if (j < k) {
-                    lv[rl * k + j] = rv[j];
-                    lt[rl * k + j] = rt[j];
+                  for (int j = 0; j < 4; ++j) {
+                    const int e = 4 * q + j;
+                    if (e < k) {
+                      lv[rl * k + e] = rv[j];
+                      lt[rl * k + e] = rt[j];
+                    }
+                    if (e == k - 1) thr_v[rl] = rv[j];
                   }
                 }
-                thr_v[rl] = pick(rv, k - 1);
               } else if (lane < nr) {
                 const int rl = r0 + lane;
                 float* Lv = lv + rl * k;
@@ -591,6 +640,14 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
               }
               __syncwarp();
             }
+          }
+          // publish the rows' k-th entries for the other CTAs
+          __syncwarp();
+          if (lane < nr && changed) {
+            const float tv = thr_v[r0 + lane];
+            if (tv > kNegInf)
+              atomicMax(a.gthr + a.col0 + r0 + lane,
+                        (static_cast<unsigned long long>(a.tag) << 32) | float_key(tv));
           }
         }
         epi_barrier();   // zs is rewritten by the next chunk
@@ -661,8 +718,9 @@ cudaError_t launch_markov_fused(const CUtensorMap* tmap_w, const CUtensorMap* tm
                                 const float* L, long long l_req_stride, int V,
                                 int H, int k, int rows, int rows_per_req, int bn, int tiled,
                                 int num_sms, float* part_m, float* part_s,
-                                float* part_z, int32_t* part_t, int32_t* status,
-                                cudaStream_t stream) {
+                                float* part_z, int32_t* part_t,
+                                unsigned long long* gthr, unsigned tag,
+                                int32_t* status, cudaStream_t stream) {
   ProjArgs a{};
   a.L = L;
   a.l_req_stride = l_req_stride;
@@ -676,6 +734,8 @@ cudaError_t launch_markov_fused(const CUtensorMap* tmap_w, const CUtensorMap* tm
   a.part_s = part_s;
   a.part_z = part_z;
   a.part_t = part_t;
+  a.gthr = gthr;
+  a.tag = tag;
   a.status = status;
   switch (bn) {
     case 16: return launch_nc<16>(tmap_w, tmap_x, a, num_sms, stream);

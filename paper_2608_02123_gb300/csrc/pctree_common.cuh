@@ -35,6 +35,9 @@ struct Layout {
   // fused-round path: cross-CTA flags, per-CTA partials, parent tokens
   size_t off_sync, sync_bytes, off_fpm, off_fps, off_fcz, off_fct, off_xtok;
   size_t off_fxch;  // fused-round path: partial accumulators of shared tiles
+  // per-stage path (bf16 heads): one word per Markov row, the best k-th
+  // list entry any projection CTA holds so far, tagged with the stage
+  size_t off_gthr;
   size_t total;
 };
 
@@ -339,8 +342,9 @@ cudaError_t launch_markov_fused(const CUtensorMap* tmap_w, const CUtensorMap* tm
                                 const float* L, long long l_req_stride, int V,
                                 int H, int k, int rows, int rows_per_req, int bn, int tiled,
                                 int num_sms, float* part_m, float* part_s,
-                                float* part_z, int32_t* part_t, int32_t* status,
-                                cudaStream_t stream);
+                                float* part_z, int32_t* part_t,
+                                unsigned long long* gthr, unsigned tag,
+                                int32_t* status, cudaStream_t stream);
 
 // f32 heads: Z[row][v] = L[req(row)][v] + sum_h W_out[v][h] X[row][h] for
 // rows [0, rows), req(row) = row / rows_per_req; `L` points at depth d of

@@ -45,8 +45,12 @@ __device__ void copy_row(const void* E_in, void* X, int token, int row, int H,
 __global__ void init_kernel(const int32_t* __restrict__ root, const void* E_in,
                             void* X, int32_t* pool_tok, int32_t* pool_par,
                             float2* pool_s, int32_t* front, int V, int H,
-                            int P, int k, int x_elem, int32_t* status) {
+                            int P, int k, int x_elem, unsigned long long* gthr,
+                            int n_gthr, int32_t* status) {
   const int r = blockIdx.x;
+  // the projection's shared row thresholds start the round empty (tag 0)
+  for (int i = r * blockDim.x + threadIdx.x; i < n_gthr; i += gridDim.x * blockDim.x)
+    gthr[i] = 0ull;
   int tok = root[r];
   if (tok < 0 || tok >= V) {
     if (threadIdx.x == 0) set_status(status, PCTREE_ERR_INVALID_ARG);
@@ -662,7 +666,8 @@ cudaError_t launch_init(const pctree_config& c, const Layout& lay,
       reinterpret_cast<int32_t*>(ws + lay.off_pool_par),
       reinterpret_cast<float2*>(ws + lay.off_pool_s),
       reinterpret_cast<int32_t*>(ws + lay.off_front), c.V, c.H, lay.P, c.k,
-      lay.x_elem, status);
+      lay.x_elem, reinterpret_cast<unsigned long long*>(ws + lay.off_gthr),
+      lay.rows_max, status);
   return cudaGetLastError();
 }
 
