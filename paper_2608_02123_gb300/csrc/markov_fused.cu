@@ -175,6 +175,11 @@ markov_fused_kernel(const __grid_constant__ CUtensorMap tmap_w,
   tc_fence_after_sync();
   const uint32_t tmem_base = *tmem_slot;
   volatile int* abort_v = abort_flag;
+  // the set-up above overlaps the previous kernel of the stream (the merge
+  // that wrote this stage's parent rows); nothing below runs before it is
+  // complete
+  pdl_launch_dependents();
+  pdl_wait();
 
   if (warp == 0) {
     // --------------------------------------------------------------- producer
@@ -697,10 +702,21 @@ cudaError_t launch_nc(const CUtensorMap* tmap_w, const CUtensorMap* tmap_x,
   a.n_stages = stages;
   const int grid = fused_proj_parts(a.V, num_sms);
   const int rows = a.rows;
+  // programmatic dependent launch: a pass may be scheduled while the kernel
+  // before it finishes (the kernel waits for it before touching memory)
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
   for (int col0 = 0; col0 < rows; col0 += NC) {
     a.col0 = col0;
-    markov_fused_kernel<NC><<<grid, kThreads, smem, stream>>>(*tmap_w, *tmap_x, a);
-    e = cudaGetLastError();
+    e = cudaLaunchKernelEx(&cfg, markov_fused_kernel<NC>, *tmap_w, *tmap_x, a);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;

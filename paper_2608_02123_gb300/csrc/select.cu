@@ -245,7 +245,132 @@ __device__ void gather_rows(const void* E_in, void* X, const int* tok,
   }
 }
 
-__global__ void __launch_bounds__(1024)
+// The k best of one row's sorted candidate lists (one per projection CTA or
+// vocabulary chunk, each best first), by a tournament: lane l owns lists
+// l, l + 32, ..., holding each one's head and next entry in registers; each
+// of k rounds takes the warp's best head ((value desc, token asc), the lane
+// breaking exact ties of padding) and advances that list.  Lane r ends with
+// the r-th best entry.  For at most 32 * L lists (L <= 5 fits the
+// register budget of a 1024-thread block; more lists take the scan below).
+template <int L>
+__device__ __forceinline__ void merge_sorted_lists(const float* __restrict__ cz,
+                                                   const int32_t* __restrict__ ct,
+                                                   int n_lists, int k, float& out_v,
+                                                   int& out_t) {
+  const int lane = threadIdx.x & 31;
+  float hv[L], nv[L];
+  int ht[L], nt[L], pos[L];
+#pragma unroll
+  for (int li = 0; li < L; ++li) {
+    const int id = lane + 32 * li;
+    const bool ok = id < n_lists;
+    const size_t o = static_cast<size_t>(ok ? id : 0) * k;
+    hv[li] = ok ? cz[o] : kNegInf;
+    ht[li] = ok ? ct[o] : 0x7fffffff;
+    nv[li] = ok && k > 1 ? cz[o + 1] : kNegInf;
+    nt[li] = ok && k > 1 ? ct[o + 1] : 0x7fffffff;
+    pos[li] = 1;                          // list index of the entry in nv
+  }
+  out_v = kNegInf;
+  out_t = 0x7fffffff;
+  for (int r = 0; r < k; ++r) {
+    float bv = hv[0];
+    int bt = ht[0], bl = 0;
+#pragma unroll
+    for (int li = 1; li < L; ++li) {
+      const bool b = cand_better(hv[li], ht[li], bv, bt);
+      bv = b ? hv[li] : bv;
+      bt = b ? ht[li] : bt;
+      bl = b ? li : bl;
+    }
+    float wv = bv;
+    int wt = bt, wl = lane;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ov = __shfl_xor_sync(kFull, wv, o);
+      const int ot = __shfl_xor_sync(kFull, wt, o);
+      const int ol = __shfl_xor_sync(kFull, wl, o);
+      const bool take = cand_better(ov, ot, wv, wt) | ((ov == wv) & (ot == wt) & (ol < wl));
+      wv = take ? ov : wv;
+      wt = take ? ot : wt;
+      wl = take ? ol : wl;
+    }
+    if (lane == r) {
+      out_v = wv;
+      out_t = wt;
+    }
+    if (lane == wl) {
+#pragma unroll
+      for (int li = 0; li < L; ++li) {
+        if (li == bl) {
+          const size_t o = static_cast<size_t>(lane + 32 * li) * k;
+          hv[li] = nv[li];
+          ht[li] = nt[li];
+          ++pos[li];
+          const bool more = pos[li] < k;
+          nv[li] = more ? cz[o + pos[li]] : kNegInf;
+          nt[li] = more ? ct[o + pos[li]] : 0x7fffffff;
+        }
+      }
+    }
+  }
+}
+
+// The same result for any number of lists: every lane offers its candidates
+// that beat the list's k-th entry, after a seed from each lane's best of the
+// first batch.
+__device__ __forceinline__ void merge_lists_scan(const float* __restrict__ cz,
+                                                 const int32_t* __restrict__ ct,
+                                                 int n_cand, int k, float& out_v,
+                                                 int& out_t) {
+  const int lane = threadIdx.x & 31;
+  WarpList lst;
+  lst.reset();
+  for (int c0 = 0; c0 < n_cand; c0 += 32 * kUnroll) {
+    float cv[kUnroll];
+    int ci[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int c = c0 + u * 32 + lane;
+      cv[u] = c < n_cand ? cz[c] : kNegInf;
+      ci[u] = c < n_cand ? ct[c] : 0x7fffffff;
+    }
+    unsigned skip = 0;
+    if (c0 == 0) {
+      float bv = cv[0];
+      int bi = ci[0], bu = 0;
+#pragma unroll
+      for (int u = 1; u < kUnroll; ++u) {
+        const bool b = cand_better(cv[u], ci[u], bv, bi);
+        bv = b ? cv[u] : bv;
+        bi = b ? ci[u] : bi;
+        bu = b ? u : bu;
+      }
+      lst.seed(bv, bi, k);
+      skip = 1u << bu;
+    }
+    const float tv = __shfl_sync(kFull, lst.v, k - 1);
+    const int tt = __shfl_sync(kFull, lst.t, k - 1);
+    unsigned marks = 0;
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u)
+      marks |= static_cast<unsigned>(cand_better(cv[u], ci[u], tv, tt)) << u;
+    marks &= ~skip;
+    while (__any_sync(kFull, marks != 0)) {
+      const int sel = marks != 0 ? __ffs(marks) - 1 : -1;
+      marks &= marks - 1;
+      const float ov = sel >= 0 ? pick(cv, sel) : kNegInf;
+      const int ot = sel >= 0 ? pick(ci, sel) : 0x7fffffff;
+      lst.offer(ov, ot, k);
+    }
+  }
+  out_v = lst.v;
+  out_t = lst.t;
+}
+
+constexpr int kMergeThreads = 1024;
+
+__global__ void __launch_bounds__(kMergeThreads)
 merge_kernel(int d, int B, int k, int b_d, int rpq, int shared, int V, int H,
              int P, int n_chunks,
              int x_elem, const float* __restrict__ part_m,
@@ -257,7 +382,14 @@ merge_kernel(int d, int B, int k, int b_d, int rpq, int shared, int V, int H,
   const int r = blockIdx.x;
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
-  extern __shared__ unsigned long long sm_keys[];  // b_d * k layer keys
+  // launched while the stage's projection finishes: wait for it before
+  // reading its partials; the next stage's projection may launch meanwhile
+  pdl_launch_dependents();
+  pdl_wait();
+  // the layer's b_d * k (score, id) keys, then their tokens
+  extern __shared__ unsigned long long sm_keys[];
+  int* sm_ctok = reinterpret_cast<int*>(sm_keys + b_d * k);
+  __shared__ float sm_lse[32];
   __shared__ int sm_tok[PCTREE_MAX_K];
   __shared__ int sm_chain;
 
@@ -267,79 +399,73 @@ merge_kernel(int d, int B, int k, int b_d, int rpq, int shared, int V, int H,
   int32_t* fr = front + static_cast<size_t>(r) * k;
   const int base = level_base(d + 1, k);
 
-  // one warp per Markov row: a frontier slot (PCTree) or the chain parent
-  // (Shared-Markov, rpq = 1)
-  if (warp < rpq) {
-    const int j = warp;
-    const int row = r * rpq + j;
-    const size_t p0 = static_cast<size_t>(row) * n_chunks;
+  // Warp j < rpq takes Markov row j of the request (a frontier slot, or the
+  // chain parent of the Shared-Markov control, rpq = 1): its children; warp
+  // rpq + j, when there is one, meanwhile the row's normaliser.
+  const int n_warps = kMergeThreads / 32;
+  const bool lse_apart = 2 * rpq <= n_warps;
+  if (lse_apart && warp >= rpq && warp < 2 * rpq) {
+    const size_t p0 = static_cast<size_t>(r * rpq + warp - rpq) * n_chunks;
     // log-softmax normaliser from the chunk partials (Eq. 2)
-    const float lse = warp_lse_from_partials<kUnroll>(part_m + p0, part_s + p0,
-                                                      n_chunks);
-    if (lse == kNegInf && lane == 0) set_status(status, PCTREE_ERR_NONFINITE);
+    const float lse = warp_lse_from_partials<kUnroll>(part_m + p0, part_s + p0, n_chunks);
+    if (lane == 0) sm_lse[warp - rpq] = lse;
+  }
+  float cv = kNegInf;
+  int cv_t = 0x7fffffff;
+  const int j = warp;
+  // the parent of slot j and its score, loaded before they are needed
+  int pid = 0;
+  float2 spid = make_float2(0.0f, 0.0f);
+  if (j < rpq && !shared) {
+    pid = fr[j];
+    spid = sc[pid];
+  }
+  if (j < rpq) {
+    const size_t p0 = static_cast<size_t>(r * rpq + j) * n_chunks;
+    if (!lse_apart) {
+      const float lse = warp_lse_from_partials<kUnroll>(part_m + p0, part_s + p0, n_chunks);
+      if (lane == 0) sm_lse[j] = lse;
+    }
     // top-k children of this parent over every chunk's list
-    WarpList lst;
-    lst.reset();
-    const int n_cand = n_chunks * k;
     const float* cz = part_z + p0 * k;
     const int32_t* ct = part_t + p0 * k;
-    for (int c0 = 0; c0 < n_cand; c0 += 32 * kUnroll) {
-      float cv[kUnroll];
-      int ci[kUnroll];
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
-        const int c = c0 + u * 32 + lane;
-        cv[u] = c < n_cand ? cz[c] : kNegInf;
-        ci[u] = c < n_cand ? ct[c] : 0x7fffffff;
-      }
-      // The first batch seeds the list with each lane's best candidate (one
-      // sort); then every lane offers, one at a time, only its candidates
-      // that beat the list's k-th entry.
-      unsigned skip = 0;
-      if (c0 == 0) {
-        float bv = cv[0];
-        int bi = ci[0], bu = 0;
-#pragma unroll
-        for (int u = 1; u < kUnroll; ++u) {
-          const bool b = cand_better(cv[u], ci[u], bv, bi);
-          bv = b ? cv[u] : bv;
-          bi = b ? ci[u] : bi;
-          bu = b ? u : bu;
-        }
-        lst.seed(bv, bi, k);
-        skip = 1u << bu;
-      }
-      const float tv = __shfl_sync(kFull, lst.v, k - 1);
-      const int tt = __shfl_sync(kFull, lst.t, k - 1);
-      unsigned marks = 0;
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u)
-        marks |= static_cast<unsigned>(cand_better(cv[u], ci[u], tv, tt)) << u;
-      marks &= ~skip;
-      while (__any_sync(kFull, marks != 0)) {
-        const int sel = marks != 0 ? __ffs(marks) - 1 : -1;
-        marks &= marks - 1;
-        const float ov = sel >= 0 ? pick(cv, sel) : kNegInf;
-        const int ot = sel >= 0 ? pick(ci, sel) : 0x7fffffff;
-        lst.offer(ov, ot, k);
-      }
+    switch ((n_chunks + 31) / 32) {
+      case 1: merge_sorted_lists<1>(cz, ct, n_chunks, k, cv, cv_t); break;
+      case 2: merge_sorted_lists<2>(cz, ct, n_chunks, k, cv, cv_t); break;
+      case 3: merge_sorted_lists<3>(cz, ct, n_chunks, k, cv, cv_t); break;
+      case 4: merge_sorted_lists<4>(cz, ct, n_chunks, k, cv, cv_t); break;
+      case 5: merge_sorted_lists<5>(cz, ct, n_chunks, k, cv, cv_t); break;
+      default: merge_lists_scan(cz, ct, n_chunks * k, k, cv, cv_t); break;
     }
-    int t = lst.t;
-    float logpi = lst.v - lse;
+  }
+  __syncthreads();
+  if (j < rpq) {
+    const float lse = sm_lse[j];
+    if (lse == kNegInf && lane == 0) set_status(status, PCTREE_ERR_NONFINITE);
+    int t = cv_t;
+    float logpi = cv - lse;
     if (t < 0 || t >= V) {  // only when V < k (rejected on the host)
       t = 0;
       logpi = kNegInf;
     }
     // PCTree: the row's children belong to slot j; Shared-Markov: the chain
     // row's children go to every slot of the request.
+    // The layer's keys and tokens also go to shared memory for the
+    // frontier below.
     const int j_lo = shared ? 0 : j, j_hi = shared ? b_d : j + 1;
     for (int jj = j_lo; jj < j_hi; ++jj) {
-      const int pid = fr[jj];
+      const int p = shared ? fr[jj] : pid;
+      const float2 sp = shared ? sc[p] : spid;
       if (lane < k) {
         const int id = base + jj * k + lane;
+        const float2 s_id = ff_add(sp, logpi);  // Eq. 4: s(child) = s(p) + log pi
         tok[id] = t;
-        par[id] = pid;
-        sc[id] = ff_add(sc[pid], logpi);  // Eq. 4: s(child) = s(p) + log pi
+        par[id] = p;
+        sc[id] = s_id;
+        sm_keys[jj * k + lane] =
+            (static_cast<unsigned long long>(desc_key(s_id.x)) << 32) |
+            static_cast<unsigned int>(id);
+        sm_ctok[jj * k + lane] = t;
       }
     }
     const int top = __shfl_sync(kFull, t, 0);
@@ -350,18 +476,12 @@ merge_kernel(int d, int B, int k, int b_d, int rpq, int shared, int V, int H,
   // frontier: the k best nodes of this layer by (score desc, id asc)
   const int n_layer = b_d * k;
   for (int i = threadIdx.x; i < n_layer; i += blockDim.x) {
-    const int id = base + i;
-    sm_keys[i] = (static_cast<unsigned long long>(desc_key(sc[id].x)) << 32) |
-                 static_cast<unsigned int>(id);
-  }
-  __syncthreads();
-  for (int i = threadIdx.x; i < n_layer; i += blockDim.x) {
     const unsigned long long key = sm_keys[i];
     int rank = 0;
     for (int j = 0; j < n_layer; ++j) rank += sm_keys[j] < key;
     if (rank < k) {
       fr[rank] = base + i;
-      sm_tok[rank] = tok[base + i];
+      sm_tok[rank] = sm_ctok[i];
     }
   }
   __syncthreads();
@@ -690,9 +810,24 @@ cudaError_t launch_merge(const pctree_config& c, const Layout& lay, int d,
                          int32_t* status, cudaStream_t stream) {
   const int b_d = d == 0 ? 1 : c.k;
   const int rpq = rows_per_request(c, d);
-  const size_t smem = static_cast<size_t>(b_d) * c.k * sizeof(unsigned long long);
-  const int threads = rpq * 32 > 256 ? rpq * 32 : 256;
-  merge_kernel<<<c.batch, threads, smem, stream>>>(
+  const size_t smem =
+      static_cast<size_t>(b_d) * c.k * (sizeof(unsigned long long) + sizeof(int));
+  // 1024 threads: the normalisers beside the children, and the next stage's
+  // rows gathered with every load of a row in flight.  Programmatic
+  // dependent launch: scheduled while the projection finishes (the kernel
+  // waits for it before touching memory).
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(c.batch);
+  cfg.blockDim = dim3(kMergeThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(
+      &cfg, merge_kernel,
       d, c.B, c.k, b_d, rpq, c.mode == PCTREE_MODE_SHARED ? 1 : 0, c.V, c.H,
       lay.P, n_parts, lay.x_elem,
       reinterpret_cast<const float*>(ws + lay.off_pm),
@@ -704,7 +839,6 @@ cudaError_t launch_merge(const pctree_config& c, const Layout& lay, int d,
       reinterpret_cast<float2*>(ws + lay.off_pool_s),
       reinterpret_cast<int32_t*>(ws + lay.off_front), E_in, ws + lay.off_x,
       status);
-  return cudaGetLastError();
 }
 
 cudaError_t launch_pack(const pctree_config& c, const Layout& lay,

@@ -428,4 +428,19 @@ __device__ __forceinline__ void named_barrier(int id, int count) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
+// Programmatic dependent launch.  A kernel launched with programmatic
+// stream serialization may start while the kernel before it in the stream
+// is still running; griddepcontrol.wait returns once that kernel has
+// completed and its memory operations are visible, so every access that
+// depends on it (reads of what it wrote, writes of what it reads) comes
+// after the wait.  launch_dependents lets the next such kernel launch once
+// every CTA of this one has issued it (or exited).  Both are no-ops for a
+// kernel launched without the attribute.
+__device__ __forceinline__ void pdl_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 }  // namespace pct
