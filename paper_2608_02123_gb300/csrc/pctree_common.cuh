@@ -187,6 +187,97 @@ struct WarpList {
   }
 };
 
+// The k best of one row's sorted candidate lists (one per projection CTA or
+// vocabulary chunk, each best first; list i at cz / ct + i * k), by a
+// tournament: lane l owns lists l, l + 32, ..., holding each one's head and
+// next entry in registers; each of k rounds takes the warp's best head
+// ((value desc, token asc), the lane breaking exact ties of padding) and
+// advances that list.  Lane r ends with the r-th best entry.  For at most
+// 32 * L lists.  load() issues the first loads, so that other independent
+// loads can go out before run() needs them.  The lists are read through L2
+// (__ldcg): another CTA of a running kernel may have written them.
+template <int L>
+struct ListTournament {
+  float hv[L], nv[L];
+  int ht[L], nt[L], pos[L];
+  const float* cz;
+  const int32_t* ct;
+  int k;
+  __device__ __forceinline__ void load(const float* cz_, const int32_t* ct_, int n_lists,
+                                       int k_) {
+    cz = cz_;
+    ct = ct_;
+    k = k_;
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int li = 0; li < L; ++li) {
+      const int id = lane + 32 * li;
+      const bool ok = id < n_lists;
+      const size_t o = static_cast<size_t>(ok ? id : 0) * k;
+      hv[li] = ok ? __ldcg(cz + o) : -INFINITY;
+      ht[li] = ok ? __ldcg(ct + o) : 0x7fffffff;
+      nv[li] = ok && k > 1 ? __ldcg(cz + o + 1) : -INFINITY;
+      nt[li] = ok && k > 1 ? __ldcg(ct + o + 1) : 0x7fffffff;
+      pos[li] = 1;                        // list index of the entry in nv
+    }
+  }
+  __device__ __forceinline__ void run(float& out_v, int& out_t) {
+    const int lane = threadIdx.x & 31;
+    out_v = -INFINITY;
+    out_t = 0x7fffffff;
+    for (int r = 0; r < k; ++r) {
+      float bv = hv[0];
+      int bt = ht[0], bl = 0;
+#pragma unroll
+      for (int li = 1; li < L; ++li) {
+        const bool b = cand_better(hv[li], ht[li], bv, bt);
+        bv = b ? hv[li] : bv;
+        bt = b ? ht[li] : bt;
+        bl = b ? li : bl;
+      }
+      float wv = bv;
+      int wt = bt, wl = lane;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float ov = __shfl_xor_sync(kFull, wv, o);
+        const int ot = __shfl_xor_sync(kFull, wt, o);
+        const int ol = __shfl_xor_sync(kFull, wl, o);
+        const bool take = cand_better(ov, ot, wv, wt) | ((ov == wv) & (ot == wt) & (ol < wl));
+        wv = take ? ov : wv;
+        wt = take ? ot : wt;
+        wl = take ? ol : wl;
+      }
+      if (lane == r) {
+        out_v = wv;
+        out_t = wt;
+      }
+      if (lane == wl) {
+#pragma unroll
+        for (int li = 0; li < L; ++li) {
+          if (li == bl) {
+            const size_t o = static_cast<size_t>(lane + 32 * li) * k;
+            hv[li] = nv[li];
+            ht[li] = nt[li];
+            ++pos[li];
+            const bool more = pos[li] < k;
+            nv[li] = more ? __ldcg(cz + o + pos[li]) : -INFINITY;
+            nt[li] = more ? __ldcg(ct + o + pos[li]) : 0x7fffffff;
+          }
+        }
+      }
+    }
+  }
+};
+
+template <int L>
+__device__ __forceinline__ void merge_sorted_lists(const float* cz, const int32_t* ct,
+                                                   int n_lists, int k, float& out_v,
+                                                   int& out_t) {
+  ListTournament<L> tr;
+  tr.load(cz, ct, n_lists, k);
+  tr.run(out_v, out_t);
+}
+
 // Online (max, sum exp) pair; m = -inf means "no finite value yet".  The
 // terms exp(x), x <= 0, use the fast exponential: its relative error (a few
 // 1e-7) stays far below the 1e-4 tolerance on log-probabilities.

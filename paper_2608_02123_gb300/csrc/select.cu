@@ -245,77 +245,6 @@ __device__ void gather_rows(const void* E_in, void* X, const int* tok,
   }
 }
 
-// The k best of one row's sorted candidate lists (one per projection CTA or
-// vocabulary chunk, each best first), by a tournament: lane l owns lists
-// l, l + 32, ..., holding each one's head and next entry in registers; each
-// of k rounds takes the warp's best head ((value desc, token asc), the lane
-// breaking exact ties of padding) and advances that list.  Lane r ends with
-// the r-th best entry.  For at most 32 * L lists (L <= 5 fits the
-// register budget of a 1024-thread block; more lists take the scan below).
-template <int L>
-__device__ __forceinline__ void merge_sorted_lists(const float* __restrict__ cz,
-                                                   const int32_t* __restrict__ ct,
-                                                   int n_lists, int k, float& out_v,
-                                                   int& out_t) {
-  const int lane = threadIdx.x & 31;
-  float hv[L], nv[L];
-  int ht[L], nt[L], pos[L];
-#pragma unroll
-  for (int li = 0; li < L; ++li) {
-    const int id = lane + 32 * li;
-    const bool ok = id < n_lists;
-    const size_t o = static_cast<size_t>(ok ? id : 0) * k;
-    hv[li] = ok ? cz[o] : kNegInf;
-    ht[li] = ok ? ct[o] : 0x7fffffff;
-    nv[li] = ok && k > 1 ? cz[o + 1] : kNegInf;
-    nt[li] = ok && k > 1 ? ct[o + 1] : 0x7fffffff;
-    pos[li] = 1;                          // list index of the entry in nv
-  }
-  out_v = kNegInf;
-  out_t = 0x7fffffff;
-  for (int r = 0; r < k; ++r) {
-    float bv = hv[0];
-    int bt = ht[0], bl = 0;
-#pragma unroll
-    for (int li = 1; li < L; ++li) {
-      const bool b = cand_better(hv[li], ht[li], bv, bt);
-      bv = b ? hv[li] : bv;
-      bt = b ? ht[li] : bt;
-      bl = b ? li : bl;
-    }
-    float wv = bv;
-    int wt = bt, wl = lane;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float ov = __shfl_xor_sync(kFull, wv, o);
-      const int ot = __shfl_xor_sync(kFull, wt, o);
-      const int ol = __shfl_xor_sync(kFull, wl, o);
-      const bool take = cand_better(ov, ot, wv, wt) | ((ov == wv) & (ot == wt) & (ol < wl));
-      wv = take ? ov : wv;
-      wt = take ? ot : wt;
-      wl = take ? ol : wl;
-    }
-    if (lane == r) {
-      out_v = wv;
-      out_t = wt;
-    }
-    if (lane == wl) {
-#pragma unroll
-      for (int li = 0; li < L; ++li) {
-        if (li == bl) {
-          const size_t o = static_cast<size_t>(lane + 32 * li) * k;
-          hv[li] = nv[li];
-          ht[li] = nt[li];
-          ++pos[li];
-          const bool more = pos[li] < k;
-          nv[li] = more ? cz[o + pos[li]] : kNegInf;
-          nt[li] = more ? ct[o + pos[li]] : 0x7fffffff;
-        }
-      }
-    }
-  }
-}
-
 // The same result for any number of lists: every lane offers its candidates
 // that beat the list's k-th entry, after a seed from each lane's best of the
 // first batch.
@@ -426,7 +355,9 @@ merge_kernel(int d, int B, int k, int b_d, int rpq, int shared, int V, int H,
       const float lse = warp_lse_from_partials<kUnroll>(part_m + p0, part_s + p0, n_chunks);
       if (lane == 0) sm_lse[j] = lse;
     }
-    // top-k children of this parent over every chunk's list
+    // top-k children of this parent over every chunk's list (a tournament
+    // for up to 160 lists, which fits the register budget of a 1024-thread
+    // block; more lists take the scan)
     const float* cz = part_z + p0 * k;
     const int32_t* ct = part_t + p0 * k;
     switch ((n_chunks + 31) / 32) {
