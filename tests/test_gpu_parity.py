@@ -65,6 +65,19 @@ def test_small_parity(name, path):
     print(f"{name}/{path}: " + rep.summary())
 
 
+def test_many_chunks_merge_scan():
+    """An f32 head with more than 160 vocabulary chunks of 8192 logits: the
+    per-stage merge takes each row's children by its candidate scan, not by
+    the tournament over at most 5 lists per lane that every other case
+    uses."""
+    wl = WORKLOADS["tiny"].with_(V=1_320_000, H=16, B=3, k=4, N=12, batch=2, seed=27)
+    assert -(-wl.V // 8192) > 160
+    inp = draw_round(wl)
+    host = G.run_gpu(inp)
+    rep = G.compare(inp, host)
+    print("many_chunks_f32: " + rep.summary())
+
+
 def test_paths_agree_exactly_on_structure():
     inp = draw_round(SMALL["weak_head_bf16"])
     a = G.run_gpu(inp, path=0)
