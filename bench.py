@@ -58,6 +58,11 @@ def parse_args():
                          "round (a tree-attention layer and the compaction "
                          "at the 14B-shaped batch-32 shapes) that the default "
                          "line carries under 'around_round'")
+    ap.add_argument("--e2e-logits", default="host", choices=["host", "copy"],
+                    help="end-to-end leg: the kernels read each step's base "
+                         "logits from the pinned host buffer over the host "
+                         "link (host), or the step copies them into device "
+                         "memory first (copy)")
     ap.add_argument("--mode", default="parent", choices=["parent", "shared"],
                     help="child scoring: PCTree, or the Shared-Markov control")
     ap.add_argument("--sweep", action="store_true",
@@ -483,27 +488,26 @@ def run_ours(args, wl, rank, world, local_rank):
     # end to end through the public API: pinned host inputs in, tree out
     L_host = [torch.from_numpy(L).pin_memory() for L, _, _ in sets]
     root_host = [torch.from_numpy(root).pin_memory() for _, root, _ in sets]
-    out_names = ("n_nodes", "tokens", "parent", "depth", "logp",
-                 "position_ids", "mask", "retrieve", "n_leaves", "status")
-    out_host = {n: torch.empty_like(getattr(dr.tree, n), device="cpu").pin_memory()
-                for n in out_names}
-    acc_host = [torch.empty_like(t, device="cpu").pin_memory()
-                for t in (dr.accepted_idx, dr.accepted_len, dr.bonus)]
+    # the tree and the acceptance outputs share one device buffer: one copy
+    # brings every result back
+    out_host = torch.empty(dr.tree.blob.shape, dtype=torch.uint8, pin_memory=True)
     h2d = L_host[0].numel() * 4 + root_host[0].numel() * 4
-    d2h = sum(t.numel() * t.element_size() for t in out_host.values()) + \
-        sum(t.numel() * t.element_size() for t in acc_host)
+    d2h = out_host.numel()
     L_stage = torch.empty_like(L_dev[0])
     root_stage = torch.empty_like(root_dev[0])
+    zero_copy = args.e2e_logits == "host"
 
     def e2e_step(i):
-        L_stage.copy_(L_host[i % n_sets], non_blocking=True)
-        root_stage.copy_(root_host[i % n_sets], non_blocking=True)
-        dr.draft(L_stage, E, W, root_stage, stream)
+        if zero_copy:
+            # the kernels read the pinned host inputs as they need them
+            L_in, root_in = L_host[i % n_sets], root_host[i % n_sets]
+        else:
+            L_stage.copy_(L_host[i % n_sets], non_blocking=True)
+            root_stage.copy_(root_host[i % n_sets], non_blocking=True)
+            L_in, root_in = L_stage, root_stage
+        dr.draft(L_in, E, W, root_in, stream)
         dr.accept(target_of(i), stream)
-        for n in out_names:
-            out_host[n].copy_(getattr(dr.tree, n), non_blocking=True)
-        for h, t in zip(acc_host, (dr.accepted_idx, dr.accepted_len, dr.bonus)):
-            h.copy_(t, non_blocking=True)
+        out_host.copy_(dr.tree.blob, non_blocking=True)
         stream.synchronize()   # the caller reads the tree before the next round
 
     for i in range(3):
@@ -582,7 +586,14 @@ def run_ours(args, wl, rank, world, local_rank):
                          f"property of the input generator, not of a model)",
         "e2e": {"value": job_rounds_per_s(e2e_ms, args.steps, world, wl.batch),
                 "unit": "rounds/s",
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "inputs": ("base logits and root tokens in pinned host memory, "
+                           "read by the kernels over the host link as they need "
+                           "them (no copy)" if zero_copy else
+                           "base logits and root tokens copied to device memory "
+                           "each step (cudaMemcpyAsync)"),
+                "outputs": "tree and acceptance results in one device buffer, "
+                           "one copy back per step"},
         "gpu_launches": kernels_per_step * args.steps,
         "clocks": clk,
     }

@@ -179,6 +179,11 @@ PCTREE_API size_t pctree_workspace_bytes(const pctree_config* cfg);
  * One PCTree drafting round (Algorithm 1; Eqs. 2-4; Sec. 4.2; Appendix A).
  *   base_logits  [batch][B][V] float32: the backbone's shared logits L_d per
  *                request (Sec. 3.2 "Parallel backbone"); -inf allowed.
+ *                Device memory, or page-locked host memory that CUDA maps
+ *                into the device's address space (cudaHostAlloc,
+ *                cudaHostRegister): the kernels then read it over the host
+ *                link as each stage needs it, and no copy is made.  Any
+ *                other host pointer: PCTREE_ERR_INVALID_ARG.
  *   head_emb     [V][H] E_in  (weight_dtype), 16-byte aligned: Markov-head
  *                input rows, one per parent token.
  *   head_out     W_out (weight_dtype), 16-byte aligned, [V][H] or tiled as
@@ -187,7 +192,8 @@ PCTREE_API size_t pctree_workspace_bytes(const pctree_config* cfg);
  *                Markov(p)[v] = sum_h W_out[v][h] * E_in[p][h] (Sec. 3.2,
  *                "low-rank Markov head"), accumulated in float32.
  *   root_token   [batch] int32: the last verified token x_t of each request;
- *                out of range -> status PCTREE_ERR_INVALID_ARG.
+ *                out of range -> status PCTREE_ERR_INVALID_ARG.  Device
+ *                memory or mapped page-locked host memory, as base_logits.
  *   out          output tensors (see pctree_tree); all non-optional pointers
  *                required.
  *   workspace    device scratch of at least pctree_workspace_bytes(cfg)

@@ -21,6 +21,28 @@ bool aligned(const void* p, size_t a) {
   return (reinterpret_cast<uintptr_t>(p) % a) == 0;
 }
 
+// Memory the kernels may read through `p`: device or managed memory, or
+// page-locked host memory mapped into the device's address space at the same
+// address (the kernels then read it over the host link, with no copy).
+// Pageable host memory the driver does not know is refused, so that no
+// kernel faults on it.
+bool device_readable(const void* p) {
+  cudaPointerAttributes at{};
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return false;
+  }
+  switch (at.type) {
+    case cudaMemoryTypeDevice:
+    case cudaMemoryTypeManaged:
+      return true;
+    case cudaMemoryTypeHost:
+      return at.devicePointer == p;
+    default:
+      return false;
+  }
+}
+
 pctree_status check_config(const pctree_config* c) {
   if (c == nullptr) return PCTREE_ERR_INVALID_ARG;
   if (c->V < 1 || c->H < 1 || c->B < 1 || c->k < 1 || c->N < 1 ||
@@ -358,6 +380,8 @@ pctree_status pctree_draft(const pctree_config* cfg, const float* base_logits,
   int num_sms = 0;
   st = device_facts(&num_sms);
   if (st != PCTREE_OK) return st;
+  if (!device_readable(base_logits) || !device_readable(root_token))
+    return PCTREE_ERR_INVALID_ARG;
 
   cudaStream_t stream = static_cast<cudaStream_t>(stream_ptr);
   unsigned char* ws = static_cast<unsigned char*>(workspace);

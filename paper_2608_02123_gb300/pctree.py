@@ -8,6 +8,7 @@ library is missing, importing this module raises -- there is no fallback.
 from __future__ import annotations
 
 import ctypes
+import math
 import dataclasses
 import os
 from typing import Dict, Optional
@@ -215,22 +216,45 @@ class Tree:
                 for f in dataclasses.fields(self)}
 
 
-def alloc_tree(cfg: Config, device, with_pool: bool = False) -> Tree:
+def _carve(device, specs):
+    """Tensors of the given (name, shape, dtype) as views of one device
+    buffer, each starting on a 256-byte boundary: a caller reads them all
+    back with one copy.  Returns (buffer, {name: tensor})."""
+    offs, off = [], 0
+    for name, shape, dt in specs:
+        n = math.prod(shape) * torch.empty(0, dtype=dt).element_size()
+        offs.append((name, off, n, shape, dt))
+        off = (off + n + 255) // 256 * 256
+    blob = torch.empty(max(off, 256), dtype=torch.uint8, device=device)
+    return blob, {name: blob[o:o + n].view(dt).view(*shape)
+                  for name, o, n, shape, dt in offs}
+
+
+def alloc_tree(cfg: Config, device, with_pool: bool = False, extra=()) -> Tree:
+    """The output tensors of a round, carved from one device buffer
+    (``tree.blob``) together with the ``extra`` (name, shape, dtype) tensors
+    (``tree.extra``), so that all of them come back with one copy."""
     R, N, B = cfg.batch, cfg.N, cfg.B
-    i32 = dict(dtype=torch.int32, device=device)
+    i32, f32, u8 = torch.int32, torch.float32, torch.uint8
     P = pctree_pool_capacity(cfg)
-    return Tree(
-        n_nodes=torch.empty(R, **i32), tokens=torch.empty(R, N, **i32),
-        parent=torch.empty(R, N, **i32), depth=torch.empty(R, N, **i32),
-        logp=torch.empty(R, N, dtype=torch.float32, device=device),
-        position_ids=torch.empty(R, N, **i32),
-        mask=torch.empty(R, N, N, dtype=torch.uint8, device=device),
-        retrieve=torch.empty(R, N, B + 1, **i32),
-        n_leaves=torch.empty(R, **i32), status=torch.empty(1, **i32),
-        pool_token=torch.empty(R, P, **i32) if with_pool else None,
-        pool_parent=torch.empty(R, P, **i32) if with_pool else None,
-        pool_logp=(torch.empty(R, P, dtype=torch.float32, device=device)
+    specs = [("n_nodes", (R,), i32), ("tokens", (R, N), i32),
+             ("parent", (R, N), i32), ("depth", (R, N), i32),
+             ("logp", (R, N), f32), ("position_ids", (R, N), i32),
+             ("mask", (R, N, N), u8), ("retrieve", (R, N, B + 1), i32),
+             ("n_leaves", (R,), i32), ("status", (1,), i32)] + list(extra)
+    blob, t = _carve(device, specs)
+    tree = Tree(
+        n_nodes=t["n_nodes"], tokens=t["tokens"], parent=t["parent"],
+        depth=t["depth"], logp=t["logp"], position_ids=t["position_ids"],
+        mask=t["mask"], retrieve=t["retrieve"], n_leaves=t["n_leaves"],
+        status=t["status"],
+        pool_token=torch.empty(R, P, dtype=i32, device=device) if with_pool else None,
+        pool_parent=torch.empty(R, P, dtype=i32, device=device) if with_pool else None,
+        pool_logp=(torch.empty(R, P, dtype=f32, device=device)
                    if with_pool else None))
+    tree.blob = blob
+    tree.extra = {name: t[name] for name, _, _ in extra}
+    return tree
 
 
 def alloc_workspace(cfg: Config, device) -> torch.Tensor:
@@ -246,15 +270,24 @@ def _stream_ptr(stream: Optional[torch.cuda.Stream]) -> int:
     return s.cuda_stream
 
 
+def _check_inputs(base_logits, head_emb, head_out, root_token) -> None:
+    for name, t in (("base_logits", base_logits), ("head_emb", head_emb),
+                    ("head_out", head_out), ("root_token", root_token)):
+        host_ok = name in ("base_logits", "root_token")
+        ok = t.is_cuda or (host_ok and t.is_pinned())
+        if not ok or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous CUDA tensor"
+                             + (" or a pinned CPU tensor" if host_ok else ""))
+
+
 def pctree_draft(cfg: Config, base_logits: torch.Tensor, head_emb: torch.Tensor,
                  head_out: torch.Tensor, root_token: torch.Tensor, tree: Tree,
                  workspace: torch.Tensor,
                  stream: Optional[torch.cuda.Stream] = None) -> None:
-    """Enqueue one drafting round (see pctree_draft in include/pctree.h)."""
-    for name, t in (("base_logits", base_logits), ("head_emb", head_emb),
-                    ("head_out", head_out), ("root_token", root_token)):
-        if not t.is_cuda or not t.is_contiguous():
-            raise ValueError(f"{name} must be a contiguous CUDA tensor")
+    """Enqueue one drafting round (see pctree_draft in include/pctree.h).
+    base_logits and root_token may also be pinned CPU tensors: the kernels
+    read them over the host link."""
+    _check_inputs(base_logits, head_emb, head_out, root_token)
     ts = tree.c_struct()
     rc = LIB.pctree_draft(ctypes.byref(cfg), base_logits.data_ptr(),
                           head_emb.data_ptr(), head_out.data_ptr(),
@@ -273,10 +306,7 @@ def pctree_draft_noalloc(cfg: Config, base_logits: torch.Tensor,
     16 MiB device array serves as scratch, for callers that cannot allocate
     device memory when they draft (see pctree_draft_noalloc in
     include/pctree.h)."""
-    for name, t in (("base_logits", base_logits), ("head_emb", head_emb),
-                    ("head_out", head_out), ("root_token", root_token)):
-        if not t.is_cuda or not t.is_contiguous():
-            raise ValueError(f"{name} must be a contiguous CUDA tensor")
+    _check_inputs(base_logits, head_emb, head_out, root_token)
     ts = tree.c_struct()
     rc = LIB.pctree_draft_noalloc(ctypes.byref(cfg), base_logits.data_ptr(),
                                   head_emb.data_ptr(), head_out.data_ptr(),
@@ -426,11 +456,14 @@ class Drafter:
         self.cfg = cfg
         self.device = torch.device(device)
         self.workspace = alloc_workspace(cfg, self.device)
-        self.tree = alloc_tree(cfg, self.device, with_pool)
-        i32 = dict(dtype=torch.int32, device=self.device)
-        self.accepted_idx = torch.empty(cfg.batch, cfg.B + 1, **i32)
-        self.accepted_len = torch.empty(cfg.batch, **i32)
-        self.bonus = torch.empty(cfg.batch, **i32)
+        # the acceptance outputs share the tree's buffer (one copy back)
+        self.tree = alloc_tree(cfg, self.device, with_pool, extra=(
+            ("accepted_idx", (cfg.batch, cfg.B + 1), torch.int32),
+            ("accepted_len", (cfg.batch,), torch.int32),
+            ("bonus", (cfg.batch,), torch.int32)))
+        self.accepted_idx = self.tree.extra["accepted_idx"]
+        self.accepted_len = self.tree.extra["accepted_len"]
+        self.bonus = self.tree.extra["bonus"]
 
     def draft(self, base_logits, head_emb, head_out, root_token, stream=None):
         pctree_draft(self.cfg, base_logits, head_emb, head_out, root_token,
@@ -451,17 +484,25 @@ class Drafter:
                         root_host: torch.Tensor, head_emb, head_out,
                         stream=None):
         """End-to-end call a serving loop makes: pinned host inputs in, packed
-        tree back on the host.  Returns the host tree arrays."""
+        tree back on the host.  The kernels read the base logits and root
+        tokens from the pinned host buffers as they need them (no copy); the
+        outputs come back with one copy of the tree's buffer.  Returns the
+        host tree arrays."""
         s = stream if stream is not None else torch.cuda.current_stream()
+        blob = torch.empty(self.tree.blob.shape, dtype=torch.uint8, pin_memory=True)
         with torch.cuda.stream(s):
-            L = base_logits_host.to(self.device, non_blocking=True)
-            root = root_host.to(self.device, non_blocking=True)
-            self.draft(L, head_emb, head_out, root, s)
-            host = {name: getattr(self.tree, name).to("cpu", non_blocking=True)
-                    for name in ("n_nodes", "tokens", "parent", "depth",
-                                 "logp", "position_ids", "mask", "retrieve",
-                                 "n_leaves", "status")}
+            self.draft(base_logits_host, head_emb, head_out, root_host, s)
+            blob.copy_(self.tree.blob, non_blocking=True)
         s.synchronize()
+        names = ("n_nodes", "tokens", "parent", "depth", "logp", "position_ids",
+                 "mask", "retrieve", "n_leaves", "status")
+        base = self.tree.blob.data_ptr()
+        host = {}
+        for name in names:
+            t = getattr(self.tree, name)
+            o = t.data_ptr() - base
+            n = t.numel() * t.element_size()
+            host[name] = blob[o:o + n].view(t.dtype).view(t.shape).numpy()
         return host
 
 

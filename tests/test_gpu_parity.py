@@ -168,6 +168,63 @@ def test_host_errors_need_no_work():
     assert ei.value.code == -1
 
 
+@pytest.mark.parametrize("path", sorted(PATHS))
+@pytest.mark.parametrize("name", ["ragged_V_bf16", "multipass_bf16", "tiny_f32"])
+def test_base_logits_in_pinned_host_memory(name, path):
+    """Base logits and root tokens in page-locked host memory are read by
+    the kernels over the host link, with no copy: the round is the same, bit
+    for bit, as from device memory (also through draft_from_host, which
+    reads all outputs back with one copy)."""
+    from paper_2608_02123_gb300 import pctree as P
+    inp = draw_round(SMALL[name])
+    wl = inp.wl
+    cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, inp.L.shape[0],
+                        wl.pos_offset, wl.weight_dtype, wl.mode)
+    L, E, W, root = G.device_inputs(inp)
+    L_pinned = L.cpu().pin_memory()
+    root_pinned = root.cpu().pin_memory()
+    assert L_pinned.is_pinned() and root_pinned.is_pinned()
+    P.pctree_set_path(PATHS[path])
+    try:
+        a = P.Drafter(cfg)
+        ha = a.draft(L, E, W, root).to_host()
+        b = P.Drafter(cfg)
+        hb = b.draft(L_pinned, E, W, root_pinned).to_host()
+        torch.cuda.synchronize()
+        c = P.Drafter(cfg)
+        hc = c.draft_from_host(L_pinned, root_pinned, E, W)
+    finally:
+        P.pctree_set_path(P.PATH_AUTO)
+    a.check_status()
+    b.check_status()
+    for key in ha:
+        np.testing.assert_array_equal(ha[key], hb[key], err_msg=key)
+        if key in hc:
+            np.testing.assert_array_equal(ha[key], hc[key], err_msg=key)
+
+
+def test_pageable_base_logits_refused():
+    """A host pointer CUDA cannot read from the device is refused on the
+    host, before any launch."""
+    import ctypes
+    from paper_2608_02123_gb300 import pctree as P
+    wl = SMALL["ragged_V_bf16"]
+    cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, wl.batch)
+    dr = P.Drafter(cfg)
+    _, E, W, root = G.device_inputs(draw_round(wl))
+    pageable = np.zeros((wl.batch, wl.B, wl.V), np.float32)
+    ts = dr.tree.c_struct()
+    rc = P.LIB.pctree_draft(ctypes.byref(cfg), ctypes.c_void_p(pageable.ctypes.data),
+                            E.data_ptr(), W.data_ptr(), root.data_ptr(),
+                            ctypes.byref(ts), dr.workspace.data_ptr(),
+                            dr.workspace.numel(),
+                            torch.cuda.current_stream().cuda_stream)
+    assert rc == -1
+    with pytest.raises(ValueError):
+        P.pctree_draft(cfg, torch.from_numpy(pageable), E, W, root, dr.tree,
+                       dr.workspace)
+
+
 # ---------------------------------------------------------------------------
 # full-size Qwen3-shaped workloads
 # ---------------------------------------------------------------------------
