@@ -50,6 +50,9 @@ constexpr int kCC = 64;           // accumulator columns per transpose chunk
 constexpr int kRowsPerWarp = kCC / kEpiWarps;
 constexpr int kCand = 16;         // compacted candidates per row and round
 constexpr int kRegList = 16;      // k up to this: a row's list in registers
+// the register lists are spread four lanes per row, four entries per lane
+static_assert(kRowsPerWarp * 4 == 32 && kRegList == 4 * 4,
+              "four lanes per row and four entries per lane");
 constexpr int kMaxStages = 8;
 constexpr int kSmemLimit = 227 * 1024;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per bounded wait

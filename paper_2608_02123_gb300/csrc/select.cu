@@ -245,9 +245,10 @@ __device__ void gather_rows(const void* E_in, void* X, const int* tok,
   }
 }
 
-// The same result for any number of lists: every lane offers its candidates
-// that beat the list's k-th entry, after a seed from each lane's best of the
-// first batch.
+// The k best of a row's candidate lists (n_cand entries, list after list)
+// for any number of lists, where merge_sorted_lists would need more than 5
+// lists per lane: every lane offers its candidates that beat the warp list's
+// k-th entry, after a seed from each lane's best of the first batch.
 __device__ __forceinline__ void merge_lists_scan(const float* __restrict__ cz,
                                                  const int32_t* __restrict__ ct,
                                                  int n_cand, int k, float& out_v,
