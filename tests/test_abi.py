@@ -155,3 +155,31 @@ def test_tiled_head_layout_config(P):
     # ceil(V/128) * ceil(H/64) blocks of 128 x 64 bf16
     assert P.pctree_packed_head_bytes(mk(151936, 2560, 16, 8, 64)) == 1187 * 40 * 128 * 64 * 2
     assert P.pctree_packed_head_bytes(mk(3000, 72, 2, 2, 4)) == 24 * 2 * 128 * 64 * 2
+
+
+def test_outputs_share_one_buffer(P):
+    """The round's outputs and any extra tensors are views of one buffer,
+    each on a 256-byte boundary and disjoint, so that one copy brings all of
+    them back."""
+    import torch
+    cfg = P.make_config(1000, 64, 5, 4, 24, 3)
+    extra = (("accepted_idx", (3, 6), torch.int32), ("bonus", (3,), torch.int32))
+    tree = P.alloc_tree(cfg, "cpu", extra=extra)
+    base = tree.blob.data_ptr()
+    spans = []
+    for name in ("n_nodes", "tokens", "parent", "depth", "logp", "position_ids",
+                 "mask", "retrieve", "n_leaves", "status"):
+        t = getattr(tree, name)
+        spans.append((t.data_ptr() - base, t.numel() * t.element_size(), name))
+    for name, shape, dt in extra:
+        t = tree.extra[name]
+        assert tuple(t.shape) == shape and t.dtype == dt
+        spans.append((t.data_ptr() - base, t.numel() * t.element_size(), name))
+    assert tuple(tree.mask.shape) == (3, 24, 24) and tree.mask.dtype == torch.uint8
+    assert tuple(tree.retrieve.shape) == (3, 24, 6)
+    spans.sort()
+    for (o, n, name), (o2, _, name2) in zip(spans, spans[1:]):
+        assert o % 256 == 0, name
+        assert o + n <= o2, (name, name2)
+    o, n, name = spans[-1]
+    assert o % 256 == 0 and o + n <= tree.blob.numel()
