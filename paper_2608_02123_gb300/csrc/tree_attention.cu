@@ -309,6 +309,11 @@ tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
     T->abort = 0;
     fence_barrier_init();
   }
+  // programmatic dependent launch: the launch and the set-up above overlap
+  // the previous kernel of the stream; every global access (request sizes,
+  // Q, K, V, the output) comes after it is complete
+  pdl_launch_dependents();
+  pdl_wait();
   if (!ranked && (threadIdx.x == 0 || threadIdx.x == 32)) {
     const AttnItem it = item_facts(a, T, static_cast<int>(blockIdx.x), false, false);
     q_pre = it.nblk > 0;                 // known to the S issuer (thread 32) too
@@ -802,6 +807,10 @@ constexpr int kMergeRows = 16;
 
 __global__ void __launch_bounds__(kMergeThreads)
 tree_attn_merge_kernel(AttnArgs a) {
+  // launched while the attention kernel finishes: its partials are read
+  // after it is complete
+  pdl_launch_dependents();
+  pdl_wait();
   const int unit = blockIdx.x;
   const int row = blockIdx.y * kMergeRows + (threadIdx.x >> 3);   // tile row
   const int d0 = (threadIdx.x & 7) * 16;
@@ -1032,17 +1041,33 @@ pctree_status pctree_tree_attention(const pctree_attn_config* cfg, const void* q
       limit2.ensure(reinterpret_cast<const void*>(tree_attn_kernel<2>), attn_smem<2>()) !=
           cudaSuccess)
     return PCTREE_ERR_CUDA;
-  // persistent: one CTA per SM walks its share of the items
-  const dim3 grid(static_cast<unsigned>(a.items < num_sms ? a.items : num_sms));
-  if (g.tpc == 2)
-    tree_attn_kernel<2><<<grid, AttnCfg<2>::kThreads, attn_smem<2>(), stream>>>(tm_q, tm_k, tm_v, a);
-  else
-    tree_attn_kernel<1><<<grid, AttnCfg<1>::kThreads, attn_smem<1>(), stream>>>(tm_q, tm_k, tm_v, a);
-  if (cudaGetLastError() != cudaSuccess) return PCTREE_ERR_CUDA;
+  // persistent: one CTA per SM walks its share of the items; both kernels
+  // are launched with programmatic stream serialization (each waits for its
+  // predecessor before touching global memory)
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = dim3(static_cast<unsigned>(a.items < num_sms ? a.items : num_sms));
+  lc.stream = stream;
+  lc.attrs = attr;
+  lc.numAttrs = 1;
+  cudaError_t e;
+  if (g.tpc == 2) {
+    lc.blockDim = dim3(AttnCfg<2>::kThreads);
+    lc.dynamicSmemBytes = attn_smem<2>();
+    e = cudaLaunchKernelEx(&lc, tree_attn_kernel<2>, tm_q, tm_k, tm_v, a);
+  } else {
+    lc.blockDim = dim3(AttnCfg<1>::kThreads);
+    lc.dynamicSmemBytes = attn_smem<1>();
+    e = cudaLaunchKernelEx(&lc, tree_attn_kernel<1>, tm_q, tm_k, tm_v, a);
+  }
+  if (e != cudaSuccess) return PCTREE_ERR_CUDA;
   if (g.n_split > 1) {
-    const dim3 mgrid(static_cast<unsigned>(g.units), (g.R + kMergeRows - 1) / kMergeRows);
-    tree_attn_merge_kernel<<<mgrid, kMergeThreads, 0, stream>>>(a);
-    if (cudaGetLastError() != cudaSuccess) return PCTREE_ERR_CUDA;
+    lc.gridDim = dim3(static_cast<unsigned>(g.units), (g.R + kMergeRows - 1) / kMergeRows);
+    lc.blockDim = dim3(kMergeThreads);
+    lc.dynamicSmemBytes = 0;
+    if (cudaLaunchKernelEx(&lc, tree_attn_merge_kernel, a) != cudaSuccess) return PCTREE_ERR_CUDA;
   }
   return PCTREE_OK;
 }
