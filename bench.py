@@ -428,9 +428,11 @@ def run_ours(args, wl, rank, world, local_rank):
     cfg = P.make_config(wl.V, wl.H, wl.B, wl.k, wl.N, wl.batch, wl.pos_offset,
                         wl.weight_dtype, wl.mode, layout)
     if layout == "tiled":
-        # the weights are fixed: repacked once, as a serving process does at load
+        # the weights are fixed: repacked once, as a serving process does at
+        # load; the row-major copy is released
         W = P.pack_head(cfg, W)
         torch.cuda.synchronize()
+        torch.cuda.empty_cache()
     path = P.PATH_AUTO if args.path == "auto" else P.PATH_STAGEWISE
     P.pctree_set_path(path)
     fused = P.uses_fused_round(cfg, path)
